@@ -1,0 +1,44 @@
+"""Plant one mistake at a time in a copy of the oracle (on the CPU) and check that
+the pins in test_oracle_pins.py catch it.  This shows the pins constrain every
+part of the oracle the parity tests rely on."""
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "kf_oracle.c")
+
+MUTATIONS = {
+    "bias_sign": ("case ORC_BIAS: return v + orc_load", "case ORC_BIAS: return v - orc_load"),
+    "gelu_cubic": ("0.044715 * v * v * v", "0.04715 * v * v * v"),
+    "gemm_k_index": ("orc_load(jb->W, jb->wt, j * jb->ldw + k)",
+                     "orc_load(jb->W, jb->wt, j * jb->ldw + (jb->K - 1 - k))"),
+    "gn_unbiased_var": ("    var /= (double)gs;", "    var /= (double)(gs > 1 ? gs - 1 : 1);"),
+    "gn_no_eps": ("sqrt(var + op->eps)", "sqrt(var)"),
+    "lse_drop_max": ("return m + log(acc);", "return log(acc);"),
+    "route_tie_upper": ("l[e] > l[best]", "l[e] >= l[best]"),
+    "route_unstable": ("  for (int64_t p = 0; p < P; ++p) {\n    int32_t e = topk_ids[p];",
+                       "  for (int64_t p = P - 1; p >= 0; --p) {\n    int32_t e = topk_ids[p];"),
+    "swiglu_swap": ("s[j] = g * orc_sigmoid(g) * u;", "s[j] = u * orc_sigmoid(u) * g;"),
+    "moe_drop_weight": ("y[c] += wt * acc;", "y[c] += acc;"),
+    "bf16_round_bits": ("ldexp(1.0, e - 8)", "ldexp(1.0, e - 9)"),
+    "scale_ignored": ("case ORC_SCALE: return v * op->scalar;", "case ORC_SCALE: return v;"),
+    "residual_dropped": ("case ORC_RESIDUAL_ADD: return v + orc_load", "case ORC_RESIDUAL_ADD: return v + 0 * orc_load"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    old, new = MUTATIONS[name]
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor for {name} not unique/found"
+    mpath = tmp_path / "kf_oracle.c"
+    mpath.write_text(src.replace(old, new))
+    env = dict(os.environ, KF_ORACLE_SRC=str(mpath), KF_ORACLE_BUILD=str(tmp_path / "_build"))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
+    assert "failed" in r.stdout, r.stdout[-2000:]

@@ -1,0 +1,340 @@
+"""Pins of the fp64 oracle against facts that do not come from the oracle itself:
+closed forms, library routines for special cases, exact rational brute force and
+invariants.  Each test is chosen so that a plausible slip in the oracle (a dropped
+term, a wrong sign, a swapped index, a transposed operand) fails at least one."""
+import math
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+import torch.nn.functional as F
+
+import oracle
+
+pytestmark = pytest.mark.filterwarnings("ignore")
+
+
+def bf16(a):
+    return torch.as_tensor(a, dtype=torch.float32).to(torch.bfloat16)
+
+
+def f64(t):
+    return t.to(torch.float64).numpy()
+
+
+# --------------------------------------------------------------------- GEMM core
+def test_gemm_identity_gives_transposed_rows():
+    g = torch.Generator().manual_seed(1)
+    K, N = 24, 40
+    W = bf16(torch.randint(-4, 5, (N, K), generator=g).float())
+    X = bf16(torch.eye(K))
+    Y = oracle.fused_gemm(X, W, [])
+    assert np.array_equal(Y, f64(W).T)
+
+
+def test_gemm_rank1_closed_form():
+    g = torch.Generator().manual_seed(2)
+    M, N, K = 7, 11, 33
+    u = torch.randint(-3, 4, (M, 1), generator=g).float()
+    a = torch.randint(-3, 4, (1, K), generator=g).float()
+    v = torch.randint(-3, 4, (N, 1), generator=g).float()
+    c = torch.randint(-3, 4, (1, K), generator=g).float()
+    X, W = bf16(u @ a), bf16(v @ c)
+    Y = oracle.fused_gemm(X, W, [])
+    ref = (u.double() @ v.double().T) * float((a.double() * c.double()).sum())
+    assert np.array_equal(Y, ref.numpy())
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 1, 1), (2, 3, 5), (6, 4, 6), (5, 6, 3)])
+def test_gemm_bruteforce_fractions(M, N, K):
+    g = torch.Generator().manual_seed(M * 100 + N * 10 + K)
+    X = bf16(torch.randn(M, K, generator=g) * 3)
+    W = bf16(torch.randn(N, K, generator=g) * 3)
+    xs = [[Fraction(float(v)) for v in row] for row in X.float().tolist()]
+    ws = [[Fraction(float(v)) for v in row] for row in W.float().tolist()]
+    Y = oracle.fused_gemm(X, W, [])
+    for i in range(M):
+        for j in range(N):
+            exact = sum(xs[i][k] * ws[j][k] for k in range(K))
+            assert abs(Fraction(Y[i, j]) - exact) <= abs(exact) * Fraction(1, 2**50) + Fraction(1, 2**200)
+
+
+def test_gemm_fp32_operands_and_row_subset():
+    g = torch.Generator().manual_seed(3)
+    X = torch.rand(9, 17, generator=g) * 2 - 1
+    W = torch.rand(5, 17, generator=g) * 2 - 1
+    Y = oracle.fused_gemm(X, W, [])
+    ref = X.double().numpy() @ W.double().numpy().T
+    assert np.allclose(Y, ref, rtol=1e-14, atol=1e-14)
+    Ys = oracle.fused_gemm(X, W, [], rows=[8, 0, 3])
+    assert np.array_equal(Ys, Y[[8, 0, 3]])
+
+
+# ------------------------------------------------------ elementwise tail ops
+def _through_identity(vals, chain, extra=None):
+    """Make s = vals exactly: X = I, W = vals^T (vals must be bf16-exact)."""
+    vals = bf16(vals)
+    M, N = vals.shape
+    X = bf16(torch.eye(M))
+    W = vals.T.contiguous()
+    return oracle.fused_gemm(X, W, chain), f64(vals)
+
+
+def _grid(M=8, N=64, lo=-6, hi=6):
+    return torch.linspace(lo, hi, M * N).reshape(M, N)
+
+
+@pytest.mark.parametrize("kind,fn", [
+    ("gelu_tanh", lambda t: F.gelu(t, approximate="tanh")),
+    ("silu", F.silu),
+    ("sigmoid", torch.sigmoid),
+    ("relu", F.relu),
+    ("mish", F.mish),
+])
+def test_activation_matches_library_fp64(kind, fn):
+    Y, s = _through_identity(_grid(), [(kind, {})])
+    ref = fn(torch.from_numpy(s)).numpy()
+    assert np.allclose(Y, ref, rtol=1e-14, atol=1e-15)
+
+
+def test_leaky_relu_slope():
+    Y, s = _through_identity(_grid(), [("leaky_relu", {"scalar": 0.2})])
+    assert np.allclose(Y, F.leaky_relu(torch.from_numpy(s), 0.2).numpy(), rtol=0, atol=0)
+
+
+def test_gelu_odd_part_identity_and_limits():
+    Y, s = _through_identity(_grid(4, 32, -9, 9), [("gelu_tanh", {})])
+    Yn, _ = _through_identity(-_grid(4, 32, -9, 9), [("gelu_tanh", {})])
+    assert np.allclose(Y - Yn, s, atol=1e-13)          # gelu(x) - gelu(-x) = x
+    Y0, _ = _through_identity(torch.zeros(2, 8), [("gelu_tanh", {})])
+    assert np.all(Y0 == 0)
+    Yb, sb = _through_identity(torch.full((1, 8), 40.0), [("gelu_tanh", {})])
+    assert np.allclose(Yb, sb, rtol=1e-15)             # -> x for large x
+
+
+def test_sigmoid_silu_symmetries():
+    Y, s = _through_identity(_grid(), [("sigmoid", {})])
+    Yn, _ = _through_identity(-_grid(), [("sigmoid", {})])
+    assert np.allclose(Y + Yn, 1.0, atol=1e-15)
+    S, _ = _through_identity(_grid(), [("silu", {})])
+    Sn, _ = _through_identity(-_grid(), [("silu", {})])
+    assert np.allclose(S - Sn, s, atol=1e-13)
+
+
+def test_bias_scale_residual_chain_order():
+    g = torch.Generator().manual_seed(4)
+    M, N, K = 6, 10, 12
+    X = bf16(torch.randint(-3, 4, (M, K), generator=g).float())
+    W = bf16(torch.randint(-3, 4, (N, K), generator=g).float())
+    b = bf16(torch.randint(-5, 6, (N,), generator=g).float())
+    R = bf16(torch.randint(-5, 6, (M, N), generator=g).float())
+    s = f64(X) @ f64(W).T
+    Y = oracle.fused_gemm(X, W, [("bias", {"p0": b}), ("scale", {"scalar": 2.0}),
+                                 ("residual_add", {"p0": R})])
+    assert np.array_equal(Y, (s + f64(b)[None, :]) * 2.0 + f64(R))
+    # a different order is a different function
+    Y2 = oracle.fused_gemm(X, W, [("scale", {"scalar": 2.0}), ("bias", {"p0": b}),
+                                  ("residual_add", {"p0": R})])
+    assert np.array_equal(Y2, s * 2.0 + f64(b)[None, :] + f64(R))
+    Ym = oracle.fused_gemm(X, W, [("mul", {"p0": b})])
+    assert np.array_equal(Ym, s * f64(b)[None, :])
+
+
+def test_residual_uses_true_row_under_subset():
+    g = torch.Generator().manual_seed(5)
+    X = bf16(torch.randn(8, 16, generator=g))
+    W = bf16(torch.randn(4, 16, generator=g))
+    R = bf16(torch.randn(8, 4, generator=g))
+    full = oracle.fused_gemm(X, W, [("residual_add", {"p0": R})])
+    sub = oracle.fused_gemm(X, W, [("residual_add", {"p0": R})], rows=[7, 2])
+    assert np.array_equal(sub, full[[7, 2]])
+
+
+# ------------------------------------------------------------- row logsumexp
+def test_row_lse_matches_scipy_and_bounds():
+    g = torch.Generator().manual_seed(6)
+    M, N, K = 5, 300, 64
+    X = bf16(torch.randn(M, K, generator=g))
+    W = bf16(torch.randn(N, K, generator=g))
+    Y = oracle.fused_gemm(X, W, [("scale", {"scalar": 0.125}), ("row_logsumexp", {})])
+    S = 0.125 * (f64(X) @ f64(W).T)
+    ref = scipy.special.logsumexp(S, axis=1)
+    assert Y.shape == (M, 1)
+    assert np.allclose(Y[:, 0], ref, rtol=1e-14, atol=1e-13)
+    m = S.max(axis=1)
+    assert np.all(Y[:, 0] >= m) and np.all(Y[:, 0] <= m + math.log(N) + 1e-12)
+    assert np.allclose(np.exp(S - Y).sum(axis=1), 1.0, atol=1e-12)
+
+
+def test_row_lse_constant_row_and_shift():
+    c = 3.0
+    Y, _ = _through_identity(torch.full((3, 64), c), [("row_logsumexp", {})])
+    assert np.allclose(Y[:, 0], c + math.log(64), atol=1e-14)
+    base = torch.round(_grid(2, 64, -4, 4) * 8) / 8   # bf16-exact before and after +16
+    Y1, _ = _through_identity(base, [("row_logsumexp", {})])
+    Y2, _ = _through_identity(base + 16.0, [("row_logsumexp", {})])
+    assert np.allclose(Y2 - Y1, 16.0, atol=1e-12)
+    # huge offsets must not overflow (max subtraction)
+    Y3, _ = _through_identity(torch.full((1, 16), 1000.0), [("row_logsumexp", {})])
+    assert np.isfinite(Y3).all() and abs(Y3[0, 0] - (1000.0 + math.log(16))) < 1e-10
+
+
+# ----------------------------------------------------------------- GroupNorm
+def test_groupnorm_matches_torch_fp64():
+    g = torch.Generator().manual_seed(7)
+    M, N, K, G = 6, 96, 40, 4
+    X = bf16(torch.randn(M, K, generator=g))
+    W = bf16(torch.randn(N, K, generator=g))
+    b = bf16(torch.randn(N, generator=g))
+    gam = torch.rand(N, generator=g) + 0.5
+    bet = torch.rand(N, generator=g) * 0.2 - 0.1
+    chain = [("bias", {"p0": b}), ("groupnorm", {"groups": G, "eps": 1e-5, "p0": gam, "p1": bet}),
+             ("silu", {})]
+    Y = oracle.fused_gemm(X, W, chain)
+    Z = torch.from_numpy(f64(X) @ f64(W).T + f64(b)[None, :])
+    ref = F.silu(F.group_norm(Z, G, gam.double(), bet.double(), 1e-5)).numpy()
+    assert np.allclose(Y, ref, rtol=1e-12, atol=1e-13)
+
+
+def test_groupnorm_unit_affine_moments():
+    g = torch.Generator().manual_seed(8)
+    M, N, K, G, eps = 4, 64, 32, 2, 1e-5
+    X = bf16(torch.randn(M, K, generator=g) * 0.05)
+    W = bf16(torch.randn(N, K, generator=g) * 0.05)
+    Y = oracle.fused_gemm(X, W, [("groupnorm", {"groups": G, "eps": eps})])
+    Z = f64(X) @ f64(W).T
+    for gi in range(G):
+        sl = slice(gi * N // G, (gi + 1) * N // G)
+        var = Z[:, sl].var(axis=1)
+        assert np.allclose(Y[:, sl].mean(axis=1), 0.0, atol=1e-12)
+        assert np.allclose(Y[:, sl].var(axis=1), var / (var + eps), rtol=1e-10)
+    # constant group -> beta
+    bet = torch.linspace(-1, 1, 16)
+    Yc, _ = _through_identity(torch.full((2, 16), 5.0),
+                              [("groupnorm", {"groups": 2, "eps": eps, "p0": torch.ones(16), "p1": bet})])
+    assert np.allclose(Yc, bet.double().numpy()[None, :], atol=1e-12)
+
+
+# ------------------------------------------------------------------- routing
+def test_route_matches_torch_topk_and_softmax():
+    g = torch.Generator().manual_seed(9)
+    T, E, k = 50, 32, 4
+    logits = torch.randn(T, E, generator=g)
+    r = oracle.moe_route(logits, k)
+    v, idx = torch.topk(logits, k, dim=1)
+    assert np.array_equal(r["topk_ids"], idx.int().numpy())
+    ref_w = torch.softmax(v.double(), dim=1).numpy()
+    assert np.allclose(r["topk_w"], ref_w, rtol=1e-15, atol=1e-16)
+    assert np.allclose(r["topk_w"].sum(1), 1.0, atol=1e-15)
+    flat = r["topk_ids"].reshape(-1)
+    order = np.argsort(flat, kind="stable")
+    assert np.array_equal(r["sorted_pair"], order)
+    assert np.array_equal(r["sorted_token"], order // k)
+    assert np.array_equal(r["offsets"], np.concatenate([[0], np.cumsum(np.bincount(flat, minlength=E))]))
+    assert np.array_equal(r["sorted_w"], r["topk_w"].reshape(-1)[order])
+
+
+def test_route_ties_take_lower_index():
+    logits = torch.zeros(2, 8)
+    logits[0, 5] = 1.0
+    logits[1] = torch.tensor([0.0, 2.0, 2.0, 1.0, 2.0, 0.0, 1.0, 1.0])
+    r = oracle.moe_route(logits, 3)
+    assert r["topk_ids"][0].tolist() == [5, 0, 1]
+    assert r["topk_ids"][1].tolist() == [1, 2, 4]
+    assert np.allclose(r["topk_w"][1], 1 / 3, atol=1e-15)
+
+
+# ------------------------------------------------------------------ bf16 round
+def test_round_bf16_matches_torch_on_fp32_values():
+    g = torch.Generator().manual_seed(10)
+    x = torch.cat([torch.randn(4000, generator=g) * 10 ** torch.randint(-30, 30, (4000,), generator=g).float(),
+                   # exact ties between two bf16 neighbours
+                   (torch.arange(1, 200).float() * 2 + 1) * 2.0 ** -8 + 1.0 - 2.0 ** -8])
+    ref = x.to(torch.bfloat16).double().numpy()
+    got = np.array([oracle.round_bf16(float(v)) for v in x.tolist()])
+    assert np.array_equal(got, ref)
+
+
+# ------------------------------------------------------------------------ MoE
+def _moe_small(T=6, H=24, I=16, E=4, k=2, seed=11):
+    g = torch.Generator().manual_seed(seed)
+    X = bf16(torch.randn(T, H, generator=g))
+    Wgu = bf16(torch.randn(E, 2 * I, H, generator=g) * 0.2)
+    Wd = bf16(torch.randn(E, H, I, generator=g) * 0.2)
+    logits = torch.randn(T, E, generator=g)
+    return X, Wgu, Wd, logits
+
+
+def _ffn_numpy(x, wgu, wd, round_h):
+    I = wgu.shape[0] // 2
+    gt, up = wgu[:I] @ x, wgu[I:] @ x
+    h = gt / (1 + np.exp(-gt)) * up
+    if round_h:
+        h = torch.from_numpy(h).float().to(torch.bfloat16).double().numpy()
+    return wd @ h
+
+
+def test_moe_ffn_matches_numpy_definition():
+    X, Wgu, Wd, logits = _moe_small()
+    r = oracle.moe_route(logits, 2)
+    Y = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"], round_h=False)
+    x, wgu, wd = f64(X), f64(Wgu), f64(Wd)
+    for t in range(X.shape[0]):
+        ref = sum(r["topk_w"][t, j] * _ffn_numpy(x[t], wgu[r["topk_ids"][t, j]], wd[r["topk_ids"][t, j]], False)
+                  for j in range(2))
+        assert np.allclose(Y[t], ref, rtol=1e-12, atol=1e-13)
+    Yr = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"], round_h=True)
+    t = 3
+    ref = sum(r["topk_w"][t, j] * _ffn_numpy(x[t], wgu[r["topk_ids"][t, j]], wd[r["topk_ids"][t, j]], True)
+              for j in range(2))
+    assert np.allclose(Yr[t], ref, rtol=1e-9, atol=1e-9)
+    assert not np.allclose(Yr, Y, rtol=0, atol=0)  # the rounding point is live
+
+
+def test_moe_identical_experts_ignore_routing():
+    X, Wgu, Wd, logits = _moe_small(E=3, k=2)
+    Wgu = Wgu[:1].repeat(3, 1, 1)
+    Wd = Wd[:1].repeat(3, 1, 1)
+    r = oracle.moe_route(logits, 2)
+    Y = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"])
+    ids = np.zeros_like(r["topk_ids"])
+    Y0 = oracle.moe_ffn(X, Wgu, Wd, ids, r["topk_w"])
+    assert np.allclose(Y, Y0, rtol=1e-13, atol=1e-14)
+    dense = np.stack([_ffn_numpy(f64(X)[t], f64(Wgu)[0], f64(Wd)[0], True) for t in range(X.shape[0])])
+    assert np.allclose(Y, dense, rtol=1e-9, atol=1e-9)
+
+
+def test_grouped_gemm_composition_equals_moe_ffn():
+    X, Wgu, Wd, logits = _moe_small(T=9, E=4, k=2)
+    T, H = X.shape
+    I = Wgu.shape[1] // 2
+    r = oracle.moe_route(logits, 2)
+    h = oracle.grouped_gemm(X, Wgu, r["offsets"], I, [("swiglu", {})], row_index=r["sorted_token"])
+    # gate/up from numpy for one routed row
+    row = 5
+    e = int(np.searchsorted(r["offsets"], row, side="right") - 1)
+    x = f64(X)[r["sorted_token"][row]]
+    g = f64(Wgu)[e, :I] @ x
+    u = f64(Wgu)[e, I:] @ x
+    assert np.allclose(h[row], g / (1 + np.exp(-g)) * u, rtol=1e-12, atol=1e-13)
+    hb = torch.from_numpy(h).float().to(torch.bfloat16)
+    sw = torch.from_numpy(r["sorted_w"]).float()
+    st = torch.from_numpy(r["sorted_token"]).int()
+    Y = oracle.grouped_gemm(hb, Wd, r["offsets"], H,
+                            [("row_scale_scatter_add", {"p0": sw, "p1": st})], out_rows=T)
+    w32 = torch.from_numpy(r["topk_w"]).float().double().numpy()
+    Yref = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], w32)
+    assert np.allclose(Y, Yref, rtol=1e-5, atol=1e-5)
+
+
+def test_grouped_single_group_equals_dense():
+    g = torch.Generator().manual_seed(12)
+    X = bf16(torch.randn(7, 20, generator=g))
+    W = bf16(torch.randn(9, 20, generator=g))
+    b = bf16(torch.randn(9, generator=g))
+    chain = [("bias", {"p0": b}), ("gelu_tanh", {})]
+    dense = oracle.fused_gemm(X, W, chain)
+    grp = oracle.grouped_gemm(X, W[None], np.array([0, 7], np.int32), 9, chain)
+    assert np.array_equal(dense, grp)
