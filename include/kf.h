@@ -1,0 +1,197 @@
+/*
+ * kf.h -- C ABI of the GB300 (sm_103a) fused GEMM + tail-op library.
+ *
+ * The library computes the work that the KForge paper's generated kernels
+ * speed up (arXiv 2606.02963):
+ *   - a dense GEMM whose post-GEMM op chain (bias, activation, scale, residual,
+ *     row log-sum-exp, GroupNorm) runs in the GEMM's epilogue, reading the
+ *     matmul result once and writing once ("layer-wise fusion", Sec. IV-B),
+ *     with 16-bit operands and fp32 accumulation / post-processing
+ *     ("mixed-precision execution", Sec. IV-B);
+ *   - the routed MoE expert FFN of the gpt-oss decode path (Sec. IV-A): top-k
+ *     routing, a grouped gate/up GEMM with a SwiGLU epilogue, and a grouped down
+ *     GEMM whose epilogue applies the routing weight and scatter-adds rows into
+ *     the output (the "MoE finalize" step of Table 1).
+ *
+ * Conventions shared by every call
+ *   - Matrices are row-major.  X is [M x K], W is [N x K] (the nn.Linear layout,
+ *     so both GEMM operands are K-major) and Y = chain(X W^T) is [M x N].
+ *   - Every pointer except host-side descriptors (kf_epilogue and its op array)
+ *     is a DEVICE pointer on the current CUDA device.  The caller owns all of
+ *     them, including the workspace; query its size with the *_workspace call.
+ *     The library allocates and frees nothing and keeps no pointer after return.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Every call is
+ *     asynchronous on it; results are valid once the stream reaches that point.
+ *   - Arguments are checked on the host before anything is launched; a bad
+ *     argument returns a status and launches nothing.  A failed launch returns
+ *     KF_ERR_CUDA.  No call aborts, exits or throws.
+ *   - Device-side waits are bounded.  A kernel whose wait runs out (or that finds
+ *     bad device-resident routing data) records an error code in a per-device
+ *     error word and returns early; kf_get_device_error reads and clears it.
+ *   - Calls on distinct streams may run concurrently if they use distinct
+ *     workspaces and outputs.
+ */
+#ifndef KF_H_
+#define KF_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum kf_status {
+  KF_OK = 0,
+  KF_ERR_INVALID_ARG = 1,    /* null pointer, bad size, bad op chain            */
+  KF_ERR_UNSUPPORTED = 2,    /* dtype combination or chain this build lacks    */
+  KF_ERR_MISALIGNED = 3,     /* TMA needs 16-byte aligned bases and row strides */
+  KF_ERR_WORKSPACE = 4,      /* workspace missing or smaller than required     */
+  KF_ERR_CUDA = 5,           /* a CUDA runtime/driver call or launch failed    */
+  KF_ERR_DEVICE_TIMEOUT = 6, /* a device-side bounded wait ran out             */
+  KF_ERR_DEVICE_BOUNDS = 7   /* device-resident indices/offsets out of range   */
+} kf_status;
+
+typedef enum kf_dtype { KF_F32 = 0, KF_BF16 = 1, KF_I32 = 2 } kf_dtype;
+
+/* Tail ops, applied in list order to the fp32 accumulator (Sec. IV-B: the
+ * post-GEMM sequence of operations, fused into one kernel). */
+typedef enum kf_op_kind {
+  KF_OP_BIAS = 0,          /* v += p0[col]                           (p0: [N])        */
+  KF_OP_SCALE = 1,         /* v *= scalar                                              */
+  KF_OP_RELU = 2,          /* max(v, 0)                                                */
+  KF_OP_GELU_TANH = 3,     /* 0.5 v (1 + tanh(sqrt(2/pi)(v + 0.044715 v^3)))           */
+  KF_OP_SILU = 4,          /* v * sigmoid(v)  (Swish)                                  */
+  KF_OP_SIGMOID = 5,       /* 1 / (1 + exp(-v))                                        */
+  KF_OP_RESIDUAL_ADD = 6,  /* v += p0[row * ld + col]               (p0: [M x ld])    */
+  KF_OP_ROW_LOGSUMEXP = 7, /* row -> max_j v_j + log sum_j exp(v_j - max); Y is [M].
+                              Only scalar ops (SCALE, RELU, GELU_TANH, SILU, SIGMOID,
+                              MISH, LEAKY_RELU) may follow it.                        */
+  KF_OP_GROUPNORM = 8,     /* per row, `groups` contiguous column groups of N/groups:
+                              (v - mean) / sqrt(biased var + eps) * p0[col] + p1[col];
+                              p0 (gamma) / p1 (beta) may be NULL (1 / 0).  Group size
+                              must be a multiple of 32 and at most 512.              */
+  KF_OP_SWIGLU = 9,        /* grouped GEMM only: B holds 2N rows per group (gate rows
+                              0..N-1, then up rows N..2N-1); C = silu(gate) * up      */
+  KF_OP_ROW_SCALE_SCATTER_ADD = 10, /* grouped GEMM only, last op: C[p1[r], :] +=
+                              p0[r] * v  with p0 fp32 [rows_total] (row scale) and
+                              p1 int32 [rows_total] (destination row); `ld` = rows of
+                              C (a destination outside [0, ld) is skipped and sets
+                              KF_ERR_DEVICE_BOUNDS); C is fp32 and must be
+                              initialised by the caller (atomic adds, so the order
+                              of the fp32 additions is not fixed).                     */
+  KF_OP_MISH = 11,         /* v * tanh(log(1 + exp(v)))                                */
+  KF_OP_LEAKY_RELU = 12,   /* v > 0 ? v : scalar * v                                   */
+  KF_OP_MUL = 13           /* v *= p0[col]                          (p0: [N])        */
+} kf_op_kind;
+
+typedef struct kf_epilogue_op {
+  int32_t kind;       /* kf_op_kind                                          */
+  float scalar;       /* SCALE factor, LEAKY_RELU slope                      */
+  float eps;          /* GROUPNORM epsilon                                   */
+  int32_t groups;     /* GROUPNORM group count                               */
+  const void* p0;     /* op operand (device pointer), see kf_op_kind         */
+  const void* p1;     /* second operand (GROUPNORM beta, scatter rows)       */
+  int32_t p_dtype;    /* kf_dtype of p0 (and of p1 for GROUPNORM)            */
+  int64_t ld;         /* leading dimension of a matrix operand (RESIDUAL_ADD);
+                         destination row count (ROW_SCALE_SCATTER_ADD)        */
+} kf_epilogue_op;
+
+typedef struct kf_epilogue {
+  int32_t num_ops;    /* 0..8 */
+  const kf_epilogue_op* ops;
+} kf_epilogue;
+
+/*
+ * kf_fused_gemm -- Y = chain(X W^T)                    (Sec. IV-B, Table 3)
+ *
+ *   X [M x K] (row stride ldx), W [N x K] (row stride ldw), Y [M x N] (row
+ *   stride ldy), or Y [M] (fp32 or bf16) when the chain holds ROW_LOGSUMEXP.
+ *   Operand dtypes: both KF_BF16 (tcgen05 tensor-core path, fp32 accumulation
+ *   in tensor memory; Y bf16 or fp32), or both KF_F32 (exact fp32 FFMA path; Y
+ *   fp32; element-wise chains only).
+ *   bf16 path: X, W must be 16-byte aligned with ldx, ldw multiples of 8, else
+ *   KF_ERR_MISALIGNED.  M == 0 or N == 0 is a no-op; K must be >= 1.
+ *   workspace: kf_fused_gemm_workspace() bytes (0 unless the chain holds a row
+ *   log-sum-exp, which keeps per-tile row partials there).
+ *   Y must not alias X or W; a RESIDUAL_ADD operand may alias Y (in place).
+ */
+kf_status kf_fused_gemm(const void* X, int32_t x_dtype, int64_t ldx, const void* W, int32_t w_dtype,
+                        int64_t ldw, void* Y, int32_t y_dtype, int64_t ldy, int64_t M, int64_t N, int64_t K,
+                        const kf_epilogue* epi, void* workspace, size_t workspace_bytes, void* stream);
+size_t kf_fused_gemm_workspace(int64_t M, int64_t N, int64_t K, const kf_epilogue* epi);
+
+/*
+ * kf_moe_route -- top-k routing of T tokens over E experts  (Sec. IV-A, decode path)
+ *
+ *   logits fp32 [T x E].  For each token the k experts with the largest logits
+ *   (ties -> lower expert index), in descending order, go to topk_ids int32
+ *   [T x k]; topk_w fp32 [T x k] is the softmax over those k logits (sums to 1).
+ *   The T*k (token, slot) pairs are then sorted by expert with a stable
+ *   counting sort (pair p = t*k + slot keeps increasing p within an expert):
+ *   expert_offsets int32 [E + 1] (offsets[e]..offsets[e+1] are expert e's rows),
+ *   sorted_token int32 [T*k] (token of each sorted row), sorted_w fp32 [T*k]
+ *   (its routing weight).  1 <= k <= E <= 256.  T == 0 writes offsets only.
+ */
+kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int32_t* topk_ids, float* topk_w,
+                       int32_t* expert_offsets, int32_t* sorted_token, float* sorted_w, void* stream);
+
+/*
+ * kf_grouped_gemm -- per-group C rows = chain(A rows B[g]^T)  (Sec. IV-A, MoE experts)
+ *
+ *   Row group g owns rows r in [group_offsets[g], group_offsets[g+1]) of the
+ *   rows_total output rows; group_offsets is a DEVICE int32 array [G + 1]
+ *   (non-decreasing, ending at <= rows_total; read on the device, so routing
+ *   never needs a host sync).  Row r of the GEMM input is A[a_row_index[r]]
+ *   when a_row_index (device int32 [rows_total]) is given (gather; a_rows is
+ *   A's row count, for bounds), else A[r].  B[g] = B + g*b_group_stride
+ *   elements, rows of K with stride ldb: N rows, or 2N rows with SWIGLU.
+ *   C is [rows_total x N] (stride ldc), bf16 or fp32; with
+ *   ROW_SCALE_SCATTER_ADD C is the fp32 scatter target instead.
+ *   A, B bf16; alignment rules as kf_fused_gemm (also b_group_stride % 8 == 0).
+ *   workspace: kf_grouped_gemm_workspace() bytes (the gathered rows live there).
+ *   Bad device-side offsets/indices set KF_ERR_DEVICE_BOUNDS in the error word.
+ */
+kf_status kf_grouped_gemm(const void* A, int32_t a_dtype, int64_t lda, int64_t a_rows, const int32_t* a_row_index,
+                          const void* B, int32_t b_dtype, int64_t ldb, int64_t b_group_stride,
+                          const int32_t* group_offsets, int32_t G, int64_t rows_total, int64_t N, int64_t K,
+                          void* C, int32_t c_dtype, int64_t ldc, const kf_epilogue* epi, void* workspace,
+                          size_t workspace_bytes, void* stream);
+size_t kf_grouped_gemm_workspace(int64_t rows_total, int64_t N, int64_t K, int32_t G, int32_t gathered,
+                                 const kf_epilogue* epi);
+
+/*
+ * kf_moe_ffn -- routed MoE expert FFN, end to end           (Sec. IV-A, Table 1)
+ *
+ *   Y_t = sum_j topk_w[t,j] * W_down[e] (silu(W_gate[e] x_t) * (W_up[e] x_t)),
+ *   e = topk_ids[t,j], with the intermediate h rounded to bf16 (the down GEMM's
+ *   input dtype).  X bf16 [T x H]; logits fp32 [T x E]; W_gu bf16 [E x 2I x H]
+ *   (gate rows 0..I-1, up rows I..2I-1 per expert); W_down bf16 [E x H x I];
+ *   Y bf16 [T x H].  Runs kf_moe_route, the gathered gate/up grouped GEMM with
+ *   the SwiGLU epilogue, and the down grouped GEMM with the routing-weight
+ *   scale + scatter-add epilogue, then converts the fp32 sum to bf16.
+ *   H and I multiples of 8.  workspace: kf_moe_ffn_workspace() bytes.
+ *   If topk_ids_out / topk_w_out are non-NULL the routing is copied there.
+ */
+kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
+                     int64_t H, int64_t I, int32_t E, int32_t k, void* workspace, size_t workspace_bytes,
+                     int32_t* topk_ids_out, float* topk_w_out, void* stream);
+size_t kf_moe_ffn_workspace(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k);
+
+/* Synchronize `stream`, read and clear this device's error word.  Returns KF_OK,
+ * KF_ERR_DEVICE_TIMEOUT or KF_ERR_DEVICE_BOUNDS; *raw (if non-NULL) receives the
+ * raw bit set (1 = producer wait, 2 = MMA wait, 4 = epilogue wait, 8 = bounds). */
+kf_status kf_get_device_error(void* stream, uint32_t* raw);
+
+/* Wall-time limit of every device-side wait, in ns, for later launches
+ * (0 restores the default of 2 s).  A short limit makes a kernel give up early
+ * and report KF_ERR_DEVICE_TIMEOUT; used by the failure-detection test. */
+kf_status kf_set_wait_timeout_ns(uint64_t ns);
+
+const char* kf_status_string(int32_t status);
+int32_t kf_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KF_H_ */

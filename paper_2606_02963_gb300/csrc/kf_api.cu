@@ -1,0 +1,615 @@
+// kf_api.cu -- the C ABI declared in include/kf.h: host-side argument checks,
+// tail-chain planning, TMA tensor-map encoding and kernel dispatch.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cstring>
+#include <mutex>
+
+#include "kf_internal.h"
+#include "kf_tc_gemm.cuh"
+
+// Per-device error word written by the kernels' bounded waits / bounds checks.
+__device__ uint32_t g_kf_err;
+
+namespace kf {
+namespace {
+
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;  // 2 s
+std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
+
+struct DevInfo {
+  bool init = false;
+  int nsm = 0;
+  uint32_t* err = nullptr;
+};
+constexpr int kMaxDevices = 64;
+DevInfo g_dev[kMaxDevices];
+std::mutex g_mu;
+
+kf_status cuda_status(cudaError_t e) { return e == cudaSuccess ? KF_OK : KF_ERR_CUDA; }
+
+kf_status device_info(DevInfo* out) {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return KF_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DevInfo& di = g_dev[d];
+  if (!di.init) {
+    if (cudaDeviceGetAttribute(&di.nsm, cudaDevAttrMultiProcessorCount, d) != cudaSuccess) return KF_ERR_CUDA;
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_kf_err) != cudaSuccess) return KF_ERR_CUDA;
+    di.err = static_cast<uint32_t*>(p);
+    di.init = true;
+  }
+  *out = di;
+  return KF_OK;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// bf16 tensor map, 128-byte swizzle, box = 64 (K) x box_rows (x 1).  Rank 2
+// for A operands ([rows, K]); rank 3 for B operands ([groups, rows, K]), which
+// the kernel always loads with 3-D coordinates (groups = 1 for dense calls).
+kf_status make_map(CUtensorMap* m, const void* base, uint64_t k, uint64_t rows, uint64_t row_stride_bytes,
+                   uint64_t groups, uint64_t group_stride_bytes, uint32_t box_rows, cuuint32_t rank) {
+  auto fn = encode_fn();
+  if (!fn) return KF_ERR_CUDA;
+  std::memset(m, 0, sizeof(*m));
+  cuuint64_t dims[3] = {k, rows, groups};
+  cuuint64_t strides[2] = {row_stride_bytes, group_stride_bytes};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kBK), box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+int elt_size(int dt) { return dt == KF_BF16 ? 2 : 4; }
+bool float_dtype(int dt) { return dt == KF_F32 || dt == KF_BF16; }
+
+bool is_scalar_op(int k) {
+  return k == KF_OP_SCALE || k == KF_OP_RELU || k == KF_OP_GELU_TANH || k == KF_OP_SILU || k == KF_OP_SIGMOID ||
+         k == KF_OP_MISH || k == KF_OP_LEAKY_RELU;
+}
+bool is_pointwise_op(int k) {
+  return is_scalar_op(k) || k == KF_OP_BIAS || k == KF_OP_MUL || k == KF_OP_RESIDUAL_ADD;
+}
+
+struct ChainPlan {
+  int mode = kModeStore;
+  int n_pre = 0, n_post = 0;
+  DevOp pre[kMaxOps];
+  DevOp post[kMaxOps];
+  DevOp norm;
+  int gs = 0;
+  const float* row_scale = nullptr;
+  const int32_t* row_dst = nullptr;
+  int64_t dst_rows = 0;
+};
+
+kf_status to_devop(const kf_epilogue_op& o, int64_t N, DevOp* d) {
+  std::memset(d, 0, sizeof(*d));
+  d->kind = o.kind;
+  d->scalar = o.scalar;
+  d->eps = o.eps;
+  d->p0 = o.p0;
+  d->p1 = o.p1;
+  d->p_dtype = o.p_dtype;
+  d->ld = o.ld;
+  switch (o.kind) {
+    case KF_OP_BIAS:
+    case KF_OP_MUL:
+      if (!o.p0 || !float_dtype(o.p_dtype)) return KF_ERR_INVALID_ARG;
+      d->vec_ok = aligned16(o.p0);
+      return KF_OK;
+    case KF_OP_RESIDUAL_ADD:
+      if (!o.p0 || !float_dtype(o.p_dtype) || o.ld < N) return KF_ERR_INVALID_ARG;
+      d->vec_ok = aligned16(o.p0) && (o.ld * elt_size(o.p_dtype)) % 16 == 0;
+      return KF_OK;
+    default:
+      return is_scalar_op(o.kind) ? KF_OK : KF_ERR_INVALID_ARG;
+  }
+}
+
+kf_status plan_chain(const kf_epilogue* epi, int64_t N, bool grouped, ChainPlan* pl) {
+  const int n = epi ? epi->num_ops : 0;
+  if (n < 0 || n > kMaxOps || (n > 0 && !epi->ops)) return KF_ERR_INVALID_ARG;
+  int special = -1;
+  for (int i = 0; i < n; ++i) {
+    const int k = epi->ops[i].kind;
+    if (k == KF_OP_ROW_LOGSUMEXP || k == KF_OP_GROUPNORM || k == KF_OP_SWIGLU || k == KF_OP_ROW_SCALE_SCATTER_ADD) {
+      if (special >= 0) return KF_ERR_UNSUPPORTED;  // one reduction / special op per chain
+      special = i;
+    } else if (!is_pointwise_op(k)) {
+      return KF_ERR_INVALID_ARG;
+    }
+  }
+  const int sk = special >= 0 ? epi->ops[special].kind : -1;
+  if (!grouped && (sk == KF_OP_SWIGLU || sk == KF_OP_ROW_SCALE_SCATTER_ADD)) return KF_ERR_INVALID_ARG;
+  if (grouped && (sk == KF_OP_ROW_LOGSUMEXP || sk == KF_OP_GROUPNORM)) return KF_ERR_UNSUPPORTED;
+  const int split = special >= 0 ? special : n;
+  pl->n_pre = split;
+  pl->n_post = special >= 0 ? n - special - 1 : 0;
+  for (int i = 0; i < split; ++i) {
+    kf_status st = to_devop(epi->ops[i], N, &pl->pre[i]);
+    if (st != KF_OK) return st;
+  }
+  for (int i = 0; i < pl->n_post; ++i) {
+    const kf_epilogue_op& o = epi->ops[special + 1 + i];
+    if (sk == KF_OP_ROW_LOGSUMEXP && !is_scalar_op(o.kind)) return KF_ERR_INVALID_ARG;
+    kf_status st = to_devop(o, N, &pl->post[i]);
+    if (st != KF_OK) return st;
+  }
+  switch (sk) {
+    case -1: pl->mode = kModeStore; break;
+    case KF_OP_ROW_LOGSUMEXP: pl->mode = kModeLse; break;
+    case KF_OP_SWIGLU:
+      pl->mode = kModeSwiglu;
+      if (pl->n_pre != 0) return KF_ERR_UNSUPPORTED;  // SwiGLU acts on the raw gate/up accumulators
+      break;
+    case KF_OP_ROW_SCALE_SCATTER_ADD: {
+      const kf_epilogue_op& o = epi->ops[special];
+      if (pl->n_post != 0) return KF_ERR_INVALID_ARG;  // must be last
+      if (!o.p0 || !o.p1 || o.ld <= 0) return KF_ERR_INVALID_ARG;
+      pl->mode = kModeScatter;
+      pl->row_scale = static_cast<const float*>(o.p0);
+      pl->row_dst = static_cast<const int32_t*>(o.p1);
+      pl->dst_rows = o.ld;
+    } break;
+    case KF_OP_GROUPNORM: {
+      const kf_epilogue_op& o = epi->ops[special];
+      if (o.groups < 1 || N % o.groups != 0) return KF_ERR_INVALID_ARG;
+      if ((o.p0 || o.p1) && !float_dtype(o.p_dtype)) return KF_ERR_INVALID_ARG;
+      if (!(o.eps >= 0.0f)) return KF_ERR_INVALID_ARG;
+      const int64_t gs = N / o.groups;
+      if (gs % 32 != 0 || !(256 % gs == 0 || gs == 512)) return KF_ERR_UNSUPPORTED;
+      pl->mode = kModeGroupNorm;
+      pl->gs = static_cast<int>(gs);
+      std::memset(&pl->norm, 0, sizeof(pl->norm));
+      pl->norm.kind = KF_OP_GROUPNORM;
+      pl->norm.eps = o.eps;
+      pl->norm.groups = static_cast<int32_t>(gs);
+      pl->norm.p0 = o.p0;
+      pl->norm.p1 = o.p1;
+      pl->norm.p_dtype = o.p_dtype;
+      pl->norm.vec_ok = (!o.p0 || aligned16(o.p0)) && (!o.p1 || aligned16(o.p1));
+    } break;
+    default: return KF_ERR_INVALID_ARG;
+  }
+  return KF_OK;
+}
+
+void fill_params_common(TcParams& p, const ChainPlan& pl, uint32_t* err) {
+  p.n_pre = pl.n_pre;
+  p.n_post = pl.n_post;
+  for (int i = 0; i < pl.n_pre; ++i) p.pre[i] = pl.pre[i];
+  for (int i = 0; i < pl.n_post; ++i) p.post[i] = pl.post[i];
+  p.norm = pl.norm;
+  p.err = err;
+  p.wait_ns = g_wait_ns.load();
+  p.drain_ns = std::max<uint64_t>(p.wait_ns, 1000000000ull);
+}
+
+// Tile width for the dense store / LSE variants: the fewest tiles per CTA of
+// the persistent grid, weighted by the tile width (+ a fixed per-tile cost).
+int pick_dense_bn(int mode, int64_t M, int64_t N, int nsm) {
+  static const int cand[] = {256, 224, 192, 128};
+  int best = 0;
+  int64_t best_cost = INT64_MAX;
+  const int64_t tm = (M + kBM - 1) / kBM;
+  for (int bn : cand) {
+    if (!tc_dense_has(mode, bn)) continue;
+    const int64_t tiles = tm * ((N + bn - 1) / bn);
+    const int64_t per_cta = (tiles + nsm - 1) / nsm;
+    const int64_t cost = per_cta * (bn + 48);
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
+}
+
+// Output-column tile for the grouped variants: the widest compiled tile that
+// divides N, else the one wasting the fewest columns.
+int pick_grouped_outn(int mode, int64_t N) {
+  static const int cand[] = {256, 192, 128};
+  int best = 0;
+  int64_t best_waste = INT64_MAX;
+  for (int bn : cand) {
+    if (!tc_grouped_has(mode, bn)) continue;
+    const int outn = mode == kModeSwiglu ? bn / 2 : bn;
+    const int64_t waste = ((N + outn - 1) / outn) * outn - N;
+    if (waste < best_waste) {
+      best_waste = waste;
+      best = bn;
+    }
+  }
+  return best;
+}
+
+// rows of one B box: the whole tile, or each of the gate / up halves for SwiGLU
+uint32_t mode_box(int mode, int bn) { return mode == kModeSwiglu ? bn / 2 : bn; }
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+size_t lse_ws_bytes(int64_t M, int64_t N) {
+  // upper bound over all tile widths (narrowest tile = most partials per row)
+  return align_up(static_cast<size_t>(M) * static_cast<size_t>((N + 127) / 128) * sizeof(float2), 256);
+}
+
+// -------------------------------------------------------------- grouped core
+struct GroupedArgs {
+  const void* A;
+  int64_t lda;
+  int64_t a_rows;
+  const int32_t* a_row_index;
+  const void* B;
+  int64_t ldb;
+  int64_t b_group_stride;
+  const int32_t* offsets;
+  int32_t G;
+  int64_t rows_total, N, K;
+  void* C;
+  int32_t c_dtype;
+  int64_t ldc;
+};
+
+size_t grouped_ws_bytes(int64_t rows_total, int64_t K, bool gathered) {
+  return gathered ? align_up(static_cast<size_t>(rows_total) * static_cast<size_t>(K) * 2, 256) : 0;
+}
+
+kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cudaStream_t s, const DevInfo& di) {
+  const void* A = g.A;
+  int64_t lda = g.lda;
+  if (g.a_row_index) {
+    kf_status st = cuda_status(gather_rows_launch(g.A, g.lda, g.a_rows, g.a_row_index, g.rows_total, g.K, ws, di.err, s));
+    if (st != KF_OK) return st;
+    A = ws;
+    lda = g.K;
+  }
+  const int bn = pick_grouped_outn(pl.mode, g.N);
+  if (bn == 0) return KF_ERR_UNSUPPORTED;
+  const int outn = pl.mode == kModeSwiglu ? bn / 2 : bn;
+  const int64_t nb = pl.mode == kModeSwiglu ? 2 * g.N : g.N;
+  CUtensorMap ma, mb;
+  kf_status st = make_map(&ma, A, g.K, g.rows_total, lda * 2, 1, 0, kBM, 2);
+  if (st != KF_OK) return st;
+  st = make_map(&mb, g.B, g.K, nb, g.ldb * 2, g.G, g.b_group_stride * 2, mode_box(pl.mode, bn), 3);
+  if (st != KF_OK) return st;
+  TcParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.M = static_cast<int32_t>(g.rows_total);
+  p.N = static_cast<int32_t>(g.N);
+  p.K = static_cast<int32_t>(g.K);
+  p.tiles_n = static_cast<int32_t>((g.N + outn - 1) / outn);
+  p.num_kb = static_cast<int32_t>((g.K + kBK - 1) / kBK);
+  p.G = g.G;
+  p.group_offsets = g.offsets;
+  p.b_rows = static_cast<int32_t>(g.N);
+  p.C = g.C;
+  p.ldc = g.ldc;
+  p.c_dtype = g.c_dtype;
+  p.c_vec_ok = aligned16(g.C) && (g.ldc * elt_size(g.c_dtype)) % 16 == 0;
+  p.row_scale = pl.row_scale;
+  p.row_dst = pl.row_dst;
+  p.dst_rows = static_cast<int32_t>(pl.dst_rows);
+  fill_params_common(p, pl, di.err);
+  const int64_t ub = ((g.rows_total + kBM - 1) / kBM + g.G) * p.tiles_n;
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
+  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, p, grid, s));
+}
+
+}  // namespace
+}  // namespace kf
+
+using namespace kf;
+
+extern "C" {
+
+const char* kf_status_string(int32_t s) {
+  switch (s) {
+    case KF_OK: return "ok";
+    case KF_ERR_INVALID_ARG: return "invalid argument";
+    case KF_ERR_UNSUPPORTED: return "unsupported dtype combination or op chain";
+    case KF_ERR_MISALIGNED: return "misaligned pointer or stride (TMA needs 16-byte alignment)";
+    case KF_ERR_WORKSPACE: return "workspace missing or too small";
+    case KF_ERR_CUDA: return "CUDA error";
+    case KF_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+    case KF_ERR_DEVICE_BOUNDS: return "device-resident index or offset out of range";
+    default: return "unknown status";
+  }
+}
+
+int32_t kf_abi_version(void) { return 1; }
+
+kf_status kf_set_wait_timeout_ns(uint64_t ns) {
+  g_wait_ns.store(ns == 0 ? kDefaultWaitNs : ns);
+  return KF_OK;
+}
+
+kf_status kf_get_device_error(void* stream, uint32_t* raw) {
+  DevInfo di;
+  kf_status st = device_info(&di);
+  if (st != KF_OK) return st;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return KF_ERR_CUDA;
+  uint32_t v = 0, z = 0;
+  if (cudaMemcpy(&v, di.err, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return KF_ERR_CUDA;
+  if (v && cudaMemcpy(di.err, &z, sizeof(z), cudaMemcpyHostToDevice) != cudaSuccess) return KF_ERR_CUDA;
+  if (raw) *raw = v;
+  if (v & (kErrWaitProducer | kErrWaitMma | kErrWaitEpilogue)) return KF_ERR_DEVICE_TIMEOUT;
+  if (v & kErrBounds) return KF_ERR_DEVICE_BOUNDS;
+  return KF_OK;
+}
+
+size_t kf_fused_gemm_workspace(int64_t M, int64_t N, int64_t K, const kf_epilogue* epi) {
+  (void)K;
+  if (!epi || M <= 0 || N <= 0) return 0;
+  for (int i = 0; i < epi->num_ops && epi->ops; ++i)
+    if (epi->ops[i].kind == KF_OP_ROW_LOGSUMEXP) return lse_ws_bytes(M, N);
+  return 0;
+}
+
+kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt, int64_t ldw, void* Y,
+                        int32_t yt, int64_t ldy, int64_t M, int64_t N, int64_t K, const kf_epilogue* epi,
+                        void* workspace, size_t ws_bytes, void* stream) {
+  if (M < 0 || N < 0 || K < 1) return KF_ERR_INVALID_ARG;
+  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return KF_ERR_INVALID_ARG;
+  if (M == 0 || N == 0) return KF_OK;  // empty problem: nothing to read or write
+  if (!X || !W || !Y) return KF_ERR_INVALID_ARG;
+  if (ldx < K || ldw < K) return KF_ERR_INVALID_ARG;
+  if (!float_dtype(xt) || !float_dtype(wt) || !float_dtype(yt)) return KF_ERR_INVALID_ARG;
+  ChainPlan pl;
+  kf_status st = plan_chain(epi, N, false, &pl);
+  if (st != KF_OK) return st;
+  if (pl.mode != kModeLse && ldy < N) return KF_ERR_INVALID_ARG;
+  const bool f32_path = xt == KF_F32 && wt == KF_F32;
+  if (f32_path) {
+    // exact fp32 FFMA path: element-wise chains only
+    if (pl.mode != kModeStore || yt != KF_F32) return KF_ERR_UNSUPPORTED;
+  } else {
+    if (xt != KF_BF16 || wt != KF_BF16) return KF_ERR_UNSUPPORTED;
+    if (!aligned16(X) || !aligned16(W) || ldx % 8 != 0 || ldw % 8 != 0) return KF_ERR_MISALIGNED;
+    if (pl.mode == kModeLse &&
+        (!workspace || !aligned16(workspace) || ws_bytes < lse_ws_bytes(M, N)))
+      return KF_ERR_WORKSPACE;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DevInfo di;
+  st = device_info(&di);
+  if (st != KF_OK) return st;
+
+  if (f32_path) {
+    SimtParams sp;
+    std::memset(&sp, 0, sizeof(sp));
+    sp.X = static_cast<const float*>(X);
+    sp.W = static_cast<const float*>(W);
+    sp.Y = static_cast<float*>(Y);
+    sp.ldx = ldx;
+    sp.ldw = ldw;
+    sp.ldy = ldy;
+    sp.M = static_cast<int32_t>(M);
+    sp.N = static_cast<int32_t>(N);
+    sp.K = static_cast<int32_t>(K);
+    sp.n_ops = pl.n_pre;
+    for (int i = 0; i < pl.n_pre; ++i) sp.ops[i] = pl.pre[i];
+    return cuda_status(simt_gemm_f32_launch(sp, s));
+  }
+
+  int bn = 0, sub = 1;
+  int64_t tiles_n = 0;
+  if (pl.mode == kModeGroupNorm) {
+    bn = 256;
+    sub = pl.gs == 512 ? 2 : 1;
+    tiles_n = (N + bn * sub - 1) / (bn * sub);
+  } else {
+    bn = pick_dense_bn(pl.mode, M, N, di.nsm);
+    if (bn == 0) return KF_ERR_UNSUPPORTED;
+    tiles_n = (N + bn - 1) / bn;
+  }
+  CUtensorMap ma, mb;
+  st = make_map(&ma, X, K, M, ldx * 2, 1, 0, kBM, 2);
+  if (st != KF_OK) return st;
+  st = make_map(&mb, W, K, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, bn, 3);
+  if (st != KF_OK) return st;
+  TcParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.M = static_cast<int32_t>(M);
+  p.N = static_cast<int32_t>(N);
+  p.K = static_cast<int32_t>(K);
+  p.tiles_m = static_cast<int32_t>((M + kBM - 1) / kBM);
+  p.tiles_n = static_cast<int32_t>(tiles_n);
+  p.num_kb = static_cast<int32_t>((K + kBK - 1) / kBK);
+  p.total_units = p.tiles_m * p.tiles_n;
+  p.C = Y;
+  p.ldc = ldy;
+  p.c_dtype = yt;
+  p.c_vec_ok = aligned16(Y) && (ldy * elt_size(yt)) % 16 == 0;
+  if (pl.mode == kModeLse) p.lse_part = static_cast<float2*>(workspace);
+  fill_params_common(p, pl, di.err);
+  const int grid = std::min(p.total_units, di.nsm);
+  st = cuda_status(tc_dense_launch(pl.mode, bn, ma, mb, p, sub, grid, s));
+  if (st != KF_OK || pl.mode != kModeLse) return st;
+  LseCombineParams cp;
+  std::memset(&cp, 0, sizeof(cp));
+  cp.part = p.lse_part;
+  cp.M = p.M;
+  cp.parts = p.tiles_n;
+  cp.out = Y;
+  cp.out_dtype = yt;
+  cp.n_post = pl.n_post;
+  for (int i = 0; i < pl.n_post; ++i) cp.post[i] = pl.post[i];
+  return cuda_status(lse_combine_launch(cp, s));
+}
+
+kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int32_t* topk_ids, float* topk_w,
+                       int32_t* offsets, int32_t* sorted_token, float* sorted_w, void* stream) {
+  if (T < 0 || E < 1 || E > 256 || k < 1 || k > E) return KF_ERR_INVALID_ARG;
+  if (T * k > INT32_MAX) return KF_ERR_INVALID_ARG;
+  if (!offsets || (T > 0 && (!logits || !topk_ids || !topk_w || !sorted_token || !sorted_w)))
+    return KF_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  kf_status st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, topk_ids, topk_w, s));
+  if (st != KF_OK) return st;
+  return cuda_status(route_sort_launch(topk_ids, topk_w, static_cast<int32_t>(T), E, k, offsets, sorted_token,
+                                       sorted_w, s));
+}
+
+size_t kf_grouped_gemm_workspace(int64_t rows_total, int64_t N, int64_t K, int32_t G, int32_t gathered,
+                                 const kf_epilogue* epi) {
+  (void)N;
+  (void)G;
+  (void)epi;
+  if (rows_total <= 0 || K <= 0) return 0;
+  return grouped_ws_bytes(rows_total, K, gathered != 0);
+}
+
+kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows, const int32_t* a_row_index,
+                          const void* B, int32_t bt, int64_t ldb, int64_t b_group_stride, const int32_t* offsets,
+                          int32_t G, int64_t rows_total, int64_t N, int64_t K, void* C, int32_t ct, int64_t ldc,
+                          const kf_epilogue* epi, void* workspace, size_t ws_bytes, void* stream) {
+  if (rows_total < 0 || N < 1 || K < 1 || G < 1 || G > kMaxGroups) return KF_ERR_INVALID_ARG;
+  if (rows_total > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return KF_ERR_INVALID_ARG;
+  if (rows_total == 0) return KF_OK;  // no rows: nothing to read or write
+  if (!A || !B || !C || !offsets) return KF_ERR_INVALID_ARG;
+  if (lda < K || ldb < K || ldc < N || b_group_stride < 0) return KF_ERR_INVALID_ARG;
+  if (a_row_index && a_rows < 1) return KF_ERR_INVALID_ARG;
+  if (at != KF_BF16 || bt != KF_BF16) return KF_ERR_UNSUPPORTED;
+  if (!float_dtype(ct)) return KF_ERR_INVALID_ARG;
+  ChainPlan pl;
+  kf_status st = plan_chain(epi, N, true, &pl);
+  if (st != KF_OK) return st;
+  if (pl.mode == kModeScatter && ct != KF_F32) return KF_ERR_UNSUPPORTED;
+  const int64_t nb = pl.mode == kModeSwiglu ? 2 * N : N;
+  if (G > 1 && b_group_stride < nb * ldb) return KF_ERR_INVALID_ARG;
+  if (!aligned16(A) || !aligned16(B) || lda % 8 != 0 || ldb % 8 != 0 || b_group_stride % 8 != 0)
+    return KF_ERR_MISALIGNED;
+  if (a_row_index && K % 8 != 0) return KF_ERR_MISALIGNED;
+  if (a_row_index) {
+    if (!workspace || !aligned16(workspace) || ws_bytes < grouped_ws_bytes(rows_total, K, true))
+      return KF_ERR_WORKSPACE;
+  }
+  DevInfo di;
+  st = device_info(&di);
+  if (st != KF_OK) return st;
+  GroupedArgs g{A, lda, a_row_index ? a_rows : rows_total, a_row_index, B, ldb,
+                G > 1 ? b_group_stride : nb * ldb, offsets, G, rows_total, N, K, C, ct, ldc};
+  return grouped_core(g, pl, workspace, static_cast<cudaStream_t>(stream), di);
+}
+
+// Workspace layout of kf_moe_ffn (each region 256-byte aligned):
+//   topk_ids i32 [T k] | topk_w f32 [T k] | offsets i32 [E+1] | sorted_token i32 [T k]
+//   | sorted_w f32 [T k] | Xg bf16 [T k, H] | h bf16 [T k, I] | Yacc f32 [T, H]
+struct MoeLayout {
+  size_t ids, w, off, st, sw, xg, h, yacc, total;
+};
+static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k) {
+  MoeLayout L;
+  const size_t P = static_cast<size_t>(T) * static_cast<size_t>(k);
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align_up(o + bytes, 256);
+    return at;
+  };
+  L.ids = take(P * 4);
+  L.w = take(P * 4);
+  L.off = take(static_cast<size_t>(E + 1) * 4);
+  L.st = take(P * 4);
+  L.sw = take(P * 4);
+  L.xg = take(P * static_cast<size_t>(H) * 2);
+  L.h = take(P * static_cast<size_t>(I) * 2);
+  L.yacc = take(static_cast<size_t>(T) * static_cast<size_t>(H) * 4);
+  L.total = o;
+  return L;
+}
+
+size_t kf_moe_ffn_workspace(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k) {
+  if (T < 0 || H < 1 || I < 1 || E < 1 || k < 1) return 0;
+  return moe_layout(T, H, I, E, k).total;
+}
+
+kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
+                     int64_t H, int64_t I, int32_t E, int32_t k, void* workspace, size_t ws_bytes,
+                     int32_t* topk_ids_out, float* topk_w_out, void* stream) {
+  if (T < 0 || H < 1 || I < 1 || E < 1 || E > 256 || k < 1 || k > E) return KF_ERR_INVALID_ARG;
+  if (T * k > INT32_MAX || H > INT32_MAX || I > INT32_MAX) return KF_ERR_INVALID_ARG;
+  if (!X || !logits || !W_gu || !W_down || !Y) return KF_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(W_gu) || !aligned16(W_down) || !aligned16(Y) || H % 8 != 0 || I % 8 != 0)
+    return KF_ERR_MISALIGNED;
+  if (T == 0) return KF_OK;
+  const MoeLayout L = moe_layout(T, H, I, E, k);
+  if (!workspace || !aligned16(workspace) || ws_bytes < L.total) return KF_ERR_WORKSPACE;
+  DevInfo di;
+  kf_status st = device_info(&di);
+  if (st != KF_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  auto* ids = reinterpret_cast<int32_t*>(ws + L.ids);
+  auto* w = reinterpret_cast<float*>(ws + L.w);
+  auto* off = reinterpret_cast<int32_t*>(ws + L.off);
+  auto* stok = reinterpret_cast<int32_t*>(ws + L.st);
+  auto* sw = reinterpret_cast<float*>(ws + L.sw);
+  void* xg = ws + L.xg;
+  void* h = ws + L.h;
+  auto* yacc = reinterpret_cast<float*>(ws + L.yacc);
+  const int64_t P = T * k;
+
+  st = kf_moe_route(logits, T, E, k, ids, w, off, stok, sw, stream);
+  if (st != KF_OK) return st;
+  // gate/up: h = silu(Xg W_gate[e]^T) * (Xg W_up[e]^T), rows gathered by token
+  {
+    kf_epilogue_op op{};
+    op.kind = KF_OP_SWIGLU;
+    kf_epilogue epi{1, &op};
+    ChainPlan pl;
+    st = plan_chain(&epi, I, true, &pl);
+    if (st != KF_OK) return st;
+    GroupedArgs g{X, H, T, stok, W_gu, H, 2 * I * H, off, E, P, I, H, h, KF_BF16, I};
+    st = grouped_core(g, pl, xg, s, di);
+    if (st != KF_OK) return st;
+  }
+  // down: Yacc[token] += w * (h W_down[e]^T)
+  if (cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
+  {
+    kf_epilogue_op op{};
+    op.kind = KF_OP_ROW_SCALE_SCATTER_ADD;
+    op.p0 = sw;
+    op.p1 = stok;
+    op.p_dtype = KF_F32;
+    op.ld = T;
+    kf_epilogue epi{1, &op};
+    ChainPlan pl;
+    st = plan_chain(&epi, H, true, &pl);
+    if (st != KF_OK) return st;
+    GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yacc, KF_F32, H};
+    st = grouped_core(g, pl, nullptr, s, di);
+    if (st != KF_OK) return st;
+  }
+  st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s));
+  if (st != KF_OK) return st;
+  if (topk_ids_out &&
+      cudaMemcpyAsync(topk_ids_out, ids, static_cast<size_t>(P) * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return KF_ERR_CUDA;
+  if (topk_w_out &&
+      cudaMemcpyAsync(topk_w_out, w, static_cast<size_t>(P) * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return KF_ERR_CUDA;
+  return KF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,238 @@
+// kf_common.cuh -- device-side structures shared by the kernels: the decoded
+// epilogue op list, the tcgen05 GEMM parameter block, and the register-level
+// tail-op interpreter that applies the chain to 32 accumulator columns of one
+// row (Sec. IV-B: the post-GEMM op chain is applied to the matmul result while it
+// is still on chip, in fp32).
+#pragma once
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "../../include/kf.h"
+
+namespace kf {
+
+constexpr int kMaxOps = 8;
+constexpr int kMaxGroups = 1024;  // grouped GEMM: row groups (experts)
+
+// error-word bits
+constexpr uint32_t kErrWaitProducer = 1u;
+constexpr uint32_t kErrWaitMma = 2u;
+constexpr uint32_t kErrWaitEpilogue = 4u;
+constexpr uint32_t kErrBounds = 8u;
+
+struct DevOp {
+  int32_t kind;
+  float scalar;
+  float eps;
+  int32_t groups;   // GROUPNORM: group size in columns (not the count)
+  const void* p0;
+  const void* p1;
+  int32_t p_dtype;
+  int32_t vec_ok;   // p0 (and p1) allow 16-byte vector access for 32-column chunks
+  int64_t ld;
+};
+
+// Modes of the tcgen05 GEMM kernel (what its epilogue does with a tile).
+enum TcMode : int {
+  kModeStore = 0,    // chain of element-wise ops -> store C tile
+  kModeLse = 1,      // element-wise pre-ops -> per-tile row (max, sum exp) partials
+  kModeGroupNorm = 2,// pre-ops -> GroupNorm -> post-ops -> store
+  kModeSwiglu = 3,   // gate/up halves -> silu(g) * u -> post-ops -> store
+  kModeScatter = 4,  // chain -> * row scale -> atomic add into C[dst row]
+};
+
+struct TcParams {
+  int32_t M;            // dense: rows of X;  grouped: rows_total
+  int32_t N;            // output columns
+  int32_t K;
+  int32_t tiles_m;      // dense only
+  int32_t tiles_n;      // output-column tiles (units for GroupNorm)
+  int32_t num_kb;       // K blocks of 64
+  int32_t total_units;  // dense: number of work units (tiles or GN units)
+  int32_t G;            // grouped: number of groups (0 = dense)
+  const int32_t* group_offsets;
+  int32_t b_rows;       // grouped: rows of B per group used for the N offset of up rows (= N)
+  int32_t n_pre;        // ops applied before the reduction / norm / store
+  int32_t n_post;       // ops applied after it
+  DevOp pre[kMaxOps];
+  DevOp post[kMaxOps];
+  DevOp norm;           // GROUPNORM op (group size in .groups)
+  void* C;
+  int64_t ldc;
+  int32_t c_dtype;
+  int32_t c_vec_ok;
+  float2* lse_part;     // [M x tiles_n] (max, sum exp) partials
+  const float* row_scale;   // scatter
+  const int32_t* row_dst;   // scatter
+  int32_t dst_rows;         // scatter: rows of C (bounds)
+  uint32_t* err;
+  uint64_t wait_ns;
+  uint64_t drain_ns;
+};
+
+// ---------------------------------------------------------------- loads/stores
+__device__ __forceinline__ float ld_elem(const void* p, int dt, int64_t i) {
+  if (dt == KF_BF16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(p)[i]);
+  return reinterpret_cast<const float*>(p)[i];
+}
+
+// Load 32 consecutive elements starting at element index i0 (first `nvalid`
+// are in bounds; the rest read as 0).  Vector path when the whole chunk is in
+// bounds and the caller guaranteed 16-byte alignment.
+__device__ __forceinline__ void ld32(const void* p, int dt, int64_t i0, int nvalid, bool vec_ok, float (&o)[32]) {
+  if (nvalid >= 32 && vec_ok) {
+    if (dt == KF_BF16) {
+      const uint4* q = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p) + i0);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        uint4 u = __ldg(q + v);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          o[v * 8 + 2 * h] = __uint_as_float(w[h] << 16);
+          o[v * 8 + 2 * h + 1] = __uint_as_float(w[h] & 0xFFFF0000u);
+        }
+      }
+    } else {
+      const float4* q = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(p) + i0);
+#pragma unroll
+      for (int v = 0; v < 8; ++v) {
+        float4 f = __ldg(q + v);
+        o[4 * v] = f.x;
+        o[4 * v + 1] = f.y;
+        o[4 * v + 2] = f.z;
+        o[4 * v + 3] = f.w;
+      }
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) o[j] = (j < nvalid) ? ld_elem(p, dt, i0 + j) : 0.0f;
+  }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ void st32(void* p, int dt, int64_t i0, int nvalid, bool vec_ok, const float (&v)[32]) {
+  if (nvalid >= 32 && vec_ok) {
+    if (dt == KF_BF16) {
+      uint4* q = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p) + i0);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint4 u;
+        u.x = pack_bf16x2(v[8 * c + 0], v[8 * c + 1]);
+        u.y = pack_bf16x2(v[8 * c + 2], v[8 * c + 3]);
+        u.z = pack_bf16x2(v[8 * c + 4], v[8 * c + 5]);
+        u.w = pack_bf16x2(v[8 * c + 6], v[8 * c + 7]);
+        q[c] = u;
+      }
+    } else {
+      float4* q = reinterpret_cast<float4*>(reinterpret_cast<float*>(p) + i0);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) q[c] = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+    }
+  } else {
+    if (dt == KF_BF16) {
+      __nv_bfloat16* q = reinterpret_cast<__nv_bfloat16*>(p) + i0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nvalid) q[j] = __float2bfloat16_rn(v[j]);
+    } else {
+      float* q = reinterpret_cast<float*>(p) + i0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nvalid) q[j] = v[j];
+    }
+  }
+}
+
+// ------------------------------------------------------------ element-wise ops
+__device__ __forceinline__ float f_sigmoid(float x) { return 1.0f / (1.0f + expf(-x)); }
+__device__ __forceinline__ float f_gelu_tanh(float x) {
+  const float c = 0.7978845608028654f;  // sqrt(2/pi)
+  return 0.5f * x * (1.0f + tanhf(c * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ float f_mish(float x) {
+  float sp = x > 20.0f ? x : log1pf(expf(x));
+  return x * tanhf(sp);
+}
+
+__device__ __forceinline__ float apply_scalar_op(const DevOp& op, float x) {
+  switch (op.kind) {
+    case KF_OP_SCALE: return x * op.scalar;
+    case KF_OP_RELU: return fmaxf(x, 0.0f);
+    case KF_OP_GELU_TANH: return f_gelu_tanh(x);
+    case KF_OP_SILU: return x * f_sigmoid(x);
+    case KF_OP_SIGMOID: return f_sigmoid(x);
+    case KF_OP_MISH: return f_mish(x);
+    case KF_OP_LEAKY_RELU: return x > 0.0f ? x : op.scalar * x;
+    default: return x;
+  }
+}
+
+// Apply ops[0..n) to the 32 values of row `row` starting at column col0 (the
+// first `nvalid` columns exist).  Operands of rows that do not exist are not
+// read (row_ok == false).
+__device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
+                                              int nvalid, bool row_ok) {
+  for (int o = 0; o < n; ++o) {
+    const DevOp& op = ops[o];
+    switch (op.kind) {
+      case KF_OP_BIAS:
+      case KF_OP_MUL: {
+        float b[32];
+        ld32(op.p0, op.p_dtype, col0, nvalid, op.vec_ok != 0, b);
+        if (op.kind == KF_OP_BIAS) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] += b[j];
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] *= b[j];
+        }
+      } break;
+      case KF_OP_RESIDUAL_ADD: {
+        if (row_ok) {
+          float r[32];
+          ld32(op.p0, op.p_dtype, row * op.ld + col0, nvalid, op.vec_ok != 0, r);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] += r[j];
+        }
+      } break;
+      case KF_OP_SCALE: {
+        const float s = op.scalar;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] *= s;
+      } break;
+      case KF_OP_RELU: {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.0f);
+      } break;
+      case KF_OP_GELU_TANH: {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = f_gelu_tanh(v[j]);
+      } break;
+      case KF_OP_SILU: {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = v[j] * f_sigmoid(v[j]);
+      } break;
+      case KF_OP_SIGMOID: {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = f_sigmoid(v[j]);
+      } break;
+      case KF_OP_MISH: {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = f_mish(v[j]);
+      } break;
+      case KF_OP_LEAKY_RELU: {
+        const float s = op.scalar;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = v[j] > 0.0f ? v[j] : s * v[j];
+      } break;
+      default: break;
+    }
+  }
+}
+
+}  // namespace kf

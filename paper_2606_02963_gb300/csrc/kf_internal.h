@@ -1,0 +1,52 @@
+// kf_internal.h -- host-side declarations shared by the library's translation
+// units (kernel launchers); not part of the public ABI.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "kf_common.cuh"
+
+namespace kf {
+
+// Tensor-core GEMM launchers.  `bn` selects the tile width among the compiled
+// variants; returns cudaErrorInvalidValue for a variant that is not built.
+bool tc_dense_has(int mode, int bn);
+bool tc_grouped_has(int mode, int bn);
+int tc_dense_smem(int mode, int bn);
+cudaError_t tc_dense_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+                            int sub_tiles, int grid, cudaStream_t s);
+cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+                              int grid, cudaStream_t s);
+
+// SIMT kernels.
+struct SimtParams {
+  const float* X;
+  const float* W;
+  float* Y;
+  int64_t ldx, ldw, ldy;
+  int32_t M, N, K;
+  int32_t n_ops;
+  DevOp ops[kMaxOps];
+};
+cudaError_t simt_gemm_f32_launch(const SimtParams& p, cudaStream_t s);
+
+struct LseCombineParams {
+  const float2* part;
+  int32_t M;
+  int32_t parts;
+  void* out;
+  int32_t out_dtype;
+  int32_t n_post;
+  DevOp post[kMaxOps];
+};
+cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s);
+
+cudaError_t route_topk_launch(const float* logits, int32_t T, int32_t E, int32_t k, int32_t* ids, float* w,
+                              cudaStream_t s);
+cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
+                              int32_t* offsets, int32_t* sorted_token, float* sorted_w, cudaStream_t s);
+cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
+                               int64_t K, void* out, uint32_t* err, cudaStream_t s);
+cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s);
+
+}  // namespace kf

@@ -1,0 +1,304 @@
+// kf_simt.cu -- CUDA-core kernels of the path:
+//   * exact fp32 FFMA GEMM + element-wise chain (fp32 operands; no TF32, since a
+//     silent downcast is exactly what the paper's candidate guardrails ban, Sec. III-D),
+//   * cross-tile combine of the row log-sum-exp partials (Sec. IV-B, online LSE),
+//   * MoE routing: per-token top-k + softmax, then a deterministic stable
+//     counting sort of the (token, slot) pairs by expert (Sec. IV-A, gpt-oss),
+//   * row gather of routed tokens, fp32 -> bf16 conversion of the MoE output.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "kf_internal.h"
+
+namespace kf {
+
+// Scalar form of the chain for one element (fp32 path).
+__device__ __forceinline__ float apply_chain1(const DevOp* ops, int n, float v, int64_t row, int64_t col) {
+  for (int o = 0; o < n; ++o) {
+    const DevOp& op = ops[o];
+    switch (op.kind) {
+      case KF_OP_BIAS: v += ld_elem(op.p0, op.p_dtype, col); break;
+      case KF_OP_MUL: v *= ld_elem(op.p0, op.p_dtype, col); break;
+      case KF_OP_RESIDUAL_ADD: v += ld_elem(op.p0, op.p_dtype, row * op.ld + col); break;
+      default: v = apply_scalar_op(op, v); break;
+    }
+  }
+  return v;
+}
+
+// ------------------------------------------------------------------ fp32 GEMM
+// 32x32 output tile per 256-thread block, 2x2 outputs per thread, K in steps
+// of 32 through shared memory (both operands K-contiguous in global memory).
+constexpr int kSB = 32;
+__global__ void __launch_bounds__(256) simt_gemm_f32_kernel(const __grid_constant__ SimtParams p) {
+  __shared__ float xs[kSB][kSB + 1];  // [k][m]
+  __shared__ float ws[kSB][kSB + 1];  // [k][n]
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  const int m0 = blockIdx.y * kSB, n0 = blockIdx.x * kSB;
+  float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+  for (int k0 = 0; k0 < p.K; k0 += kSB) {
+    for (int i = threadIdx.x; i < kSB * kSB; i += 256) {
+      const int r = i / kSB, c = i % kSB;  // c runs along K: coalesced
+      const int gm = m0 + r, gn = n0 + r, gk = k0 + c;
+      xs[c][r] = (gm < p.M && gk < p.K) ? p.X[static_cast<int64_t>(gm) * p.ldx + gk] : 0.f;
+      ws[c][r] = (gn < p.N && gk < p.K) ? p.W[static_cast<int64_t>(gn) * p.ldw + gk] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int k = 0; k < kSB; ++k) {
+      const float a0 = xs[k][ty * 2], a1 = xs[k][ty * 2 + 1];
+      const float b0 = ws[k][tx * 2], b1 = ws[k][tx * 2 + 1];
+      acc[0][0] = fmaf(a0, b0, acc[0][0]);
+      acc[0][1] = fmaf(a0, b1, acc[0][1]);
+      acc[1][0] = fmaf(a1, b0, acc[1][0]);
+      acc[1][1] = fmaf(a1, b1, acc[1][1]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int gm = m0 + ty * 2 + i, gn = n0 + tx * 2 + j;
+      if (gm < p.M && gn < p.N)
+        p.Y[static_cast<int64_t>(gm) * p.ldy + gn] = apply_chain1(p.ops, p.n_ops, acc[i][j], gm, gn);
+    }
+}
+
+cudaError_t simt_gemm_f32_launch(const SimtParams& p, cudaStream_t s) {
+  dim3 grid((p.N + kSB - 1) / kSB, (p.M + kSB - 1) / kSB);
+  simt_gemm_f32_kernel<<<grid, 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------- row log-sum-exp combine
+// (m, s) (+) (m', s') = (M, s e^{m-M} + s' e^{m'-M}),  out = M + log S.
+__global__ void lse_combine_kernel(const __grid_constant__ LseCombineParams p) {
+  const int warps = blockDim.x >> 5;
+  const int row = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= p.M) return;
+  const float2* part = p.part + static_cast<int64_t>(row) * p.parts;
+  float m = -INFINITY, s = 0.f;
+  for (int i = lane; i < p.parts; i += 32) {
+    const float2 q = part[i];
+    const float nm = fmaxf(m, q.x);
+    if (nm != -INFINITY) {
+      s = (m == -INFINITY ? 0.f : s * expf(m - nm)) + (q.x == -INFINITY ? 0.f : q.y * expf(q.x - nm));
+      m = nm;
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, m, off);
+    const float os = __shfl_xor_sync(0xffffffffu, s, off);
+    const float nm = fmaxf(m, om);
+    if (nm != -INFINITY) {
+      s = (m == -INFINITY ? 0.f : s * expf(m - nm)) + (om == -INFINITY ? 0.f : os * expf(om - nm));
+      m = nm;
+    }
+  }
+  if (lane == 0) {
+    float v = (m == -INFINITY) ? -INFINITY : m + logf(s);
+    for (int o = 0; o < p.n_post; ++o) v = apply_scalar_op(p.post[o], v);
+    if (p.out_dtype == KF_BF16)
+      reinterpret_cast<__nv_bfloat16*>(p.out)[row] = __float2bfloat16_rn(v);
+    else
+      reinterpret_cast<float*>(p.out)[row] = v;
+  }
+}
+
+cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s) {
+  const int warps = 8;
+  lse_combine_kernel<<<(p.M + warps - 1) / warps, warps * 32, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------- routing
+// One warp per token; expert e lives in lane e % 32, slot e / 32 (E <= 256).
+// Selection order: larger logit first, ties -> lower expert index.
+constexpr int kMaxExperts = 256;
+__global__ void route_topk_kernel(const float* __restrict__ logits, int32_t T, int32_t E, int32_t k,
+                                  int32_t* __restrict__ ids, float* __restrict__ w) {
+  const int warps = blockDim.x >> 5;
+  const int t = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (t >= T) return;
+  float val[kMaxExperts / 32];
+  uint32_t taken = 0;
+#pragma unroll
+  for (int i = 0; i < kMaxExperts / 32; ++i) {
+    const int e = i * 32 + lane;
+    val[i] = e < E ? logits[static_cast<int64_t>(t) * E + e] : -INFINITY;
+    if (e >= E) taken |= 1u << i;
+  }
+  float sel_v = 0.f, vmax = 0.f, den = 0.f;
+  int sel_e = 0;
+  for (int j = 0; j < k; ++j) {
+    float bv = -INFINITY;
+    int be = 0x7fffffff;
+#pragma unroll
+    for (int i = 0; i < kMaxExperts / 32; ++i) {
+      const int e = i * 32 + lane;
+      if (!(taken >> i & 1u) && (val[i] > bv || (val[i] == bv && e < be))) {
+        bv = val[i];
+        be = e;
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+      const int oe = __shfl_xor_sync(0xffffffffu, be, off);
+      if (ov > bv || (ov == bv && oe < be)) {
+        bv = ov;
+        be = oe;
+      }
+    }
+    if ((be & 31) == lane) taken |= 1u << (be >> 5);
+    if (j == 0) vmax = bv;
+    const float ex = expf(bv - vmax);
+    den += ex;
+    if (lane == j) {  // lane j keeps slot j (k <= 32 handled below)
+      sel_v = ex;
+      sel_e = be;
+    }
+    if (k > 32 && lane == 0) {
+      ids[static_cast<int64_t>(t) * k + j] = be;
+      w[static_cast<int64_t>(t) * k + j] = ex;  // normalised in a second pass below
+    }
+  }
+  if (k <= 32) {
+    if (lane < k) {
+      ids[static_cast<int64_t>(t) * k + lane] = sel_e;
+      w[static_cast<int64_t>(t) * k + lane] = sel_v / den;
+    }
+  } else if (lane == 0) {
+    for (int j = 0; j < k; ++j) w[static_cast<int64_t>(t) * k + j] /= den;
+  }
+}
+
+cudaError_t route_topk_launch(const float* logits, int32_t T, int32_t E, int32_t k, int32_t* ids, float* w,
+                              cudaStream_t s) {
+  if (T == 0) return cudaSuccess;
+  const int warps = 8;
+  route_topk_kernel<<<(T + warps - 1) / warps, warps * 32, 0, s>>>(logits, T, E, k, ids, w);
+  return cudaGetLastError();
+}
+
+// Stable counting sort of P = T*k pairs by expert, one 1024-thread block.
+// Warp w owns the contiguous pair range [w*chunk, (w+1)*chunk); counts per
+// (warp, expert), scanned expert-major then warp-minor, give each warp's first
+// slot per expert; a second in-order walk ranks equal experts within each
+// 32-pair batch with __match_any_sync.  Output order = increasing pair index
+// within each expert (bit-identical to a sequential stable sort).
+constexpr int kSortWarps = 32;
+__global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32_t* __restrict__ ids,
+                                                                     const float* __restrict__ w, int32_t P,
+                                                                     int32_t E, int32_t k, int32_t* offsets,
+                                                                     int32_t* sorted_token, float* sorted_w) {
+  extern __shared__ int32_t cnt[];  // [kSortWarps][E]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < kSortWarps * E; i += blockDim.x) cnt[i] = 0;
+  __syncthreads();
+  const int32_t chunk = (P + kSortWarps - 1) / kSortWarps;
+  const int32_t beg = min(P, warp * chunk), end = min(P, beg + chunk);
+  for (int32_t p = beg + lane; p < end; p += 32) atomicAdd(&cnt[warp * E + ids[p]], 1);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int32_t run = 0;
+    for (int e = 0; e < E; ++e) {
+      offsets[e] = run;
+      for (int ww = 0; ww < kSortWarps; ++ww) {
+        const int32_t c = cnt[ww * E + e];
+        cnt[ww * E + e] = run;  // becomes the first slot of (warp ww, expert e)
+        run += c;
+      }
+    }
+    offsets[E] = run;
+  }
+  __syncthreads();
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  for (int32_t b = beg; b < end; b += 32) {
+    const int32_t p = b + lane;
+    const bool valid = p < end;
+    const int32_t e = valid ? ids[p] : E + lane;  // invalid lanes never match a real expert
+    const uint32_t peers = __match_any_sync(0xffffffffu, e);
+    const int rank = __popc(peers & lt_mask);
+    if (valid) {
+      const int32_t pos = cnt[warp * E + e] + rank;
+      sorted_token[pos] = p / k;
+      sorted_w[pos] = w[p];
+    }
+    __syncwarp();
+    if (valid && rank == 0) cnt[warp * E + e] += __popc(peers);
+    __syncwarp();
+  }
+}
+
+cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
+                              int32_t* offsets, int32_t* sorted_token, float* sorted_w, cudaStream_t s) {
+  const int32_t P = T * k;
+  const size_t smem = sizeof(int32_t) * kSortWarps * E;
+  route_sort_kernel<<<1, kSortWarps * 32, smem, s>>>(ids, w, P, E, k, offsets, sorted_token, sorted_w);
+  return cudaGetLastError();
+}
+
+// ----------------------------------------------------------------- row gather
+// out[r, :] = A[idx[r], :] (16-byte vectors; K % 8 == 0 bf16).  An index out of
+// range writes a zero row and sets the bounds bit of the error word.
+__global__ void gather_rows_kernel(const uint4* __restrict__ A, int64_t lda_v, int64_t a_rows,
+                                   const int32_t* __restrict__ idx, int64_t rows, int64_t kv,
+                                   uint4* __restrict__ out, uint32_t* err) {
+  const int64_t total = rows * kv;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / kv, c = i % kv;
+    const int32_t src = idx[r];
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (src >= 0 && src < a_rows)
+      v = __ldg(A + src * lda_v + c);
+    else if (c == 0)
+      atomicOr(err, kErrBounds);
+    out[i] = v;
+  }
+}
+
+cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
+                               int64_t K, void* out, uint32_t* err, cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  const int64_t kv = K / 8, total = rows * kv;
+  int blocks = static_cast<int>(std::min<int64_t>((total + 255) / 256, 148 * 16));
+  gather_rows_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4*>(A), lda / 8, a_rows, idx, rows, kv,
+                                            reinterpret_cast<uint4*>(out), err);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ fp32 -> bf16
+__global__ void cvt_f32_bf16_kernel(const float4* __restrict__ in, uint2* __restrict__ out, int64_t n4) {
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n4;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const float4 f = in[i];
+    uint2 o;
+    o.x = pack_bf16x2(f.x, f.y);
+    o.y = pack_bf16x2(f.z, f.w);
+    out[i] = o;
+  }
+}
+__global__ void cvt_f32_bf16_tail_kernel(const float* in, __nv_bfloat16* out, int64_t beg, int64_t n) {
+  const int64_t i = beg + threadIdx.x;
+  if (i < n) out[i] = __float2bfloat16_rn(in[i]);
+}
+
+cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s) {
+  const int64_t n4 = n / 4;
+  if (n4 > 0) {
+    int blocks = static_cast<int>(std::min<int64_t>((n4 + 255) / 256, 148 * 8));
+    cvt_f32_bf16_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const float4*>(in), reinterpret_cast<uint2*>(out),
+                                               n4);
+  }
+  if (n % 4) cvt_f32_bf16_tail_kernel<<<1, 4, 0, s>>>(in, reinterpret_cast<__nv_bfloat16*>(out), n4 * 4, n);
+  return cudaGetLastError();
+}
+
+}  // namespace kf

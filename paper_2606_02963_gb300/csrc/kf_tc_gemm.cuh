@@ -1,0 +1,493 @@
+// kf_tc_gemm.cuh -- persistent, warp-specialised tcgen05 GEMM with the tail-op
+// chain fused into its epilogue (sm_103a).
+//
+// One CTA per SM, 6 warps:
+//   warp 0      TMA producer: streams 128x64 A tiles and BNx64 B tiles (bf16,
+//               128-byte swizzle) into a STAGES-deep shared-memory ring.
+//   warp 1      owns the tensor memory (alloc/dealloc) and, from one thread,
+//               issues tcgen05.mma (M=128, N=BN, K=16) into one of two TMEM
+//               accumulators; tcgen05.commit frees ring slots / publishes tiles.
+//   warps 2..5  epilogue: warp w reads TMEM lanes 32*(w%4).. (one output row per
+//               thread), applies the op chain in fp32 registers and writes the
+//               result once (Sec. IV-B: layer-wise fusion -- the matmul result is
+//               read once and the output written once; mixed precision -- bf16
+//               operands, fp32 accumulation and post-processing).
+// Row reductions run per thread over its row: the row log-sum-exp keeps an
+// online (max, sum exp) pair per tile and a second tiny kernel combines tiles
+// (Sec. IV-B: streaming online reduction); GroupNorm computes each group's
+// mean and variance from the accumulator in TMEM (exact two-pass per tile,
+// Chan's pairwise merge across the two 256-column halves of a 512-wide group).
+//
+// Every mbarrier wait is bounded (wall-time limit); a wait that runs out raises
+// a CTA-wide abort flag and an error bit, the producer waits (bounded) for its
+// in-flight TMA copies, the MMA thread for its in-flight MMAs, TMEM is freed and
+// the CTA returns.
+#pragma once
+#include "kf_common.cuh"
+#include "kf_ptx.cuh"
+
+namespace kf {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+constexpr int kABytes = kBM * kBK * 2;
+
+__host__ __device__ constexpr int pow2_at_least(int x) {
+  return x <= 32 ? 32 : x <= 64 ? 64 : x <= 128 ? 128 : x <= 256 ? 256 : 512;
+}
+
+template <int BN, int STAGES, int MODE, bool GROUPED>
+struct TcCfg {
+  static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN");
+  static constexpr int kOutN = (MODE == kModeSwiglu) ? BN / 2 : BN;  // output columns of a (sub)tile
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  // accumulator buffer b starts at TMEM column b * kAccStride
+  static constexpr int kAccStride = pow2_at_least(BN);
+  static constexpr int kTmemCols = 2 * kAccStride;
+  static constexpr int kBarBytes = 8 * (2 * STAGES + 5);
+  static constexpr int kMiscBytes = 64;
+  static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
+  static constexpr int kSmemUse = STAGES * kStageBytes + kBarBytes + kMiscBytes + kTableBytes;
+  // pad to > half of the SM's shared memory so that at most one such CTA is
+  // resident per SM (tensor-memory allocation then never has to wait)
+  static constexpr int kSmemBytes = 1024 + (kSmemUse > 120 * 1024 ? kSmemUse : 120 * 1024);
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN);
+  static_assert(kSmemBytes <= 232448, "shared memory");
+  static_assert(kBBytes % 1024 == 0, "B stage alignment");
+};
+
+struct UnitInfo {
+  int32_t m0, m_end, n0, g, n_blk;
+};
+
+template <int BN, int STAGES, int MODE, bool GROUPED>
+__global__ void __launch_bounds__(kThreads, 1)
+    kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const __grid_constant__ TcParams p, const int32_t sub_tiles) {
+  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* smA = sm;
+  uint8_t* smB = sm + STAGES * kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + STAGES * Cfg::kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* accf = bars + 2 * STAGES;
+  uint64_t* acce = bars + 2 * STAGES + 2;
+  uint64_t* drain = bars + 2 * STAGES + 4;
+  uint32_t* misc = reinterpret_cast<uint32_t*>(sm + STAGES * Cfg::kStageBytes + Cfg::kBarBytes);
+  uint32_t* tmem_slot = misc;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
+  int32_t* total_s = reinterpret_cast<int32_t*>(misc + 2);
+  volatile int* zero_flag = reinterpret_cast<volatile int*>(misc + 3);
+  int32_t* off_s = reinterpret_cast<int32_t*>(sm + STAGES * Cfg::kStageBytes + Cfg::kBarBytes + Cfg::kMiscBytes);
+  int32_t* ustart_s = off_s + (kMaxGroups + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&accf[a], 1);
+      mbar_init(&acce[a], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *zero_flag = 0;
+    *total_s = GROUPED ? 0 : p.total_units;
+    fence_mbarrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    __syncwarp();
+    tmem_alloc(tmem_slot, Cfg::kTmemCols);
+    tmem_relinquish();
+  }
+  if constexpr (GROUPED) {
+    if (threadIdx.x == 64) {
+      // Group table: validate the device-resident offsets and count work units
+      // (ceil(rows/128) row tiles x tiles_n column tiles per group).
+      bool ok = p.G >= 1 && p.G <= kMaxGroups;
+      int32_t units = 0;
+      int32_t prev = 0;
+      for (int g = 0; ok && g <= p.G; ++g) {
+        int32_t o = p.group_offsets[g];
+        if (o < prev || o > p.M) ok = false;
+        off_s[g] = o;
+        if (g > 0) {
+          ustart_s[g - 1] = units;
+          units += ((o - prev + kBM - 1) / kBM) * p.tiles_n;
+        }
+        prev = o;
+      }
+      if (!ok) {
+        atomicOr(p.err, kErrBounds);
+        units = 0;
+      }
+      if (ok) ustart_s[p.G] = units;
+      *total_s = units;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int32_t total = *total_s;
+
+  auto decode = [&](int32_t u) -> UnitInfo {
+    UnitInfo r;
+    if constexpr (GROUPED) {
+      int lo = 0, hi = p.G - 1;  // last g with ustart_s[g] <= u
+      while (lo < hi) {
+        int mid = (lo + hi + 1) >> 1;
+        if (ustart_s[mid] <= u) lo = mid; else hi = mid - 1;
+      }
+      // skip empty groups that share the same start
+      int g = lo;
+      while (g + 1 < p.G && ustart_s[g + 1] <= u) ++g;
+      const int32_t rows = off_s[g + 1] - off_s[g];
+      const int32_t tm = (rows + kBM - 1) / kBM;
+      const int32_t local = u - ustart_s[g];
+      const int32_t mb = local % tm;
+      r.n_blk = local / tm;
+      r.g = g;
+      r.m0 = off_s[g] + mb * kBM;
+      r.m_end = min(off_s[g + 1], r.m0 + kBM);
+      r.n0 = r.n_blk * Cfg::kOutN;
+    } else {
+      const int32_t mb = u % p.tiles_m;
+      r.n_blk = u / p.tiles_m;
+      r.g = 0;
+      r.m0 = mb * kBM;
+      r.m_end = min(p.M, r.m0 + kBM);
+      r.n0 = r.n_blk * Cfg::kOutN * sub_tiles;
+    }
+    return r;
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int32_t it = 0;
+      bool ok = true;
+      for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
+        const UnitInfo ui = decode(u);
+        for (int s = 0; ok && s < sub_tiles; ++s) {
+          const int32_t nb0 = ui.n0 + s * BN;
+          for (int32_t kb = 0; kb < p.num_kb; ++kb) {
+            const int st = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1;
+            if (!mbar_wait(&empty[st], ph ^ 1, abort_flag, p.wait_ns)) {
+              *abort_flag = 1;
+              atomicOr(p.err, kErrWaitProducer);
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[st], Cfg::kStageBytes);
+            tma_load_2d(smA + st * kABytes, &tmA, &full[st], kb * kBK, ui.m0);
+            uint8_t* b = smB + st * Cfg::kBBytes;
+            if constexpr (MODE == kModeSwiglu) {
+              tma_load_3d(b, &tmB, &full[st], kb * kBK, ui.n0, ui.g);
+              tma_load_3d(b + Cfg::kOutN * 128, &tmB, &full[st], kb * kBK, p.b_rows + ui.n0, ui.g);
+            } else {
+              tma_load_3d(b, &tmB, &full[st], kb * kBK, nb0, ui.g);
+            }
+            ++it;
+          }
+        }
+      }
+      if (!ok) {
+        // wait (bounded) for the copies still in flight before the CTA exits
+        for (int32_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
+          mbar_wait(&full[j % STAGES], (j / STAGES) & 1, zero_flag, p.drain_ns);
+      }
+    }
+  } else if (warp == 1) {
+    // ----------------------------------------------------------------- MMA
+    if (lane == 0) {
+      int32_t it = 0, tl = 0;
+      bool ok = true;
+      for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
+        for (int s = 0; ok && s < sub_tiles; ++s) {
+          const int acc = tl & 1;
+          if (!mbar_wait(&acce[acc], ((tl >> 1) & 1) ^ 1, abort_flag, p.wait_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + acc * Cfg::kAccStride;
+          for (int32_t kb = 0; kb < p.num_kb; ++kb) {
+            const int st = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1;
+            if (!mbar_wait(&full[st], ph, abort_flag, p.wait_ns)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a0 = smem_u32(smA + st * kABytes);
+            const uint32_t b0 = smem_u32(smB + st * Cfg::kBBytes);
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk) {
+              tc_mma_bf16(d, desc_sw128_kmajor(a0 + kk * 32), desc_sw128_kmajor(b0 + kk * 32), Cfg::kIdesc,
+                          (kb | kk) != 0 ? 1u : 0u);
+            }
+            tc_commit(&empty[st]);
+            ++it;
+          }
+          if (!ok) break;
+          tc_commit(&accf[acc]);
+          ++tl;
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(p.err, kErrWaitMma);
+        tc_commit(drain);  // arrives once every MMA issued so far has completed
+        mbar_wait(drain, 0, zero_flag, p.drain_ns);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int32_t row_in_tile = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    int32_t tl = 0;
+    bool ok = true;
+
+    auto wait_acc = [&](int32_t t) -> bool {
+      bool w = mbar_wait(&accf[t & 1], (t >> 1) & 1, abort_flag, p.wait_ns);
+      w = __all_sync(0xffffffffu, w);
+      if (!w) {
+        *abort_flag = 1;
+        if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+        return false;
+      }
+      tc_fence_after();
+      return true;
+    };
+    auto release_acc = [&](int32_t t) {
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acce[t & 1]);
+    };
+
+    for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
+      const UnitInfo ui = decode(u);
+      const int32_t grow = ui.m0 + row_in_tile;
+      const bool row_ok = grow < ui.m_end;
+
+      if constexpr (MODE == kModeStore || MODE == kModeSwiglu || MODE == kModeScatter) {
+        if (!wait_acc(tl)) { ok = false; break; }
+        const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
+        float rs = 0.0f;
+        int32_t dst = 0;
+        bool wr = row_ok;
+        if constexpr (MODE == kModeScatter) {
+          if (row_ok) {
+            rs = p.row_scale[grow];
+            dst = p.row_dst[grow];
+            if (dst < 0 || dst >= p.dst_rows) {
+              atomicOr(p.err, kErrBounds);
+              wr = false;
+            }
+          }
+        }
+        for (int c = 0; c < Cfg::kOutN / 32; ++c) {
+          const int32_t col0 = ui.n0 + c * 32;
+          const int nvalid = min(32, p.N - col0);
+          if (nvalid <= 0) break;  // uniform across the warp
+          __syncwarp();
+          float v[32];
+          if constexpr (MODE == kModeSwiglu) {
+            float gt[32];
+            tmem_ld32(tb + c * 32, gt);
+            tmem_ld32(tb + Cfg::kOutN + c * 32, v);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = gt[j] * f_sigmoid(gt[j]) * v[j];
+            apply_chain32(p.post, p.n_post, v, grow, col0, nvalid, row_ok);
+          } else {
+            tmem_ld32(tb + c * 32, v);
+            apply_chain32(p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+          }
+          if constexpr (MODE == kModeScatter) {
+            if (wr) {
+              float* dstp = reinterpret_cast<float*>(p.C) + static_cast<int64_t>(dst) * p.ldc + col0;
+              if (nvalid == 32 && p.c_vec_ok) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                  atomicAdd(reinterpret_cast<float4*>(dstp) + j,
+                            make_float4(v[4 * j] * rs, v[4 * j + 1] * rs, v[4 * j + 2] * rs, v[4 * j + 3] * rs));
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  if (j < nvalid) atomicAdd(dstp + j, v[j] * rs);
+              }
+            }
+          } else {
+            if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, nvalid, p.c_vec_ok != 0, v);
+          }
+        }
+        release_acc(tl);
+        ++tl;
+      } else if constexpr (MODE == kModeLse) {
+        if (!wait_acc(tl)) { ok = false; break; }
+        const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
+        float m = -INFINITY, s = 0.0f;
+        for (int c = 0; c < BN / 32; ++c) {
+          const int32_t col0 = ui.n0 + c * 32;
+          const int nvalid = min(32, p.N - col0);
+          if (nvalid <= 0) break;
+          __syncwarp();
+          float v[32];
+          tmem_ld32(tb + c * 32, v);
+          apply_chain32(p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+          float cm = -INFINITY;
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (j < nvalid) cm = fmaxf(cm, v[j]);
+          const float nm = fmaxf(m, cm);
+          float add = 0.0f;
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (j < nvalid) add += expf(v[j] - nm);
+          s = (m == -INFINITY ? 0.0f : s * expf(m - nm)) + add;
+          m = nm;
+        }
+        release_acc(tl);
+        ++tl;
+        if (row_ok) p.lse_part[static_cast<int64_t>(grow) * p.tiles_n + ui.n_blk] = make_float2(m, s);
+      } else if constexpr (MODE == kModeGroupNorm) {
+        const int32_t gs = p.norm.groups;  // group size (columns)
+        if (sub_tiles == 1) {
+          if (!wait_acc(tl)) { ok = false; break; }
+          const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
+          for (int gi = 0; gi < BN / gs; ++gi) {
+            const int32_t g0 = ui.n0 + gi * gs;
+            if (g0 >= p.N) break;
+            const int nch = gs / 32;
+            float sum = 0.0f;
+            for (int c = 0; c < nch; ++c) {
+              __syncwarp();
+              float v[32];
+              tmem_ld32(tb + gi * gs + c * 32, v);
+              apply_chain32(p.pre, p.n_pre, v, grow, g0 + c * 32, 32, row_ok);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) sum += v[j];
+            }
+            const float mean = sum / static_cast<float>(gs);
+            float m2 = 0.0f;
+            for (int c = 0; c < nch; ++c) {
+              __syncwarp();
+              float v[32];
+              tmem_ld32(tb + gi * gs + c * 32, v);
+              apply_chain32(p.pre, p.n_pre, v, grow, g0 + c * 32, 32, row_ok);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) m2 += (v[j] - mean) * (v[j] - mean);
+            }
+            const float rstd = rsqrtf(m2 / static_cast<float>(gs) + p.norm.eps);
+            for (int c = 0; c < nch; ++c) {
+              __syncwarp();
+              float v[32], ga[32], be[32];
+              const int32_t col0 = g0 + c * 32;
+              tmem_ld32(tb + gi * gs + c * 32, v);
+              apply_chain32(p.pre, p.n_pre, v, grow, col0, 32, row_ok);
+              if (p.norm.p0) ld32(p.norm.p0, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, ga);
+              if (p.norm.p1) ld32(p.norm.p1, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, be);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                float z = (v[j] - mean) * rstd;
+                if (p.norm.p0) z *= ga[j];
+                if (p.norm.p1) z += be[j];
+                v[j] = z;
+              }
+              apply_chain32(p.post, p.n_post, v, grow, col0, 32, row_ok);
+              if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
+            }
+          }
+          release_acc(tl);
+          ++tl;
+        } else {
+          // group of 2*BN columns spread over two accumulators (tl, tl+1):
+          // exact two-pass moments per half, merged with Chan's formula.
+          float mh[2], qh[2];
+          for (int h = 0; h < 2; ++h) {
+            if (!wait_acc(tl + h)) { ok = false; break; }
+            const uint32_t tb = tmem + lane_off + ((tl + h) & 1) * Cfg::kAccStride;
+            const int32_t c0 = ui.n0 + h * BN;
+            float sum = 0.0f;
+            for (int c = 0; c < BN / 32; ++c) {
+              __syncwarp();
+              float v[32];
+              tmem_ld32(tb + c * 32, v);
+              apply_chain32(p.pre, p.n_pre, v, grow, c0 + c * 32, 32, row_ok);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) sum += v[j];
+            }
+            const float mean = sum / static_cast<float>(BN);
+            float m2 = 0.0f;
+            for (int c = 0; c < BN / 32; ++c) {
+              __syncwarp();
+              float v[32];
+              tmem_ld32(tb + c * 32, v);
+              apply_chain32(p.pre, p.n_pre, v, grow, c0 + c * 32, 32, row_ok);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) m2 += (v[j] - mean) * (v[j] - mean);
+            }
+            mh[h] = mean;
+            qh[h] = m2;
+          }
+          if (!ok) break;
+          const float d = mh[1] - mh[0];
+          const float mean = 0.5f * (mh[0] + mh[1]);
+          const float m2 = qh[0] + qh[1] + d * d * (0.5f * static_cast<float>(BN));
+          const float rstd = rsqrtf(m2 / static_cast<float>(2 * BN) + p.norm.eps);
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t tb = tmem + lane_off + ((tl + h) & 1) * Cfg::kAccStride;
+            const int32_t c0 = ui.n0 + h * BN;
+            for (int c = 0; c < BN / 32; ++c) {
+              __syncwarp();
+              float v[32], ga[32], be[32];
+              const int32_t col0 = c0 + c * 32;
+              tmem_ld32(tb + c * 32, v);
+              apply_chain32(p.pre, p.n_pre, v, grow, col0, 32, row_ok);
+              if (p.norm.p0) ld32(p.norm.p0, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, ga);
+              if (p.norm.p1) ld32(p.norm.p1, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, be);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                float z = (v[j] - mean) * rstd;
+                if (p.norm.p0) z *= ga[j];
+                if (p.norm.p1) z += be[j];
+                v[j] = z;
+              }
+              apply_chain32(p.post, p.n_post, v, grow, col0, 32, row_ok);
+              if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
+            }
+            release_acc(tl + h);
+          }
+          tl += 2;
+        }
+      }
+    }
+  }
+
+  // ---------------------------------------------------------------- teardown
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, Cfg::kTmemCols);
+  }
+}
+
+}  // namespace kf
