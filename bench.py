@@ -1,0 +1,422 @@
+"""Benchmark of the fused GEMM + tail path on GB300.
+
+Default workload (the headline line): bf16 Y = GELU_tanh(X W^T + b) * 2 + R,
+X[1024x4096], W[4096x4096] -- one kf_fused_gemm call per step.  The JSON line
+also carries the other workloads of the path (row log-sum-exp, GroupNorm +
+Swish, MoE expert FFN at T=64 and T=4096) under "workloads", each next to its
+unfused torch-eager baseline.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl kf|reference] [--main-only]
+
+Timing: CUDA events on the launching stream around each step; a 256 MiB
+buffer is written between steps so every step starts with a cold L2 (the
+inputs, 59 MB, would otherwise stay resident in the 129 MB L2).  Under
+torchrun each rank runs its own replica (weak scaling; no data-path
+collective) and the max time over ranks is reported.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import subprocess
+import sys
+import tempfile
+import time
+
+import torch
+import torch.nn.functional as F
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import kf_workloads  # noqa: E402
+
+MAIN = "bf16_gelu_scale_residual"
+FLUSH_BYTES = 256 << 20
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"],
+                    src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+KERNEL_FILES = ("kf_ptx.cuh", "kf_common.cuh", "kf_tc_gemm.cuh", "kf_tc_dense.cu")
+
+
+def kernel_source_hash() -> str:
+    """Hash of the sources of the dense tensor-core kernel; a stored ncu traffic
+    figure is used only while they are unchanged since it was captured."""
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2606_02963_gb300", "csrc")
+    for fn in KERNEL_FILES:
+        h.update(fn.encode())
+        h.update(open(os.path.join(d, fn), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def stored_traffic(kernel_tag: str):
+    """Per-launch DRAM bytes from profiles/ncu_traffic.txt (lines:
+    '<tag> <source-hash> <bytes>'), or None if absent or stale."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    if not os.path.exists(p):
+        return None
+    cur = kernel_source_hash()
+    for line in open(p):
+        f = line.split()
+        if len(f) >= 3 and f[0] == kernel_tag and f[1] == cur:
+            return float(f[2])
+    return None
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                          "-i", str(self.index), "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return None
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def time_steps(fn, steps, warmup, flush, stream, host_slack=True):
+    """Mean device time (ms) of fn() over `steps` calls; L2 flushed before each.
+    With host_slack, a ~100 us device-side sleep follows the flush so that the
+    host has enqueued the step before its start event fires (host-side argument
+    marshalling is then outside the device-timed window)."""
+    for _ in range(warmup):
+        flush.zero_()
+        fn()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for a, b in evs:
+        flush.zero_()
+        if host_slack:
+            torch.cuda._sleep(200_000)
+        a.record(stream)
+        fn()
+        b.record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs) / steps
+
+
+# --------------------------------------------------------------- workloads
+def dense_setup(name, dev):
+    inp = kf_workloads.generate(name, seed=0)
+    d = {k: v.to(dev) for k, v in inp.items()}
+    wl = kf_workloads.WORKLOADS[name]
+    chain = []
+    for kind, prm in kf_workloads.chain_spec(wl):
+        chain.append((kind, {k: (d[v] if k in ("p0", "p1") else v) for k, v in prm.items()}))
+    return wl, inp, d, chain
+
+
+def dense_bytes(name, wl):
+    M, N, K = wl.M, wl.N, wl.K
+    b = 2 * (M * K + N * K)
+    if name == MAIN:
+        b += 2 * N + 2 * M * N + 2 * M * N          # bias, R, Y
+    elif name == "bf16_scale_rowlse":
+        b += 4 * M
+    elif name == "bf16_groupnorm_swish":
+        b += 2 * N + 4 * N * 2 + 2 * M * N          # bias, gamma/beta (fp32), Y
+    return b
+
+
+def eager_dense(name, d):
+    X, W = d["X"], d["W"]
+    if name == MAIN:
+        return lambda: F.gelu(F.linear(X, W, d["b"]), approximate="tanh") * 2.0 + d["R"]
+    if name == "bf16_scale_rowlse":
+        return lambda: torch.logsumexp((X @ W.t()).float() * 0.125, dim=1)
+    if name == "bf16_groupnorm_swish":
+        def f():
+            z = F.group_norm(F.linear(X, W, d["b"]), 16, d["gamma"], d["beta"], 1e-5)
+            return z * torch.sigmoid(z)
+        return f
+    raise KeyError(name)
+
+
+def moe_eager(X, logits, Wgu, Wd, k):
+    T, H = X.shape
+    E, I2, _ = Wgu.shape
+    I = I2 // 2
+    v, ids = torch.topk(logits, k, dim=1)
+    w = torch.softmax(v, dim=1)
+    Y = torch.zeros(T, H, dtype=torch.float32, device=X.device)
+    flat = ids.reshape(-1)
+    order = torch.argsort(flat, stable=True)
+    counts = torch.bincount(flat, minlength=E).tolist()
+    tok = order // k
+    wf = w.reshape(-1)[order]
+    s = 0
+    for e in range(E):
+        c = counts[e]
+        if c == 0:
+            continue
+        t = tok[s:s + c]
+        xe = X[t]
+        gu = xe @ Wgu[e].t()
+        h = F.silu(gu[:, :I]) * gu[:, I:]
+        y = h @ Wd[e].t()
+        Y.index_add_(0, t, y.float() * wf[s:s + c, None])
+        s += c
+    return Y.to(torch.bfloat16)
+
+
+def run_kf(args, rank, world, dev):
+    import paper_2606_02963_gb300 as kf
+    kf.lib()
+    peaks = _peaks()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    # ------------------------------------------------------- headline workload
+    wl, inp, d, chain = dense_setup(MAIN, dev)
+    flops = 2.0 * wl.M * wl.N * wl.K
+    out = torch.empty(wl.M, wl.N, dtype=torch.bfloat16, device=dev)
+    step = lambda: kf.fused_gemm(d["X"], d["W"], chain, out=out)
+
+    # e2e: pinned host inputs -> device, kernel, device -> pinned host output
+    hin = {k: v.pin_memory() for k, v in inp.items()}
+    hout = torch.empty(wl.M, wl.N, dtype=torch.bfloat16).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in hin.values())
+    d2h = hout.numel() * hout.element_size()
+
+    def e2e_step():
+        for k2 in hin:
+            d[k2].copy_(hin[k2], non_blocking=True)
+        kf.fused_gemm(d["X"], d["W"], chain, out=out)
+        hout.copy_(out, non_blocking=True)
+
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with Clocks(dev.index if dev.index is not None else 0) as clk:
+        ms = time_steps(step, args.steps, args.warmup, flush, stream)
+    clocks = clk.summary()
+    ms_e2e = time_steps(e2e_step, max(3, args.steps // 2), args.warmup, flush, stream, host_slack=False)
+    if world > 1:
+        t = torch.tensor([ms, ms_e2e], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms, ms_e2e = t.tolist()
+    value = world * flops / (ms * 1e-3) / 1e12
+    e2e_value = world * flops / (ms_e2e * 1e-3) / 1e12
+    ms_eager = time_steps(eager_dense(MAIN, d), args.steps, args.warmup, flush, stream)
+    ms_cublas = time_steps(lambda: torch.matmul(d["X"], d["W"].t()), args.steps, args.warmup, flush, stream)
+    traffic = stored_traffic("dense_store_gelu_1024x4096x4096")
+    achieved = flops / (ms * 1e-3) / 1e12
+    line = {
+        "metric": "fused GEMM+tail TFLOP/s & % of GB300 roofline; speedup vs unfused torch eager",
+        "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 operands, fp32 accumulate", "data": "synthetic (seeded)",
+        "config": {"workload": MAIN, "M": wl.M, "N": wl.N, "K": wl.K,
+                   "chain": "bias -> gelu_tanh -> x2.0 -> +R", "l2": "flushed (256 MiB write) before each step",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peaks["bf16"],
+                     "peak_src": f"{peaks['src']} bf16 burst", "unit": "TFLOP/s",
+                     "frac": round(achieved / peaks["bf16"], 4), "traffic": traffic,
+                     "algorithmic_bytes": dense_bytes(MAIN, wl)},
+        "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "ms_per_step": round(ms_e2e, 4),
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "eager": {"ms_per_step": round(ms_eager, 5), "speedup": round(ms_eager / ms, 3),
+                  "cublas_gemm_only_ms": round(ms_cublas, 5)},
+        "gpu_launches": args.steps,
+        "clocks": clocks,
+    }
+    # -------------------------------------------------- CPU baseline (oracle)
+    if rank == 0 and world == 1 and not args.no_cpu:
+        line["cpu_baseline"] = cpu_baseline(inp, wl, chain_cpu(MAIN, inp), target_s=args.cpu_seconds)
+    # ------------------------------------------------------ other workloads
+    if not args.main_only:
+        line["workloads"] = other_workloads(args, kf, dev, flush, stream, peaks)
+    return line
+
+
+def chain_cpu(name, inp):
+    wl = kf_workloads.WORKLOADS[name]
+    return [(kind, {k: (inp[v] if k in ("p0", "p1") else v) for k, v in prm.items()})
+            for kind, prm in kf_workloads.chain_spec(wl)]
+
+
+def cpu_baseline(inp, wl, chain, target_s=8.0):
+    """The oracle as it stands, on all host cores, over a bounded sample of rows."""
+    import oracle
+    oracle.build()
+    cores = os.cpu_count() or 1
+    rows = 8
+    while True:
+        t0 = time.perf_counter()
+        oracle.fused_gemm(inp["X"], inp["W"], chain, rows=list(range(rows)), nthreads=cores)
+        dt = time.perf_counter() - t0
+        if dt >= target_s / 4 or rows >= wl.M:
+            break
+        rows = min(wl.M, max(rows * 2, int(rows * target_s / max(dt, 1e-3) / 2)))
+    flops = 2.0 * rows * wl.N * wl.K
+    return {"value": round(flops / dt / 1e12, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+            "sample": f"{rows} of {wl.M} rows of {wl.name} (fp64 C, {dt:.2f} s)"}
+
+
+def other_workloads(args, kf, dev, flush, stream, peaks):
+    res = {}
+    steps = max(3, min(args.steps, 20))
+    for name in ("bf16_scale_rowlse", "bf16_groupnorm_swish"):
+        wl, inp, d, chain = dense_setup(name, dev)
+        flops = 2.0 * wl.M * wl.N * wl.K
+        ms = time_steps(lambda: kf.fused_gemm(d["X"], d["W"], chain), steps, args.warmup, flush, stream)
+        ms_e = time_steps(eager_dense(name, d), steps, args.warmup, flush, stream)
+        ms_c = time_steps(lambda: torch.matmul(d["X"], d["W"].t()), steps, args.warmup, flush, stream)
+        t_roof = max(flops / (peaks["bf16"] * 1e12), dense_bytes(name, wl) / (peaks["hbm"] * 1e9)) * 1e3
+        res[name] = {"tflops": round(flops / ms / 1e9, 2), "ms": round(ms, 5), "bound": "tensor",
+                     "roofline_frac": round(t_roof / ms, 4), "eager_ms": round(ms_e, 5),
+                     "speedup_vs_eager": round(ms_e / ms, 3), "cublas_gemm_only_ms": round(ms_c, 5),
+                     "launches_per_step": 2 if name == "bf16_scale_rowlse" else 1}
+        del d, inp
+    E, k, H, I = 32, 4, 2880, 2880
+    m = None
+    for T in (64, 4096):
+        g = torch.Generator("cpu").manual_seed(0)
+        X = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
+        logits = torch.randn(T, E, generator=g).to(dev)
+        if m is None:
+            gd = torch.Generator(dev).manual_seed(1)
+            m = dict(W_gu=(torch.randn(E, 2 * I, H, generator=gd, device=dev) * 0.02).to(torch.bfloat16),
+                     W_down=(torch.randn(E, H, I, generator=gd, device=dev) * 0.02).to(torch.bfloat16))
+        ws = torch.empty(kf.moe_ffn_workspace_bytes(T, H, I, E, k), dtype=torch.uint8, device=dev)
+        out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
+        fn = lambda: kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, out=out, workspace=ws)
+        ms = time_steps(fn, steps, args.warmup, flush, stream)
+        ms_e = time_steps(lambda: moe_eager(X, logits, m["W_gu"], m["W_down"], k), max(3, steps // 2),
+                          args.warmup, flush, stream)
+        ids = torch.topk(logits, k, dim=1).indices
+        touched = int(torch.unique(ids).numel())
+        wbytes = touched * (2 * I * H + H * I) * 2
+        byts = wbytes + 2 * T * H * 2 + 4 * T * E
+        flops = 2.0 * T * k * (2 * I * H + H * I)
+        t_roof = max(flops / (peaks["bf16"] * 1e12), byts / (peaks["hbm"] * 1e9)) * 1e3
+        bound = "hbm" if byts / (peaks["hbm"] * 1e9) > flops / (peaks["bf16"] * 1e12) else "tensor"
+        res[f"moe_T{T}"] = {"tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
+                            "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
+                            "experts_touched": touched, "eager_ms": round(ms_e, 5),
+                            "speedup_vs_eager": round(ms_e / ms, 3), "launches_per_step": 6}
+    return res
+
+
+def run_reference(args, rank, world):
+    """The oracle as it stands on the host cores, on bounded row samples of the
+    headline workload (one sample per step)."""
+    import oracle
+    oracle.build()
+    wl = kf_workloads.WORKLOADS[MAIN]
+    inp = kf_workloads.generate(MAIN, seed=0)
+    chain = chain_cpu(MAIN, inp)
+    cores = os.cpu_count() or 1
+    rows = args.ref_rows
+    sample = lambda i: [(i * rows + r) % wl.M for r in range(rows)]
+    for i in range(args.warmup):
+        oracle.fused_gemm(inp["X"], inp["W"], chain, rows=sample(i), nthreads=cores)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle.fused_gemm(inp["X"], inp["W"], chain, rows=sample(args.warmup + i), nthreads=cores)
+    dt = (time.perf_counter() - t0) / args.steps
+    flops = 2.0 * rows * wl.N * wl.K
+    v = flops / dt / 1e12
+    return {"metric": "fused GEMM+tail TFLOP/s & % of GB300 roofline; speedup vs unfused torch eager",
+            "impl": "reference", "value": round(v, 6), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
+            "config": {"workload": MAIN, "M": wl.M, "N": wl.N, "K": wl.K,
+                       "chain": "bias -> gelu_tanh -> x2.0 -> +R"},
+            "cpu_baseline": {"value": round(v, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{rows} rows of {wl.M} per step (fp64 C oracle)"},
+            "e2e": {"value": round(v, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="kf", choices=["kf", "reference"])
+    ap.add_argument("--main-only", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=8.0)
+    ap.add_argument("--ref-rows", type=int, default=16)
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=dev)
+    line = run_kf(args, rank, world, dev)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
