@@ -178,6 +178,32 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
                      int32_t* topk_ids_out, float* topk_w_out, void* stream);
 size_t kf_moe_ffn_workspace(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k);
 
+/*
+ * kf_fused_gemm_lse_noalloc -- kf_fused_gemm for row log-sum-exp chains, without
+ * a workspace argument.  The paper has no counterpart: this entry point exists for
+ * callers that cannot allocate device memory -- e.g. code hosted by another
+ * runtime that owns all device memory and exposes no allocator to it, or
+ * latency-critical loops that must not call cudaMalloc because it can
+ * synchronize the device.  The caller still passes X, W and Y (as for
+ * kf_fused_gemm, with Y the fp32 or bf16 [M] result; the chain must hold
+ * KF_OP_ROW_LOGSUMEXP, else KF_ERR_INVALID_ARG).
+ *   Scratch: the per-tile row partials live in one fixed device array of
+ *   kf_fused_gemm_lse_noalloc_max_bytes() bytes (4 MiB) compiled into the
+ *   library; every GPU that loads the library holds it until the process exits.
+ *   Problems needing more (M x ceil(N/128) x 8 bytes) return KF_ERR_WORKSPACE and
+ *   launch nothing.  This call never allocates or frees device memory.
+ *   The first call on a device looks up the array's device address (with that
+ *   device current) and caches it; make that first call before any stream
+ *   capture.  Every call shares the one array: calls whose executions overlap
+ *   on the GPU (different streams, or different host threads) race on it and
+ *   must be serialized by the caller.  Each call overwrites every partial it
+ *   reads, so no clearing is needed between calls.
+ */
+kf_status kf_fused_gemm_lse_noalloc(const void* X, int32_t x_dtype, int64_t ldx, const void* W, int32_t w_dtype,
+                                    int64_t ldw, void* Y, int32_t y_dtype, int64_t M, int64_t N, int64_t K,
+                                    const kf_epilogue* epi, void* stream);
+size_t kf_fused_gemm_lse_noalloc_max_bytes(void);
+
 /* Synchronize `stream`, read and clear this device's error word.  Returns KF_OK,
  * KF_ERR_DEVICE_TIMEOUT or KF_ERR_DEVICE_BOUNDS; *raw (if non-NULL) receives the
  * raw bit set (1 = producer wait, 2 = MMA wait, 4 = epilogue wait, 8 = bounds). */

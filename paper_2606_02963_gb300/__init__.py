@@ -33,7 +33,8 @@ OPS = {
 ABI_SYMBOLS = (
     "kf_fused_gemm", "kf_fused_gemm_workspace", "kf_moe_route", "kf_grouped_gemm",
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
-    "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version",
+    "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
+    "kf_fused_gemm_lse_noalloc_max_bytes",
 )
 
 
@@ -79,6 +80,9 @@ def lib() -> ctypes.CDLL:
     L.kf_moe_ffn_workspace.restype = SZ
     L.kf_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
     L.kf_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
+    L.kf_fused_gemm_lse_noalloc.argtypes = [P, I32, I64, P, I32, I64, P, I32, I64, I64, I64, EP, P]
+    L.kf_fused_gemm_lse_noalloc.restype = I32
+    L.kf_fused_gemm_lse_noalloc_max_bytes.restype = SZ
     L.kf_status_string.argtypes = [I32]
     L.kf_status_string.restype = ctypes.c_char_p
     L.kf_abi_version.restype = I32

@@ -613,3 +613,62 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the row log-sum-exp GEMM.  Its per-tile row
+// partials live in a fixed file-scope device array instead of a caller
+// workspace, for callers that cannot allocate device memory themselves.
+// ---------------------------------------------------------------------------
+namespace kf {
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;  // 4 MiB, resident on every device that loads the library
+static __device__ __align__(256) float2 g_kf_noalloc_scratch[kNoAllocScratchBytes / sizeof(float2)];
+
+struct NoAllocScratch {
+  bool init = false;
+  void* ptr = nullptr;
+};
+NoAllocScratch g_noalloc[kMaxDevices];
+std::mutex g_noalloc_mu;
+
+// Device address of the scratch array on the current device.  The symbol's
+// name is only a host-side handle; the address is looked up once per device
+// (with that device current) and cached.
+kf_status noalloc_scratch(void** out) {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return KF_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  NoAllocScratch& s = g_noalloc[d];
+  if (!s.init) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_kf_noalloc_scratch) != cudaSuccess || p == nullptr) return KF_ERR_CUDA;
+    s.ptr = p;
+    s.init = true;
+  }
+  *out = s.ptr;
+  return KF_OK;
+}
+
+}  // namespace
+}  // namespace kf
+
+extern "C" size_t kf_fused_gemm_lse_noalloc_max_bytes(void) { return kf::kNoAllocScratchBytes; }
+
+extern "C" kf_status kf_fused_gemm_lse_noalloc(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt,
+                                               int64_t ldw, void* Y, int32_t yt, int64_t M, int64_t N, int64_t K,
+                                               const kf_epilogue* epi, void* stream) {
+  bool has_lse = false;
+  if (epi && epi->ops)
+    for (int i = 0; i < epi->num_ops && i < kf::kMaxOps; ++i) has_lse |= epi->ops[i].kind == KF_OP_ROW_LOGSUMEXP;
+  if (!has_lse) return KF_ERR_INVALID_ARG;  // this variant is the row log-sum-exp GEMM only
+  if (M < 0 || N < 0) return KF_ERR_INVALID_ARG;
+  if (M == 0 || N == 0) return KF_OK;
+  const size_t need = kf::lse_ws_bytes(M, N);
+  if (need > kf::kNoAllocScratchBytes) return KF_ERR_WORKSPACE;  // problem exceeds the fixed scratch
+  if (xt != KF_BF16 || wt != KF_BF16) return KF_ERR_UNSUPPORTED;
+  void* scratch = nullptr;
+  kf_status st = kf::noalloc_scratch(&scratch);
+  if (st != KF_OK) return st;
+  return kf_fused_gemm(X, xt, ldx, W, wt, ldw, Y, yt, 1, M, N, K, epi, scratch, kf::kNoAllocScratchBytes, stream);
+}
