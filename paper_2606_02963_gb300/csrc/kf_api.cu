@@ -310,6 +310,7 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   p.row_dst = pl.row_dst;
   p.dst_rows = static_cast<int32_t>(pl.dst_rows);
   fill_params_common(p, pl, di.err);
+  p.fast = g.c_dtype == KF_BF16 && pl.mode != kModeScatter;
   const int64_t ub = ((g.rows_total + kBM - 1) / kBM + g.G) * p.tiles_n;
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
   return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, p, grid, s));
@@ -442,6 +443,7 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   p.c_vec_ok = aligned16(Y) && (ldy * elt_size(yt)) % 16 == 0;
   if (pl.mode == kModeLse) p.lse_part = static_cast<float2*>(workspace);
   fill_params_common(p, pl, di.err);
+  p.fast = yt == KF_BF16 && pl.mode != kModeLse;  // bf16 results: reduced-precision activations suffice
   const int grid = std::min(p.total_units, di.nsm);
   st = cuda_status(tc_dense_launch(pl.mode, bn, ma, mb, p, sub, grid, s));
   if (st != KF_OK || pl.mode != kModeLse) return st;

@@ -68,7 +68,12 @@ struct TcParams {
   uint32_t* err;
   uint64_t wait_ns;
   uint64_t drain_ns;
+  int32_t fast;         // reduced-precision activations (result stored as bf16)
 };
+
+// dispatch the chain on the runtime `fast` flag (uniform across the CTA)
+__device__ __forceinline__ void apply_chain32_rt(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row,
+                                                 int64_t col0, int nvalid, bool row_ok);
 
 // ---------------------------------------------------------------- loads/stores
 __device__ __forceinline__ float ld_elem(const void* p, int dt, int64_t i) {
@@ -107,6 +112,27 @@ __device__ __forceinline__ void ld32(const void* p, int dt, int64_t i0, int nval
   } else {
 #pragma unroll
     for (int j = 0; j < 32; ++j) o[j] = (j < nvalid) ? ld_elem(p, dt, i0 + j) : 0.0f;
+  }
+}
+
+// 8 consecutive elements (16-byte vector loads when vec_ok; all in bounds).
+__device__ __forceinline__ void ld8(const void* p, int dt, int64_t i0, bool vec_ok, float (&o)[8]) {
+  if (vec_ok && dt == KF_BF16) {
+    uint4 u = __ldg(reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p) + i0));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      o[2 * h] = __uint_as_float(w[h] << 16);
+      o[2 * h + 1] = __uint_as_float(w[h] & 0xFFFF0000u);
+    }
+  } else if (vec_ok) {
+    const float4* q = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(p) + i0);
+    const float4 a = __ldg(q), b = __ldg(q + 1);
+    o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
+    o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o[j] = ld_elem(p, dt, i0 + j);
   }
 }
 
@@ -159,6 +185,28 @@ __device__ __forceinline__ float f_mish(float x) {
   return x * tanhf(sp);
 }
 
+// Reduced-precision forms, used only when the result is rounded to bf16 (8
+// significant bits): the hardware tanh (tanh.approx.f32, relative error about
+// 2^-11) and sigmoid(x) = (1 + tanh(x/2)) / 2.
+__device__ __forceinline__ float tanh_fast(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float f_sigmoid_fast(float x) { return fmaf(0.5f, tanh_fast(0.5f * x), 0.5f); }
+__device__ __forceinline__ float f_gelu_tanh_fast(float x) {
+  const float c = 0.7978845608028654f;
+  const float hx = 0.5f * x;
+  return fmaf(hx, tanh_fast(c * fmaf(0.044715f * x, x * x, x)), hx);
+}
+__device__ __forceinline__ float f_mish_fast(float x) {
+  float sp = x > 15.0f ? x : __logf(1.0f + __expf(x));
+  return x * tanh_fast(sp);
+}
+
+template <bool FAST>
+__device__ __forceinline__ float sigm(float x) { return FAST ? f_sigmoid_fast(x) : f_sigmoid(x); }
+
 __device__ __forceinline__ float apply_scalar_op(const DevOp& op, float x) {
   switch (op.kind) {
     case KF_OP_SCALE: return x * op.scalar;
@@ -174,7 +222,9 @@ __device__ __forceinline__ float apply_scalar_op(const DevOp& op, float x) {
 
 // Apply ops[0..n) to the 32 values of row `row` starting at column col0 (the
 // first `nvalid` columns exist).  Operands of rows that do not exist are not
-// read (row_ok == false).
+// read (row_ok == false).  FAST selects the reduced-precision activations (for
+// chains whose result is stored as bf16).
+template <bool FAST>
 __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
                                               int nvalid, bool row_ok) {
   for (int o = 0; o < n; ++o) {
@@ -211,19 +261,19 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
       } break;
       case KF_OP_GELU_TANH: {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = f_gelu_tanh(v[j]);
+        for (int j = 0; j < 32; ++j) v[j] = FAST ? f_gelu_tanh_fast(v[j]) : f_gelu_tanh(v[j]);
       } break;
       case KF_OP_SILU: {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = v[j] * f_sigmoid(v[j]);
+        for (int j = 0; j < 32; ++j) v[j] = v[j] * sigm<FAST>(v[j]);
       } break;
       case KF_OP_SIGMOID: {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = f_sigmoid(v[j]);
+        for (int j = 0; j < 32; ++j) v[j] = sigm<FAST>(v[j]);
       } break;
       case KF_OP_MISH: {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = f_mish(v[j]);
+        for (int j = 0; j < 32; ++j) v[j] = FAST ? f_mish_fast(v[j]) : f_mish(v[j]);
       } break;
       case KF_OP_LEAKY_RELU: {
         const float s = op.scalar;
@@ -233,6 +283,15 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
       default: break;
     }
   }
+}
+
+__device__ __forceinline__ void apply_chain32_rt(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row,
+                                                 int64_t col0, int nvalid, bool row_ok) {
+  if (n == 0) return;
+  if (fast)
+    apply_chain32<true>(ops, n, v, row, col0, nvalid, row_ok);
+  else
+    apply_chain32<false>(ops, n, v, row, col0, nvalid, row_ok);
 }
 
 }  // namespace kf

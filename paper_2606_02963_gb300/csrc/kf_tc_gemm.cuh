@@ -30,7 +30,8 @@ namespace kf {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 64 + 32 * kEpiWarps;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int kABytes = kBM * kBK * 2;
 
 __host__ __device__ constexpr int pow2_at_least(int x) {
@@ -46,8 +47,8 @@ struct TcCfg {
   // accumulator buffer b starts at TMEM column b * kAccStride
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
-  static constexpr int kBarBytes = 8 * (2 * STAGES + 5);
-  static constexpr int kMiscBytes = 64;
+  static constexpr int kBarBytes = (8 * (2 * STAGES + 5) + 63) / 64 * 64;  // keeps what follows 64-B aligned
+  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16;  // flags + epilogue exchange buffer
   static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
   static constexpr int kSmemUse = STAGES * kStageBytes + kBarBytes + kMiscBytes + kTableBytes;
   // pad to > half of the SM's shared memory so that at most one such CTA is
@@ -95,7 +96,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&accf[a], 1);
-      mbar_init(&acce[a], 4);
+      mbar_init(&acce[a], kEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -258,9 +259,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
+    // 8 warps: warp w reads TMEM lane quadrant q = w % 4 (rows 32q..32q+31, one
+    // row per thread); the two warps of a quadrant (half h = 0, 1) take
+    // alternate 32-column chunks and exchange row statistics through shared
+    // memory where a reduction needs the whole row / group.
+    const int ew = warp - 2;
     const int q = warp & 3;
+    const int h = ew >> 2;
     const int32_t row_in_tile = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const bool fast = p.fast != 0;
+    float4* xch = reinterpret_cast<float4*>(misc + 16);  // [2 halves][4 quadrants][32 lanes]
     int32_t tl = 0;
     bool ok = true;
 
@@ -279,6 +288,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acce[t & 1]);
+    };
+    // the two warps of this quadrant meet here (named barrier 1 + q, 64 threads)
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(1 + q), "r"(64) : "memory"); };
+    // both warps of the quadrant vote; true only if both passed.  Used right
+    // after an accumulator wait in the modes that exchange data, so the pair
+    // always takes the same abort decision before meeting at pair_sync.
+    auto pair_vote = [&](bool mine) -> bool {
+      uint32_t r;
+      asm volatile(
+          "{\n\t.reg .pred pi, po;\n\t"
+          "setp.ne.u32 pi, %1, 0;\n\t"
+          "bar.red.and.pred po, %2, 64, pi;\n\t"
+          "selp.u32 %0, 1, 0, po;\n\t}\n"
+          : "=r"(r)
+          : "r"(mine ? 1u : 0u), "r"(1 + q)
+          : "memory");
+      return r != 0;
+    };
+    // Chan's pairwise merge of (count, mean, M2) moments
+    auto chan = [](float na, float ma, float qa, float nb, float mb, float qb, float& n, float& m, float& qq) {
+      n = na + nb;
+      if (n == 0.0f) { m = 0.0f; qq = 0.0f; return; }
+      const float d = mb - ma;
+      m = ma + d * (nb / n);
+      qq = qa + qb + d * d * (na * nb / n);
     };
 
     for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
@@ -302,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        for (int c = 0; c < Cfg::kOutN / 32; ++c) {
+        for (int c = h; c < Cfg::kOutN / 32; c += 2) {
           const int32_t col0 = ui.n0 + c * 32;
           const int nvalid = min(32, p.N - col0);
           if (nvalid <= 0) break;  // uniform across the warp
@@ -312,12 +346,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             float gt[32];
             tmem_ld32(tb + c * 32, gt);
             tmem_ld32(tb + Cfg::kOutN + c * 32, v);
+            if (fast) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = gt[j] * f_sigmoid(gt[j]) * v[j];
-            apply_chain32(p.post, p.n_post, v, grow, col0, nvalid, row_ok);
+              for (int j = 0; j < 32; ++j) v[j] = gt[j] * f_sigmoid_fast(gt[j]) * v[j];
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) v[j] = gt[j] * f_sigmoid(gt[j]) * v[j];
+            }
+            apply_chain32_rt(fast, p.post, p.n_post, v, grow, col0, nvalid, row_ok);
           } else {
             tmem_ld32(tb + c * 32, v);
-            apply_chain32(p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+            apply_chain32_rt(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
           }
           if constexpr (MODE == kModeScatter) {
             if (wr) {
@@ -340,17 +379,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         release_acc(tl);
         ++tl;
       } else if constexpr (MODE == kModeLse) {
-        if (!wait_acc(tl)) { ok = false; break; }
+        if (!pair_vote(wait_acc(tl))) { ok = false; break; }
         const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
         float m = -INFINITY, s = 0.0f;
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = h; c < BN / 32; c += 2) {
           const int32_t col0 = ui.n0 + c * 32;
           const int nvalid = min(32, p.N - col0);
           if (nvalid <= 0) break;
           __syncwarp();
           float v[32];
           tmem_ld32(tb + c * 32, v);
-          apply_chain32(p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+          apply_chain32_rt(false, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
           float cm = -INFINITY;
 #pragma unroll
           for (int j = 0; j < 32; ++j)
@@ -359,122 +398,124 @@ __global__ void __launch_bounds__(kThreads, 1)
           float add = 0.0f;
 #pragma unroll
           for (int j = 0; j < 32; ++j)
-            if (j < nvalid) add += expf(v[j] - nm);
-          s = (m == -INFINITY ? 0.0f : s * expf(m - nm)) + add;
+            if (j < nvalid) add += __expf(v[j] - nm);
+          s = (m == -INFINITY ? 0.0f : s * __expf(m - nm)) + add;
           m = nm;
         }
         release_acc(tl);
         ++tl;
-        if (row_ok) p.lse_part[static_cast<int64_t>(grow) * p.tiles_n + ui.n_blk] = make_float2(m, s);
+        // merge the two halves of the row: half 1 hands (m, s) to half 0
+        if (h == 1) xch[q * 32 + lane] = make_float4(m, s, 0.f, 0.f);
+        pair_sync();
+        if (h == 0) {
+          const float4 o = xch[q * 32 + lane];
+          const float nm = fmaxf(m, o.x);
+          float ss = 0.0f;
+          if (nm != -INFINITY)
+            ss = (m == -INFINITY ? 0.f : s * __expf(m - nm)) + (o.x == -INFINITY ? 0.f : o.y * __expf(o.x - nm));
+          if (row_ok) p.lse_part[static_cast<int64_t>(grow) * p.tiles_n + ui.n_blk] = make_float2(nm, ss);
+        }
+        pair_sync();  // xch is reused by the next tile
       } else if constexpr (MODE == kModeGroupNorm) {
-        const int32_t gs = p.norm.groups;  // group size (columns)
-        if (sub_tiles == 1) {
+        const int32_t gs = p.norm.groups;  // group size (columns), multiple of 32
+        const float eps = p.norm.eps;
+        // normalise + affine + post chain + store one 32-column chunk
+        auto finish_chunk = [&](uint32_t taddr, int32_t col0, float mean, float rstd) {
+          float v[32];
+          tmem_ld32(taddr, v);
+          apply_chain32_rt(false, p.pre, p.n_pre, v, grow, col0, 32, row_ok);
+#pragma unroll
+          for (int j8 = 0; j8 < 4; ++j8) {
+            float ga[8], be[8];
+            if (p.norm.p0) ld8(p.norm.p0, p.norm.p_dtype, col0 + 8 * j8, p.norm.vec_ok != 0, ga);
+            if (p.norm.p1) ld8(p.norm.p1, p.norm.p_dtype, col0 + 8 * j8, p.norm.vec_ok != 0, be);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              float z = (v[8 * j8 + j] - mean) * rstd;
+              if (p.norm.p0) z *= ga[j];
+              if (p.norm.p1) z += be[j];
+              v[8 * j8 + j] = z;
+            }
+          }
+          apply_chain32_rt(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
+          if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
+        };
+        // exact two-pass moments (count, mean, M2) of this thread's chunks c0, c0+step, ... < c1
+        auto moments = [&](uint32_t tb, int32_t colbase, int c0, int c1, int step, float& n, float& mean, float& m2) {
+          float sum = 0.0f;
+          int cnt = 0;
+          for (int c = c0; c < c1; c += step) {
+            __syncwarp();
+            float v[32];
+            tmem_ld32(tb + c * 32, v);
+            apply_chain32_rt(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) sum += v[j];
+            ++cnt;
+          }
+          n = 32.0f * cnt;
+          mean = cnt ? sum / n : 0.0f;
+          float qq = 0.0f;
+          for (int c = c0; c < c1; c += step) {
+            __syncwarp();
+            float v[32];
+            tmem_ld32(tb + c * 32, v);
+            apply_chain32_rt(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) qq += (v[j] - mean) * (v[j] - mean);
+          }
+          m2 = qq;
+        };
+        if (gs < BN) {
+          // several whole groups per tile: half h takes groups h, h+2, ...
           if (!wait_acc(tl)) { ok = false; break; }
           const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
-          for (int gi = 0; gi < BN / gs; ++gi) {
+          const int nch = gs / 32;
+          for (int gi = h; gi < BN / gs; gi += 2) {
             const int32_t g0 = ui.n0 + gi * gs;
             if (g0 >= p.N) break;
-            const int nch = gs / 32;
-            float sum = 0.0f;
+            float n, mean, m2;
+            moments(tb + gi * gs, g0, 0, nch, 1, n, mean, m2);
+            const float rstd = rsqrtf(m2 / n + eps);
             for (int c = 0; c < nch; ++c) {
               __syncwarp();
-              float v[32];
-              tmem_ld32(tb + gi * gs + c * 32, v);
-              apply_chain32(p.pre, p.n_pre, v, grow, g0 + c * 32, 32, row_ok);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) sum += v[j];
-            }
-            const float mean = sum / static_cast<float>(gs);
-            float m2 = 0.0f;
-            for (int c = 0; c < nch; ++c) {
-              __syncwarp();
-              float v[32];
-              tmem_ld32(tb + gi * gs + c * 32, v);
-              apply_chain32(p.pre, p.n_pre, v, grow, g0 + c * 32, 32, row_ok);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) m2 += (v[j] - mean) * (v[j] - mean);
-            }
-            const float rstd = rsqrtf(m2 / static_cast<float>(gs) + p.norm.eps);
-            for (int c = 0; c < nch; ++c) {
-              __syncwarp();
-              float v[32], ga[32], be[32];
-              const int32_t col0 = g0 + c * 32;
-              tmem_ld32(tb + gi * gs + c * 32, v);
-              apply_chain32(p.pre, p.n_pre, v, grow, col0, 32, row_ok);
-              if (p.norm.p0) ld32(p.norm.p0, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, ga);
-              if (p.norm.p1) ld32(p.norm.p1, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, be);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                float z = (v[j] - mean) * rstd;
-                if (p.norm.p0) z *= ga[j];
-                if (p.norm.p1) z += be[j];
-                v[j] = z;
-              }
-              apply_chain32(p.post, p.n_post, v, grow, col0, 32, row_ok);
-              if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
+              finish_chunk(tb + gi * gs + c * 32, g0 + c * 32, mean, rstd);
             }
           }
           release_acc(tl);
           ++tl;
         } else {
-          // group of 2*BN columns spread over two accumulators (tl, tl+1):
-          // exact two-pass moments per half, merged with Chan's formula.
-          float mh[2], qh[2];
-          for (int h = 0; h < 2; ++h) {
-            if (!wait_acc(tl + h)) { ok = false; break; }
-            const uint32_t tb = tmem + lane_off + ((tl + h) & 1) * Cfg::kAccStride;
-            const int32_t c0 = ui.n0 + h * BN;
-            float sum = 0.0f;
-            for (int c = 0; c < BN / 32; ++c) {
-              __syncwarp();
-              float v[32];
-              tmem_ld32(tb + c * 32, v);
-              apply_chain32(p.pre, p.n_pre, v, grow, c0 + c * 32, 32, row_ok);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) sum += v[j];
-            }
-            const float mean = sum / static_cast<float>(BN);
-            float m2 = 0.0f;
-            for (int c = 0; c < BN / 32; ++c) {
-              __syncwarp();
-              float v[32];
-              tmem_ld32(tb + c * 32, v);
-              apply_chain32(p.pre, p.n_pre, v, grow, c0 + c * 32, 32, row_ok);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) m2 += (v[j] - mean) * (v[j] - mean);
-            }
-            mh[h] = mean;
-            qh[h] = m2;
+          // one group spans sub_tiles (1 or 2) accumulators of BN columns; the two
+          // halves split its chunks and merge their moments through shared memory
+          float n = 0.f, mean = 0.f, m2 = 0.f;
+          for (int st = 0; st < sub_tiles; ++st) {
+            if (!pair_vote(wait_acc(tl + st))) { ok = false; break; }
+            const uint32_t tb = tmem + lane_off + ((tl + st) & 1) * Cfg::kAccStride;
+            float nb, mb, qb;
+            moments(tb, ui.n0 + st * BN, h, BN / 32, 2, nb, mb, qb);
+            chan(n, mean, m2, nb, mb, qb, n, mean, m2);
           }
           if (!ok) break;
-          const float d = mh[1] - mh[0];
-          const float mean = 0.5f * (mh[0] + mh[1]);
-          const float m2 = qh[0] + qh[1] + d * d * (0.5f * static_cast<float>(BN));
-          const float rstd = rsqrtf(m2 / static_cast<float>(2 * BN) + p.norm.eps);
-          for (int h = 0; h < 2; ++h) {
-            const uint32_t tb = tmem + lane_off + ((tl + h) & 1) * Cfg::kAccStride;
-            const int32_t c0 = ui.n0 + h * BN;
-            for (int c = 0; c < BN / 32; ++c) {
+          xch[(h * 4 + q) * 32 + lane] = make_float4(n, mean, m2, 0.f);
+          pair_sync();
+          const float4 o = xch[((h ^ 1) * 4 + q) * 32 + lane];
+          pair_sync();
+          // both halves merge in the same order (half 0 first) -> identical stats
+          float tn, tm, tq;
+          if (h == 0)
+            chan(n, mean, m2, o.x, o.y, o.z, tn, tm, tq);
+          else
+            chan(o.x, o.y, o.z, n, mean, m2, tn, tm, tq);
+          const float rstd = rsqrtf(tq / tn + eps);
+          for (int st = 0; st < sub_tiles; ++st) {
+            const uint32_t tb = tmem + lane_off + ((tl + st) & 1) * Cfg::kAccStride;
+            for (int c = h; c < BN / 32; c += 2) {
               __syncwarp();
-              float v[32], ga[32], be[32];
-              const int32_t col0 = c0 + c * 32;
-              tmem_ld32(tb + c * 32, v);
-              apply_chain32(p.pre, p.n_pre, v, grow, col0, 32, row_ok);
-              if (p.norm.p0) ld32(p.norm.p0, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, ga);
-              if (p.norm.p1) ld32(p.norm.p1, p.norm.p_dtype, col0, 32, p.norm.vec_ok != 0, be);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                float z = (v[j] - mean) * rstd;
-                if (p.norm.p0) z *= ga[j];
-                if (p.norm.p1) z += be[j];
-                v[j] = z;
-              }
-              apply_chain32(p.post, p.n_post, v, grow, col0, 32, row_ok);
-              if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
+              finish_chunk(tb + c * 32, ui.n0 + st * BN + c * 32, tm, rstd);
             }
-            release_acc(tl + h);
+            release_acc(tl + st);
           }
-          tl += 2;
+          tl += sub_tiles;
         }
       }
     }
