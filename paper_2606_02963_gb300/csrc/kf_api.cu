@@ -205,18 +205,21 @@ void fill_params_common(TcParams& p, const ChainPlan& pl, uint32_t* err) {
   p.drain_ns = std::max<uint64_t>(p.wait_ns, 1000000000ull);
 }
 
-// Tile width for the dense store / LSE variants: the fewest tiles per CTA of
-// the persistent grid, weighted by the tile width (+ a fixed per-tile cost).
-int pick_dense_bn(int mode, int64_t M, int64_t N, int nsm) {
+// Tile width for the dense store / LSE variants: the fewest tiles per CTA (or
+// CTA pair) of the persistent grid, weighted by the tile width (+ a fixed
+// per-tile cost).
+int pick_dense_bn(int mode, int64_t M, int64_t N, int nsm, bool cta2) {
   static const int cand[] = {256, 224, 192, 128};
   int best = 0;
   int64_t best_cost = INT64_MAX;
-  const int64_t tm = (M + kBM - 1) / kBM;
+  const int64_t rows = cta2 ? 2 * kBM : kBM;
+  const int64_t workers = cta2 ? nsm / 2 : nsm;
+  const int64_t tm = (M + rows - 1) / rows;
   for (int bn : cand) {
-    if (!tc_dense_has(mode, bn)) continue;
+    if (!tc_dense_has(mode, bn, cta2)) continue;
     const int64_t tiles = tm * ((N + bn - 1) / bn);
-    const int64_t per_cta = (tiles + nsm - 1) / nsm;
-    const int64_t cost = per_cta * (bn + 48);
+    const int64_t per = (tiles + workers - 1) / workers;
+    const int64_t cost = per * (bn + 48);
     if (cost < best_cost) {
       best_cost = cost;
       best = bn;
@@ -412,6 +415,9 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     return cuda_status(simt_gemm_f32_launch(sp, s));
   }
 
+  // CTA pairs (256-row tiles, tcgen05.mma.cta_group::2) unless one 128-row
+  // tile already covers M
+  const bool cta2 = M > kBM && di.nsm >= 2;
   int bn = 0, sub = 1;
   int64_t tiles_n = 0;
   if (pl.mode == kModeGroupNorm) {
@@ -419,21 +425,21 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     sub = pl.gs == 512 ? 2 : 1;
     tiles_n = (N + bn * sub - 1) / (bn * sub);
   } else {
-    bn = pick_dense_bn(pl.mode, M, N, di.nsm);
+    bn = pick_dense_bn(pl.mode, M, N, di.nsm, cta2);
     if (bn == 0) return KF_ERR_UNSUPPORTED;
     tiles_n = (N + bn - 1) / bn;
   }
   CUtensorMap ma, mb;
   st = make_map(&ma, X, K, M, ldx * 2, 1, 0, kBM, 2);
   if (st != KF_OK) return st;
-  st = make_map(&mb, W, K, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, bn, 3);
+  st = make_map(&mb, W, K, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, cta2 ? bn / 2 : bn, 3);
   if (st != KF_OK) return st;
   TcParams p;
   std::memset(&p, 0, sizeof(p));
   p.M = static_cast<int32_t>(M);
   p.N = static_cast<int32_t>(N);
   p.K = static_cast<int32_t>(K);
-  p.tiles_m = static_cast<int32_t>((M + kBM - 1) / kBM);
+  p.tiles_m = static_cast<int32_t>((M + (cta2 ? 2 * kBM : kBM) - 1) / (cta2 ? 2 * kBM : kBM));
   p.tiles_n = static_cast<int32_t>(tiles_n);
   p.num_kb = static_cast<int32_t>((K + kBK - 1) / kBK);
   p.total_units = p.tiles_m * p.tiles_n;
@@ -444,8 +450,8 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   if (pl.mode == kModeLse) p.lse_part = static_cast<float2*>(workspace);
   fill_params_common(p, pl, di.err);
   p.fast = yt == KF_BF16 && pl.mode != kModeLse;  // bf16 results: reduced-precision activations suffice
-  const int grid = std::min(p.total_units, di.nsm);
-  st = cuda_status(tc_dense_launch(pl.mode, bn, ma, mb, p, sub, grid, s));
+  const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
+  st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, ma, mb, p, sub, grid, s));
   if (st != KF_OK || pl.mode != kModeLse) return st;
   LseCombineParams cp;
   std::memset(&cp, 0, sizeof(cp));

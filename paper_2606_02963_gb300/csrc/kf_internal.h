@@ -10,11 +10,14 @@ namespace kf {
 
 // Tensor-core GEMM launchers.  `bn` selects the tile width among the compiled
 // variants; returns cudaErrorInvalidValue for a variant that is not built.
-bool tc_dense_has(int mode, int bn);
+// `cta2` selects the CTA-pair variants (256-row tiles, cluster of 2, grid even).
+bool tc_dense_has(int mode, int bn, bool cta2);
+bool tc_dense2_has(int mode, int bn);
 bool tc_grouped_has(int mode, int bn);
-int tc_dense_smem(int mode, int bn);
-cudaError_t tc_dense_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
-                            int sub_tiles, int grid, cudaStream_t s);
+cudaError_t tc_dense_launch(int mode, int bn, bool cta2, const CUtensorMap& a, const CUtensorMap& b,
+                            const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
+cudaError_t tc_dense2_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+                             int sub_tiles, int grid, cudaStream_t s);
 cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
                               int grid, cudaStream_t s);
 

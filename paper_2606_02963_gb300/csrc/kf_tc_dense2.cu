@@ -1,0 +1,72 @@
+// kf_tc_dense2.cu -- dense CTA-pair instantiations of the tcgen05 fused GEMM:
+// a cluster of two CTAs computes a 256-row tile with tcgen05.mma.cta_group::2
+// (each CTA stages its own 128 rows of A and half of the B rows), which halves
+// the operand bytes each SM streams per MMA and lets a 6-8 stage ring cover the
+// TMA round trip.
+#include "kf_internal.h"
+#include "kf_tc_gemm.cuh"
+
+namespace kf {
+namespace {
+
+template <int BN, int STAGES, int MODE>
+cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int sub, int grid,
+                        cudaStream_t s) {
+  using Cfg = TcCfg<BN, STAGES, MODE, false, true>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, true>;
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  if (grid % 2 != 0) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a, b, p, static_cast<int32_t>(sub));
+}
+
+}  // namespace
+
+// Compiled CTA-pair variants: (mode, BN) -> stages
+#define KF_DENSE2_VARIANTS(X) \
+  X(kModeStore, 128, 8)       \
+  X(kModeStore, 192, 7)       \
+  X(kModeStore, 224, 7)       \
+  X(kModeStore, 256, 6)       \
+  X(kModeLse, 128, 8)         \
+  X(kModeLse, 224, 7)         \
+  X(kModeLse, 256, 6)         \
+  X(kModeGroupNorm, 256, 6)
+
+bool tc_dense2_has(int mode, int bn) {
+#define X(M_, B_, S_) \
+  if (mode == M_ && bn == B_) return true;
+  KF_DENSE2_VARIANTS(X)
+#undef X
+  return false;
+}
+
+cudaError_t tc_dense2_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+                             int sub, int grid, cudaStream_t s) {
+#define X(M_, B_, S_) \
+  if (mode == M_ && bn == B_) return launch_pair<B_, S_, M_>(a, b, p, sub, grid, s);
+  KF_DENSE2_VARIANTS(X)
+#undef X
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace kf

@@ -38,12 +38,17 @@ __host__ __device__ constexpr int pow2_at_least(int x) {
   return x <= 32 ? 32 : x <= 64 ? 64 : x <= 128 ? 128 : x <= 256 ? 256 : 512;
 }
 
-template <int BN, int STAGES, int MODE, bool GROUPED>
+template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2>
 struct TcCfg {
   static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN");
+  static_assert(!(GROUPED && CTA2), "grouped GEMMs use single-CTA tiles");
   static constexpr int kOutN = (MODE == kModeSwiglu) ? BN / 2 : BN;  // output columns of a (sub)tile
-  static constexpr int kBBytes = BN * kBK * 2;
+  // With CTA pairs each CTA stages its own 128 rows of A and half of the BN rows of B.
+  static constexpr int kBRows = CTA2 ? BN / 2 : BN;
+  static constexpr int kBBytes = kBRows * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr uint32_t kTxBytes = (CTA2 ? 2 : 1) * kStageBytes;  // bytes landing per stage on the leader's barrier
+  static constexpr int kRowsPerUnit = CTA2 ? 2 * kBM : kBM;
   // accumulator buffer b starts at TMEM column b * kAccStride
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
@@ -54,24 +59,24 @@ struct TcCfg {
   // pad to > half of the SM's shared memory so that at most one such CTA is
   // resident per SM (tensor-memory allocation then never has to wait)
   static constexpr int kSmemBytes = 1024 + (kSmemUse > 120 * 1024 ? kSmemUse : 120 * 1024);
-  static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN);
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(CTA2 ? 2 * kBM : kBM, BN);
   static_assert(kSmemBytes <= 232448, "shared memory");
-  static_assert(kBBytes % 1024 == 0, "B stage alignment");
+  static_assert(kBBytes % 1024 == 0 && (BN / 2) % 8 == 0, "B stage alignment");
 };
 
 struct UnitInfo {
   int32_t m0, m_end, n0, g, n_blk;
 };
 
-template <int BN, int STAGES, int MODE, bool GROUPED>
+template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2>
 __global__ void __launch_bounds__(kThreads, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ TcParams p, const int32_t sub_tiles) {
-  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED>;
+  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CTA2>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* smA = sm;
-  uint8_t* smB = sm + STAGES * kABytes;
+  uint8_t* smB = sm;                                // B stages first: any over-read stays inside the CTA
+  uint8_t* smA = sm + STAGES * Cfg::kBBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + STAGES * Cfg::kStageBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
@@ -88,6 +93,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = CTA2 ? cluster_ctarank() : 0u;  // 0 = leader of the CTA pair (issues the MMAs)
+  const bool leader = rank == 0;
+  const int32_t unit0 = CTA2 ? static_cast<int32_t>(blockIdx.x >> 1) : static_cast<int32_t>(blockIdx.x);
+  const int32_t unit_step = CTA2 ? static_cast<int32_t>(gridDim.x >> 1) : static_cast<int32_t>(gridDim.x);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -96,7 +105,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&accf[a], 1);
-      mbar_init(&acce[a], kEpiWarps);
+      mbar_init(&acce[a], kEpiWarps * (CTA2 ? 2 : 1));
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -111,8 +120,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp == 1) {
     __syncwarp();
-    tmem_alloc(tmem_slot, Cfg::kTmemCols);
-    tmem_relinquish();
+    if constexpr (CTA2) {
+      tmem_alloc_pair(tmem_slot, Cfg::kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, Cfg::kTmemCols);
+      tmem_relinquish();
+    }
   }
   if constexpr (GROUPED) {
     if (threadIdx.x == 64) {
@@ -141,6 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (CTA2) cluster_sync();  // peer barriers initialised, TMEM allocated in both CTAs
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int32_t total = *total_s;
@@ -169,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int32_t mb = u % p.tiles_m;
       r.n_blk = u / p.tiles_m;
       r.g = 0;
-      r.m0 = mb * kBM;
+      r.m0 = mb * Cfg::kRowsPerUnit + static_cast<int32_t>(rank) * kBM;  // this CTA's 128 rows
       r.m_end = min(p.M, r.m0 + kBM);
       r.n0 = r.n_blk * Cfg::kOutN * sub_tiles;
     }
@@ -181,10 +196,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int32_t it = 0;
       bool ok = true;
-      for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
+      for (int32_t u = unit0; ok && u < total; u += unit_step) {
         const UnitInfo ui = decode(u);
         for (int s = 0; ok && s < sub_tiles; ++s) {
-          const int32_t nb0 = ui.n0 + s * BN;
+          const int32_t nb0 = ui.n0 + s * BN + static_cast<int32_t>(rank) * Cfg::kBRows;
           for (int32_t kb = 0; kb < p.num_kb; ++kb) {
             const int st = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1;
@@ -194,31 +209,47 @@ __global__ void __launch_bounds__(kThreads, 1)
               ok = false;
               break;
             }
-            mbar_arrive_expect_tx(&full[st], Cfg::kStageBytes);
-            tma_load_2d(smA + st * kABytes, &tmA, &full[st], kb * kBK, ui.m0);
+            uint8_t* a = smA + st * kABytes;
             uint8_t* b = smB + st * Cfg::kBBytes;
-            if constexpr (MODE == kModeSwiglu) {
-              tma_load_3d(b, &tmB, &full[st], kb * kBK, ui.n0, ui.g);
-              tma_load_3d(b + Cfg::kOutN * 128, &tmB, &full[st], kb * kBK, p.b_rows + ui.n0, ui.g);
+            if constexpr (CTA2) {
+              // both CTAs' copies complete on the leader's full barrier
+              if (leader) mbar_arrive_expect_tx(&full[st], Cfg::kTxBytes);
+              const uint32_t fb = mapa_shared(smem_u32(&full[st]), 0);
+              tma_load_2d_pair(a, &tmA, fb, kb * kBK, ui.m0);
+              tma_load_3d_pair(b, &tmB, fb, kb * kBK, nb0, ui.g);
             } else {
-              tma_load_3d(b, &tmB, &full[st], kb * kBK, nb0, ui.g);
+              mbar_arrive_expect_tx(&full[st], Cfg::kTxBytes);
+              tma_load_2d(a, &tmA, &full[st], kb * kBK, ui.m0);
+              if constexpr (MODE == kModeSwiglu) {
+                tma_load_3d(b, &tmB, &full[st], kb * kBK, ui.n0, ui.g);
+                tma_load_3d(b + Cfg::kOutN * 128, &tmB, &full[st], kb * kBK, p.b_rows + ui.n0, ui.g);
+              } else {
+                tma_load_3d(b, &tmB, &full[st], kb * kBK, nb0, ui.g);
+              }
             }
             ++it;
           }
         }
       }
       if (!ok) {
-        // wait (bounded) for the copies still in flight before the CTA exits
-        for (int32_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
-          mbar_wait(&full[j % STAGES], (j / STAGES) & 1, zero_flag, p.drain_ns);
+        if (!CTA2 || leader) {
+          // wait (bounded) for the copies still in flight before the CTA exits
+          for (int32_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
+            mbar_wait(&full[j % STAGES], (j / STAGES) & 1, zero_flag, p.drain_ns);
+        } else {
+          // the peer's copies complete on the leader's barrier: give them time to land
+          const uint64_t t0 = globaltimer_ns();
+          while (globaltimer_ns() - t0 < 100000ull) {
+          }
+        }
       }
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------------- MMA
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       int32_t it = 0, tl = 0;
       bool ok = true;
-      for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
+      for (int32_t u = unit0; ok && u < total; u += unit_step) {
         for (int s = 0; ok && s < sub_tiles; ++s) {
           const int acc = tl & 1;
           if (!mbar_wait(&acce[acc], ((tl >> 1) & 1) ^ 1, abort_flag, p.wait_ns)) {
@@ -239,21 +270,34 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t b0 = smem_u32(smB + st * Cfg::kBBytes);
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {
-              tc_mma_bf16(d, desc_sw128_kmajor(a0 + kk * 32), desc_sw128_kmajor(b0 + kk * 32), Cfg::kIdesc,
-                          (kb | kk) != 0 ? 1u : 0u);
+              const uint64_t ad = desc_sw128_kmajor(a0 + kk * 32), bd = desc_sw128_kmajor(b0 + kk * 32);
+              if constexpr (CTA2)
+                tc_mma_bf16_pair(d, ad, bd, Cfg::kIdesc, (kb | kk) != 0 ? 1u : 0u);
+              else
+                tc_mma_bf16(d, ad, bd, Cfg::kIdesc, (kb | kk) != 0 ? 1u : 0u);
             }
-            tc_commit(&empty[st]);
+            if constexpr (CTA2)
+              tc_commit_pair_mc(&empty[st], 0x3);  // frees the slot in both CTAs
+            else
+              tc_commit(&empty[st]);
             ++it;
           }
           if (!ok) break;
-          tc_commit(&accf[acc]);
+          if constexpr (CTA2)
+            tc_commit_pair_mc(&accf[acc], 0x3);
+          else
+            tc_commit(&accf[acc]);
           ++tl;
         }
       }
       if (!ok) {
         *abort_flag = 1;
         atomicOr(p.err, kErrWaitMma);
-        tc_commit(drain);  // arrives once every MMA issued so far has completed
+        // arrives once every MMA issued so far has completed
+        if constexpr (CTA2)
+          tc_commit_pair(drain);
+        else
+          tc_commit(drain);
         mbar_wait(drain, 0, zero_flag, p.drain_ns);
       }
     }
@@ -287,7 +331,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto release_acc = [&](int32_t t) {
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&acce[t & 1]);
+      if (lane == 0) {
+        if (CTA2 && !leader)
+          mbar_arrive_remote(mapa_shared(smem_u32(&acce[t & 1]), 0));
+        else
+          mbar_arrive(&acce[t & 1]);
+      }
     };
     // the two warps of this quadrant meet here (named barrier 1 + q, 64 threads)
     auto pair_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(1 + q), "r"(64) : "memory"); };
@@ -315,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       qq = qa + qb + d * d * (na * nb / n);
     };
 
-    for (int32_t u = blockIdx.x; ok && u < total; u += gridDim.x) {
+    for (int32_t u = unit0; ok && u < total; u += unit_step) {
       const UnitInfo ui = decode(u);
       const int32_t grow = ui.m0 + row_in_tile;
       const bool row_ok = grow < ui.m_end;
@@ -524,10 +573,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ---------------------------------------------------------------- teardown
   tc_fence_before();
   __syncthreads();
+  if constexpr (CTA2) cluster_sync();  // no remote access to this CTA remains
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, Cfg::kTmemCols);
+    if constexpr (CTA2)
+      tmem_dealloc_pair(tmem, Cfg::kTmemCols);
+    else
+      tmem_dealloc(tmem, Cfg::kTmemCols);
   }
 }
 

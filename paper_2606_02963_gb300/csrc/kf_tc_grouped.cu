@@ -8,15 +8,16 @@ namespace {
 
 template <int BN, int STAGES, int MODE>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid, cudaStream_t s) {
-  using Cfg = TcCfg<BN, STAGES, MODE, true>;
-  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true>;
-  static int configured_dev = -1;
+  using Cfg = TcCfg<BN, STAGES, MODE, true, false>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, false>;
+  static bool configured[64] = {};  // the attribute is per device
   int dev = 0;
   cudaGetDevice(&dev);
-  if (configured_dev != dev) {
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
     if (e != cudaSuccess) return e;
-    configured_dev = dev;
+    configured[dev] = true;
   }
   kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, p, 1);
   return cudaGetLastError();
