@@ -195,6 +195,21 @@ kf_status plan_chain(const kf_epilogue* epi, int64_t N, bool grouped, ChainPlan*
 }
 
 void fill_params_common(TcParams& p, const ChainPlan& pl, uint32_t* err) {
+  // a single bf16 residual operand in the pre-chain is staged through shared
+  // memory with coalesced loads (a second one would need its own buffer)
+  int nres = 0, ires = -1;
+  for (int i = 0; i < pl.n_pre; ++i)
+    if (pl.pre[i].kind == KF_OP_RESIDUAL_ADD) {
+      ++nres;
+      ires = i;
+    }
+  p.res_op = (nres == 1 && pl.pre[ires].p_dtype == KF_BF16 && pl.pre[ires].vec_ok) ? ires : -1;
+  // the first bf16 per-column vector (bias / mul) of the pre-chain is loaded ahead
+  p.vec_op = -1;
+  for (int i = 0; i < pl.n_pre && p.vec_op < 0; ++i)
+    if ((pl.pre[i].kind == KF_OP_BIAS || pl.pre[i].kind == KF_OP_MUL) && pl.pre[i].p_dtype == KF_BF16 &&
+        pl.pre[i].vec_ok)
+      p.vec_op = i;
   p.n_pre = pl.n_pre;
   p.n_post = pl.n_post;
   for (int i = 0; i < pl.n_pre; ++i) p.pre[i] = pl.pre[i];

@@ -12,7 +12,7 @@
 namespace kf {
 
 constexpr int kMaxOps = 8;
-constexpr int kMaxGroups = 1024;  // grouped GEMM: row groups (experts)
+constexpr int kMaxGroups = 512;   // grouped GEMM: row groups (experts)
 
 // error-word bits
 constexpr uint32_t kErrWaitProducer = 1u;
@@ -69,11 +69,9 @@ struct TcParams {
   uint64_t wait_ns;
   uint64_t drain_ns;
   int32_t fast;         // reduced-precision activations (result stored as bf16)
+  int32_t res_op;       // index in pre[] of a bf16 RESIDUAL_ADD staged by coalesced loads, or -1
+  int32_t vec_op;       // index in pre[] of a bf16 BIAS / MUL whose vector is loaded ahead, or -1
 };
-
-// dispatch the chain on the runtime `fast` flag (uniform across the CTA)
-__device__ __forceinline__ void apply_chain32_rt(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row,
-                                                 int64_t col0, int nvalid, bool row_ok);
 
 // ---------------------------------------------------------------- loads/stores
 __device__ __forceinline__ float ld_elem(const void* p, int dt, int64_t i) {
@@ -174,13 +172,117 @@ __device__ __forceinline__ void st32(void* p, int dt, int64_t i0, int nvalid, bo
   }
 }
 
+// ------------------------------------------- warp-cooperative 32x32 bf16 tiles
+// A warp owns 32 rows (one per lane) x 32 columns.  Global traffic is made
+// coalesced by passing the tile through a 2 KB shared buffer: for global
+// accesses lane t handles 16 bytes of row 8i + t/4 (four lanes per 64-byte
+// row segment); for registers lane r owns row r.  The 16-byte unit u of row r
+// is stored at unit u ^ ((r >> 1) & 3) of that row, which makes both the
+// row-per-lane and the 4-lanes-per-row access patterns bank-conflict free.
+__device__ __forceinline__ uint32_t xpose_off(int row, int unit) {
+  return static_cast<uint32_t>(row * 64 + ((unit ^ ((row >> 1) & 3)) << 4));
+}
+
+// Store the lane's 32 values (row `lane`) as bf16 to dst rows [0, rows) of a
+// 32 x 32 block whose first element is `gbase` (row stride ld elements).
+__device__ __forceinline__ void store_tile32_bf16(uint8_t* stage, int lane, const float (&v)[32], void* gbase,
+                                                  int64_t ld, int rows) {
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    uint4 w;
+    w.x = pack_bf16x2(v[8 * u + 0], v[8 * u + 1]);
+    w.y = pack_bf16x2(v[8 * u + 2], v[8 * u + 3]);
+    w.z = pack_bf16x2(v[8 * u + 4], v[8 * u + 5]);
+    w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
+    *reinterpret_cast<uint4*>(stage + xpose_off(lane, u)) = w;
+  }
+  __syncwarp();
+  const int u = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = 8 * i + (lane >> 2);
+    const uint4 w = *reinterpret_cast<const uint4*>(stage + xpose_off(r, u));
+    if (r < rows) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(gbase) + r * ld + 8 * u) = w;
+  }
+  __syncwarp();
+}
+
+// 16-byte read-only load issued where it is written: volatile, so the compiler
+// cannot sink it past the accumulator wait that follows (the point of issuing
+// it early is to overlap its latency with that wait).
+__device__ __forceinline__ uint4 ldg_v4_pinned(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(reinterpret_cast<uint64_t>(p)));
+  return r;
+}
+
+// Issue the coalesced loads of rows [0, rows) of a 32 x 32 bf16 block into
+// registers (lane t: 16 bytes of row 8i + t/4); rows >= `rows` read as 0.
+__device__ __forceinline__ void tile32_issue(const void* gbase, int64_t ld, int rows, int lane, uint4 (&q)[4]) {
+  const int u = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = 8 * i + (lane >> 2);
+    q[i] = make_uint4(0, 0, 0, 0);
+    if (r < rows) q[i] = ldg_v4_pinned(reinterpret_cast<const __nv_bfloat16*>(gbase) + r * ld + 8 * u);
+  }
+}
+// Pass loaded blocks through the shared buffer; row `lane` comes back as 16
+// packed bf16 pairs (element 2k in the low half of o[k]).
+__device__ __forceinline__ void tile32_finish(uint8_t* stage, int lane, const uint4 (&q)[4], uint32_t (&o)[16]) {
+  const int u = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) *reinterpret_cast<uint4*>(stage + xpose_off(8 * i + (lane >> 2), u)) = q[i];
+  __syncwarp();
+#pragma unroll
+  for (int uu = 0; uu < 4; ++uu) {
+    const uint4 w = *reinterpret_cast<const uint4*>(stage + xpose_off(lane, uu));
+    o[4 * uu] = w.x;
+    o[4 * uu + 1] = w.y;
+    o[4 * uu + 2] = w.z;
+    o[4 * uu + 3] = w.w;
+  }
+  __syncwarp();
+}
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+// 32 consecutive bf16 of a per-column vector (same for every lane)
+__device__ __forceinline__ void vec32_issue(const void* p, int64_t i0, uint4 (&q)[4]) {
+  const __nv_bfloat16* a = reinterpret_cast<const __nv_bfloat16*>(p) + i0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) q[i] = ldg_v4_pinned(a + 8 * i);
+}
+__device__ __forceinline__ void pack16(const uint4 (&q)[4], uint32_t (&o)[16]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    o[4 * i] = q[i].x;
+    o[4 * i + 1] = q[i].y;
+    o[4 * i + 2] = q[i].z;
+    o[4 * i + 3] = q[i].w;
+  }
+}
+
+// Operands of one 32-column chunk that the caller loaded ahead of time: the
+// row's residual chunk (for pre[res_op]) and a per-column vector (for pre[vec_op]).
+struct Staged32 {
+  uint32_t res[16];  // packed bf16 pairs
+  uint32_t vec[16];  // packed bf16 pairs
+  bool use_res;
+  int vec_idx;  // op index whose operand is vec[], or -1
+};
+
 // ------------------------------------------------------------ element-wise ops
-__device__ __forceinline__ float f_sigmoid(float x) { return 1.0f / (1.0f + expf(-x)); }
-__device__ __forceinline__ float f_gelu_tanh(float x) {
+// The accurate forms (fp32 results) are kept out of line: the op interpreter is
+// unrolled over 32 columns at several call sites, and inlining the library
+// transcendentals there would multiply the kernel's code size.
+static __device__ __noinline__ float f_sigmoid(float x) { return 1.0f / (1.0f + expf(-x)); }
+static __device__ __noinline__ float f_gelu_tanh(float x) {
   const float c = 0.7978845608028654f;  // sqrt(2/pi)
   return 0.5f * x * (1.0f + tanhf(c * (x + 0.044715f * x * x * x)));
 }
-__device__ __forceinline__ float f_mish(float x) {
+static __device__ __noinline__ float f_mish(float x) {
   float sp = x > 20.0f ? x : log1pf(expf(x));
   return x * tanhf(sp);
 }
@@ -199,7 +301,7 @@ __device__ __forceinline__ float f_gelu_tanh_fast(float x) {
   const float hx = 0.5f * x;
   return fmaf(hx, tanh_fast(c * fmaf(0.044715f * x, x * x, x)), hx);
 }
-__device__ __forceinline__ float f_mish_fast(float x) {
+static __device__ __noinline__ float f_mish_fast(float x) {
   float sp = x > 15.0f ? x : __logf(1.0f + __expf(x));
   return x * tanh_fast(sp);
 }
@@ -224,16 +326,27 @@ __device__ __forceinline__ float apply_scalar_op(const DevOp& op, float x) {
 // first `nvalid` columns exist).  Operands of rows that do not exist are not
 // read (row_ok == false).  FAST selects the reduced-precision activations (for
 // chains whose result is stored as bf16).
+// `st` holds operands the caller loaded ahead of time: the RESIDUAL_ADD op uses
+// st.res when st.use_res, and op st.vec_idx uses st.vec as its per-column vector;
+// other operands are loaded here.
 template <bool FAST>
 __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
-                                              int nvalid, bool row_ok) {
+                                              int nvalid, bool row_ok, const Staged32& st) {
   for (int o = 0; o < n; ++o) {
     const DevOp& op = ops[o];
     switch (op.kind) {
       case KF_OP_BIAS:
       case KF_OP_MUL: {
         float b[32];
-        ld32(op.p0, op.p_dtype, col0, nvalid, op.vec_ok != 0, b);
+        if (o == st.vec_idx) {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            b[2 * k] = bf16lo(st.vec[k]);
+            b[2 * k + 1] = bf16hi(st.vec[k]);
+          }
+        } else {
+          ld32(op.p0, op.p_dtype, col0, nvalid, op.vec_ok != 0, b);
+        }
         if (op.kind == KF_OP_BIAS) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] += b[j];
@@ -243,7 +356,13 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
         }
       } break;
       case KF_OP_RESIDUAL_ADD: {
-        if (row_ok) {
+        if (st.use_res) {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            v[2 * k] += bf16lo(st.res[k]);
+            v[2 * k + 1] += bf16hi(st.res[k]);
+          }
+        } else if (row_ok) {
           float r[32];
           ld32(op.p0, op.p_dtype, row * op.ld + col0, nvalid, op.vec_ok != 0, r);
 #pragma unroll
@@ -286,12 +405,19 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
 }
 
 __device__ __forceinline__ void apply_chain32_rt(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row,
-                                                 int64_t col0, int nvalid, bool row_ok) {
-  if (n == 0) return;
+                                                 int64_t col0, int nvalid, bool row_ok, const Staged32& st) {
+  if (n <= 0) return;
   if (fast)
-    apply_chain32<true>(ops, n, v, row, col0, nvalid, row_ok);
+    apply_chain32<true>(ops, n, v, row, col0, nvalid, row_ok, st);
   else
-    apply_chain32<false>(ops, n, v, row, col0, nvalid, row_ok);
+    apply_chain32<false>(ops, n, v, row, col0, nvalid, row_ok, st);
+}
+__device__ __forceinline__ void apply_chain32_rt(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row,
+                                                 int64_t col0, int nvalid, bool row_ok) {
+  Staged32 none;
+  none.use_res = false;
+  none.vec_idx = -1;
+  apply_chain32_rt(fast, ops, n, v, row, col0, nvalid, row_ok, none);
 }
 
 }  // namespace kf

@@ -45,10 +45,10 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const TcPara
 #define KF_DENSE2_VARIANTS(X) \
   X(kModeStore, 128, 8)       \
   X(kModeStore, 192, 7)       \
-  X(kModeStore, 224, 7)       \
+  X(kModeStore, 224, 6)       \
   X(kModeStore, 256, 6)       \
   X(kModeLse, 128, 8)         \
-  X(kModeLse, 224, 7)         \
+  X(kModeLse, 224, 6)         \
   X(kModeLse, 256, 6)         \
   X(kModeGroupNorm, 256, 6)
 

@@ -53,7 +53,8 @@ struct TcCfg {
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
   static constexpr int kBarBytes = (8 * (2 * STAGES + 5) + 63) / 64 * 64;  // keeps what follows 64-B aligned
-  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16;  // flags + epilogue exchange buffer
+  // flags + row-statistics exchange (4 KB) + per-warp 2 KB transpose buffers
+  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16 + kEpiWarps * 2048;
   static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
   static constexpr int kSmemUse = STAGES * kStageBytes + kBarBytes + kMiscBytes + kTableBytes;
   // pad to > half of the SM's shared memory so that at most one such CTA is
@@ -154,6 +155,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   tc_fence_before();
+  // __syncthreads is an aligned barrier: every warp must reach it converged,
+  // or a warp whose lanes arrive at different times is counted too early
+  __syncwarp();
   __syncthreads();
   if constexpr (CTA2) cluster_sync();  // peer barriers initialised, TMEM allocated in both CTAs
   tc_fence_after();
@@ -314,6 +318,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const bool fast = p.fast != 0;
     float4* xch = reinterpret_cast<float4*>(misc + 16);  // [2 halves][4 quadrants][32 lanes]
+    uint8_t* stage = reinterpret_cast<uint8_t*>(misc) + 64 + 2 * 4 * 32 * 16 + ew * 2048;  // this warp's tile buffer
+    const bool res_staged = MODE == kModeStore && p.res_op >= 0;
+    const bool vec_staged = MODE == kModeStore && p.vec_op >= 0;
+    const bool c_tiles = p.c_dtype == KF_BF16 && p.c_vec_ok != 0;
     int32_t tl = 0;
     bool ok = true;
 
@@ -368,8 +376,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const UnitInfo ui = decode(u);
       const int32_t grow = ui.m0 + row_in_tile;
       const bool row_ok = grow < ui.m_end;
+      const int32_t wrow0 = ui.m0 + q * 32;                      // first row of this warp's 32
+      const int wrows = max(0, min(32, ui.m_end - wrow0));       // rows of them that exist
+      // pull this unit's residual rows toward L2 while its mainloop runs
+      if (res_staged && row_ok) {
+        const DevOp& ro = p.pre[p.res_op];
+        const __nv_bfloat16* rp = reinterpret_cast<const __nv_bfloat16*>(ro.p0) + static_cast<int64_t>(grow) * ro.ld;
+        for (int c = h + 2; c < Cfg::kOutN / 32; c += 2)
+          if (ui.n0 + c * 32 < p.N) prefetch_l2(rp + ui.n0 + c * 32);
+      }
 
       if constexpr (MODE == kModeStore || MODE == kModeSwiglu || MODE == kModeScatter) {
+        // loads of the residual / bias chunk next in line (in flight across the wait)
+        uint4 rq[4], bq[4];
+        auto issue_chunk = [&](int c) {
+          const int32_t col0 = ui.n0 + c * 32;
+          if (c >= Cfg::kOutN / 32 || p.N - col0 < 32) return;
+          if (res_staged) {
+            const DevOp& ro = p.pre[p.res_op];
+            tile32_issue(reinterpret_cast<const __nv_bfloat16*>(ro.p0) + static_cast<int64_t>(wrow0) * ro.ld + col0,
+                         ro.ld, wrows, lane, rq);
+          }
+          if (vec_staged) vec32_issue(p.pre[p.vec_op].p0, col0, bq);
+        };
+        if constexpr (MODE == kModeStore) issue_chunk(h);
         if (!wait_acc(tl)) { ok = false; break; }
         const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
         float rs = 0.0f;
@@ -391,7 +421,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (nvalid <= 0) break;  // uniform across the warp
           __syncwarp();
           float v[32];
-          if constexpr (MODE == kModeSwiglu) {
+          if constexpr (MODE == kModeStore) {
+            // operands of this chunk were issued one chunk ahead; issue the next
+            Staged32 sg;
+            sg.use_res = res_staged && nvalid == 32;
+            sg.vec_idx = (vec_staged && nvalid == 32) ? p.vec_op : -1;
+            if (sg.use_res) tile32_finish(stage, lane, rq, sg.res);
+            if (sg.vec_idx >= 0) pack16(bq, sg.vec);
+            issue_chunk(c + 2);
+            tmem_ld32(tb + c * 32, v);
+            apply_chain32_rt(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok, sg);
+          } else if constexpr (MODE == kModeSwiglu) {
             float gt[32];
             tmem_ld32(tb + c * 32, gt);
             tmem_ld32(tb + Cfg::kOutN + c * 32, v);
@@ -421,6 +461,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                   if (j < nvalid) atomicAdd(dstp + j, v[j] * rs);
               }
             }
+          } else if (c_tiles && nvalid == 32) {
+            store_tile32_bf16(stage, lane, v,
+                              reinterpret_cast<__nv_bfloat16*>(p.C) + static_cast<int64_t>(wrow0) * p.ldc + col0, p.ldc,
+                              wrows);
           } else {
             if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, nvalid, p.c_vec_ok != 0, v);
           }
@@ -487,33 +531,34 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           apply_chain32_rt(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
-          if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
+          if (c_tiles)
+            store_tile32_bf16(stage, lane, v,
+                              reinterpret_cast<__nv_bfloat16*>(p.C) + static_cast<int64_t>(wrow0) * p.ldc + col0, p.ldc,
+                              wrows);
+          else if (row_ok)
+            st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, 32, p.c_vec_ok != 0, v);
         };
-        // exact two-pass moments (count, mean, M2) of this thread's chunks c0, c0+step, ... < c1
+        // (count, mean, M2) of this thread's chunks c0, c0+step, ... < c1 in one pass over
+        // TMEM: exact two-pass moments of each 32-value chunk in registers, merged
+        // chunk by chunk with Chan's formula.
         auto moments = [&](uint32_t tb, int32_t colbase, int c0, int c1, int step, float& n, float& mean, float& m2) {
-          float sum = 0.0f;
-          int cnt = 0;
+          n = 0.0f;
+          mean = 0.0f;
+          m2 = 0.0f;
           for (int c = c0; c < c1; c += step) {
             __syncwarp();
             float v[32];
             tmem_ld32(tb + c * 32, v);
             apply_chain32_rt(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+            float sum = 0.0f;
 #pragma unroll
             for (int j = 0; j < 32; ++j) sum += v[j];
-            ++cnt;
-          }
-          n = 32.0f * cnt;
-          mean = cnt ? sum / n : 0.0f;
-          float qq = 0.0f;
-          for (int c = c0; c < c1; c += step) {
-            __syncwarp();
-            float v[32];
-            tmem_ld32(tb + c * 32, v);
-            apply_chain32_rt(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+            const float cmean = sum * (1.0f / 32.0f);
+            float cq = 0.0f;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) qq += (v[j] - mean) * (v[j] - mean);
+            for (int j = 0; j < 32; ++j) cq += (v[j] - cmean) * (v[j] - cmean);
+            chan(n, mean, m2, 32.0f, cmean, cq, n, mean, m2);
           }
-          m2 = qq;
         };
         if (gs < BN) {
           // several whole groups per tile: half h takes groups h, h+2, ...
@@ -572,6 +617,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---------------------------------------------------------------- teardown
   tc_fence_before();
+  __syncwarp();  // lane 0 of the producer / MMA warps arrives after lanes 1-31
   __syncthreads();
   if constexpr (CTA2) cluster_sync();  // no remote access to this CTA remains
   if (warp == 1) {
