@@ -466,7 +466,15 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   fill_params_common(p, pl, di.err);
   p.fast = yt == KF_BF16 && pl.mode != kModeLse;  // bf16 results: reduced-precision activations suffice
   const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
-  st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, ma, mb, p, sub, grid, s));
+  // a compiled chain program, if the chain matches one (bf16 operands staged)
+  int sig = kSigGeneric;
+  if (pl.mode == kModeStore && ProgGeluChain::matches(pl.pre, pl.n_pre) && p.vec_op == 0 && p.res_op == 3)
+    sig = kSigBiasGeluScaleRes;
+  else if (pl.mode == kModeGroupNorm && ProgBias::matches(pl.pre, pl.n_pre) && ProgSilu::matches(pl.post, pl.n_post))
+    sig = kSigBiasNormSilu;
+  else if (pl.mode == kModeLse && ProgScale::matches(pl.pre, pl.n_pre))
+    sig = kSigScaleLse;
+  st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, p, sub, grid, s));
   if (st != KF_OK || pl.mode != kModeLse) return st;
   LseCombineParams cp;
   std::memset(&cp, 0, sizeof(cp));

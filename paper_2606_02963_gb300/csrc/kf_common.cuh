@@ -5,6 +5,7 @@
 // is still on chip, in fp32).
 #pragma once
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cstdint>
 
 #include "../../include/kf.h"
@@ -174,37 +175,43 @@ __device__ __forceinline__ void st32(void* p, int dt, int64_t i0, int nvalid, bo
 
 // ------------------------------------------- warp-cooperative 32x32 bf16 tiles
 // A warp owns 32 rows (one per lane) x 32 columns.  Global traffic is made
-// coalesced by passing the tile through a 2 KB shared buffer: for global
-// accesses lane t handles 16 bytes of row 8i + t/4 (four lanes per 64-byte
-// row segment); for registers lane r owns row r.  The 16-byte unit u of row r
-// is stored at unit u ^ ((r >> 1) & 3) of that row, which makes both the
-// row-per-lane and the 4-lanes-per-row access patterns bank-conflict free.
+// coalesced by passing the tile through a 1 KB shared buffer, 16 columns (32 B
+// per row) at a time: for global accesses lane t handles 16 bytes of row
+// 16i + t/2 (two lanes per 32-byte row segment, one full sector); for
+// registers lane r owns row r.  The 16-byte unit u of row r is stored at unit
+// u ^ ((r >> 2) & 1) of that row, which makes both access patterns free of
+// shared-memory bank conflicts.
 __device__ __forceinline__ uint32_t xpose_off(int row, int unit) {
-  return static_cast<uint32_t>(row * 64 + ((unit ^ ((row >> 1) & 3)) << 4));
+  return static_cast<uint32_t>(row * 32 + ((unit ^ ((row >> 2) & 1)) << 4));
 }
 
-// Store the lane's 32 values (row `lane`) as bf16 to dst rows [0, rows) of a
-// 32 x 32 block whose first element is `gbase` (row stride ld elements).
+// Store the lane's 32 values (row `lane`) as bf16 to rows [0, rows) of the
+// 32 x 32 block at `gbase` (row stride ld elements).
 __device__ __forceinline__ void store_tile32_bf16(uint8_t* stage, int lane, const float (&v)[32], void* gbase,
                                                   int64_t ld, int rows) {
+  const int u = lane & 1;
 #pragma unroll
-  for (int u = 0; u < 4; ++u) {
-    uint4 w;
-    w.x = pack_bf16x2(v[8 * u + 0], v[8 * u + 1]);
-    w.y = pack_bf16x2(v[8 * u + 2], v[8 * u + 3]);
-    w.z = pack_bf16x2(v[8 * u + 4], v[8 * u + 5]);
-    w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
-    *reinterpret_cast<uint4*>(stage + xpose_off(lane, u)) = w;
-  }
-  __syncwarp();
-  const int u = lane & 3;
+  for (int half = 0; half < 2; ++half) {
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int r = 8 * i + (lane >> 2);
-    const uint4 w = *reinterpret_cast<const uint4*>(stage + xpose_off(r, u));
-    if (r < rows) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(gbase) + r * ld + 8 * u) = w;
+    for (int uu = 0; uu < 2; ++uu) {
+      const int c = 16 * half + 8 * uu;
+      uint4 w;
+      w.x = pack_bf16x2(v[c + 0], v[c + 1]);
+      w.y = pack_bf16x2(v[c + 2], v[c + 3]);
+      w.z = pack_bf16x2(v[c + 4], v[c + 5]);
+      w.w = pack_bf16x2(v[c + 6], v[c + 7]);
+      *reinterpret_cast<uint4*>(stage + xpose_off(lane, uu)) = w;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int r = 16 * i + (lane >> 1);
+      const uint4 w = *reinterpret_cast<const uint4*>(stage + xpose_off(r, u));
+      if (r < rows)
+        *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(gbase) + r * ld + 16 * half + 8 * u) = w;
+    }
+    __syncwarp();
   }
-  __syncwarp();
 }
 
 // 16-byte read-only load issued where it is written: volatile, so the compiler
@@ -219,32 +226,40 @@ __device__ __forceinline__ uint4 ldg_v4_pinned(const void* p) {
 }
 
 // Issue the coalesced loads of rows [0, rows) of a 32 x 32 bf16 block into
-// registers (lane t: 16 bytes of row 8i + t/4); rows >= `rows` read as 0.
+// registers: q[2*half + i] is 16 bytes of row 16i + t/2, columns
+// 16*half + 8*(t&1) ..; rows >= `rows` read as 0.
 __device__ __forceinline__ void tile32_issue(const void* gbase, int64_t ld, int rows, int lane, uint4 (&q)[4]) {
-  const int u = lane & 3;
+  const int u = lane & 1;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int r = 8 * i + (lane >> 2);
-    q[i] = make_uint4(0, 0, 0, 0);
-    if (r < rows) q[i] = ldg_v4_pinned(reinterpret_cast<const __nv_bfloat16*>(gbase) + r * ld + 8 * u);
-  }
+  for (int half = 0; half < 2; ++half)
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int r = 16 * i + (lane >> 1);
+      q[2 * half + i] = make_uint4(0, 0, 0, 0);
+      if (r < rows)
+        q[2 * half + i] = ldg_v4_pinned(reinterpret_cast<const __nv_bfloat16*>(gbase) + r * ld + 16 * half + 8 * u);
+    }
 }
 // Pass loaded blocks through the shared buffer; row `lane` comes back as 16
 // packed bf16 pairs (element 2k in the low half of o[k]).
 __device__ __forceinline__ void tile32_finish(uint8_t* stage, int lane, const uint4 (&q)[4], uint32_t (&o)[16]) {
-  const int u = lane & 3;
+  const int u = lane & 1;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) *reinterpret_cast<uint4*>(stage + xpose_off(8 * i + (lane >> 2), u)) = q[i];
-  __syncwarp();
+  for (int half = 0; half < 2; ++half) {
 #pragma unroll
-  for (int uu = 0; uu < 4; ++uu) {
-    const uint4 w = *reinterpret_cast<const uint4*>(stage + xpose_off(lane, uu));
-    o[4 * uu] = w.x;
-    o[4 * uu + 1] = w.y;
-    o[4 * uu + 2] = w.z;
-    o[4 * uu + 3] = w.w;
+    for (int i = 0; i < 2; ++i)
+      *reinterpret_cast<uint4*>(stage + xpose_off(16 * i + (lane >> 1), u)) = q[2 * half + i];
+    __syncwarp();
+#pragma unroll
+    for (int uu = 0; uu < 2; ++uu) {
+      const uint4 w = *reinterpret_cast<const uint4*>(stage + xpose_off(lane, uu));
+      o[8 * half + 4 * uu] = w.x;
+      o[8 * half + 4 * uu + 1] = w.y;
+      o[8 * half + 4 * uu + 2] = w.z;
+      o[8 * half + 4 * uu + 3] = w.w;
+    }
+    __syncwarp();
   }
-  __syncwarp();
 }
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
@@ -296,6 +311,17 @@ __device__ __forceinline__ float tanh_fast(float x) {
   return y;
 }
 __device__ __forceinline__ float f_sigmoid_fast(float x) { return fmaf(0.5f, tanh_fast(0.5f * x), 0.5f); }
+// Two tanh values with one instruction (tanh.approx.f16x2: relative error about
+// 2^-11, inputs rounded to fp16; |arguments| beyond the fp16 range saturate to
+// +-1, which is tanh's value there to fp16 precision).
+__device__ __forceinline__ void tanh2_fast(float a, float b, float& ta, float& tb) {
+  uint32_t hin, hout;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(hin) : "f"(b), "f"(a));
+  asm("tanh.approx.f16x2 %0, %1;" : "=r"(hout) : "r"(hin));
+  const __half2 h2 = *reinterpret_cast<const __half2*>(&hout);
+  ta = __low2float(h2);
+  tb = __high2float(h2);
+}
 __device__ __forceinline__ float f_gelu_tanh_fast(float x) {
   const float c = 0.7978845608028654f;
   const float hx = 0.5f * x;
@@ -379,16 +405,38 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
         for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.0f);
       } break;
       case KF_OP_GELU_TANH: {
+        if (FAST) {
+          const float c = 0.7978845608028654f;  // sqrt(2/pi)
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = FAST ? f_gelu_tanh_fast(v[j]) : f_gelu_tanh(v[j]);
-      } break;
-      case KF_OP_SILU: {
+          for (int j = 0; j < 32; j += 2) {
+            float t0, t1;
+            tanh2_fast(c * fmaf(0.044715f * v[j], v[j] * v[j], v[j]),
+                       c * fmaf(0.044715f * v[j + 1], v[j + 1] * v[j + 1], v[j + 1]), t0, t1);
+            const float h0 = 0.5f * v[j], h1 = 0.5f * v[j + 1];
+            v[j] = fmaf(h0, t0, h0);
+            v[j + 1] = fmaf(h1, t1, h1);
+          }
+        } else {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = v[j] * sigm<FAST>(v[j]);
+          for (int j = 0; j < 32; ++j) v[j] = f_gelu_tanh(v[j]);
+        }
       } break;
+      case KF_OP_SILU:
       case KF_OP_SIGMOID: {
+        if (FAST) {
+          // sigmoid(x) = (1 + tanh(x / 2)) / 2
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = sigm<FAST>(v[j]);
+          for (int j = 0; j < 32; j += 2) {
+            float t0, t1;
+            tanh2_fast(0.5f * v[j], 0.5f * v[j + 1], t0, t1);
+            const float s0 = fmaf(0.5f, t0, 0.5f), s1 = fmaf(0.5f, t1, 0.5f);
+            v[j] = op.kind == KF_OP_SILU ? v[j] * s0 : s0;
+            v[j + 1] = op.kind == KF_OP_SILU ? v[j + 1] * s1 : s1;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = op.kind == KF_OP_SILU ? v[j] * f_sigmoid(v[j]) : f_sigmoid(v[j]);
+        }
       } break;
       case KF_OP_MISH: {
 #pragma unroll
@@ -418,6 +466,130 @@ __device__ __forceinline__ void apply_chain32_rt(bool fast, const DevOp* ops, in
   none.use_res = false;
   none.vec_idx = -1;
   apply_chain32_rt(fast, ops, n, v, row, col0, nvalid, row_ok, none);
+}
+
+// ------------------------------------------------------ compiled op programs
+// A chain whose op kinds match a compiled program runs as straight-line code:
+// operand fields are read at constant offsets and there is no per-op dispatch.
+// Prog<> is the empty chain; Interp runs any chain through apply_chain32.
+template <int KIND, bool FAST>
+__device__ __forceinline__ void prog_op(const DevOp& op, float (&v)[32], int64_t row, int64_t col0, int nvalid,
+                                        bool row_ok, const Staged32& st, bool staged_vec) {
+  if constexpr (KIND == KF_OP_BIAS || KIND == KF_OP_MUL) {
+    float b[32];
+    if (staged_vec) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        b[2 * k] = bf16lo(st.vec[k]);
+        b[2 * k + 1] = bf16hi(st.vec[k]);
+      }
+    } else {
+      ld32(op.p0, op.p_dtype, col0, nvalid, op.vec_ok != 0, b);
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = KIND == KF_OP_BIAS ? v[j] + b[j] : v[j] * b[j];
+  } else if constexpr (KIND == KF_OP_RESIDUAL_ADD) {
+    if (st.use_res) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        v[2 * k] += bf16lo(st.res[k]);
+        v[2 * k + 1] += bf16hi(st.res[k]);
+      }
+    } else if (row_ok) {
+      float r[32];
+      ld32(op.p0, op.p_dtype, row * op.ld + col0, nvalid, op.vec_ok != 0, r);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] += r[j];
+    }
+  } else if constexpr (KIND == KF_OP_SCALE) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] *= op.scalar;
+  } else if constexpr (KIND == KF_OP_GELU_TANH) {
+    if constexpr (FAST) {
+      const float c = 0.7978845608028654f;
+#pragma unroll
+      for (int j = 0; j < 32; j += 2) {
+        float t0, t1;
+        tanh2_fast(c * fmaf(0.044715f * v[j], v[j] * v[j], v[j]),
+                   c * fmaf(0.044715f * v[j + 1], v[j + 1] * v[j + 1], v[j + 1]), t0, t1);
+        const float h0 = 0.5f * v[j], h1 = 0.5f * v[j + 1];
+        v[j] = fmaf(h0, t0, h0);
+        v[j + 1] = fmaf(h1, t1, h1);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = f_gelu_tanh(v[j]);
+    }
+  } else if constexpr (KIND == KF_OP_SILU) {
+    if constexpr (FAST) {
+#pragma unroll
+      for (int j = 0; j < 32; j += 2) {
+        float t0, t1;
+        tanh2_fast(0.5f * v[j], 0.5f * v[j + 1], t0, t1);
+        v[j] *= fmaf(0.5f, t0, 0.5f);
+        v[j + 1] *= fmaf(0.5f, t1, 0.5f);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] *= f_sigmoid(v[j]);
+    }
+  } else {
+    static_assert(KIND == KF_OP_BIAS, "op kind has no compiled form");
+  }
+}
+
+template <int... KINDS>
+struct Prog {
+  static constexpr int kLen = sizeof...(KINDS);
+  static constexpr bool kGeneric = false;
+  template <bool FAST>
+  __device__ __forceinline__ static void run(const DevOp* ops, float (&v)[32], int64_t row, int64_t col0, int nvalid,
+                                             bool row_ok, const Staged32& st) {
+    int i = 0;
+    ((prog_op<KINDS, FAST>(ops[i], v, row, col0, nvalid, row_ok, st, i == st.vec_idx), ++i), ...);
+  }
+  // does a runtime op list match this program?
+  __host__ static bool matches(const DevOp* ops, int n) {
+    const int kinds[] = {KINDS..., -1};
+    if (n != kLen) return false;
+    for (int i = 0; i < n; ++i)
+      if (ops[i].kind != kinds[i]) return false;
+    return true;
+  }
+};
+struct Interp {
+  static constexpr bool kGeneric = true;
+  template <bool FAST>
+  __device__ __forceinline__ static void run(const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
+                                             int nvalid, bool row_ok, const Staged32& st) {
+    apply_chain32<FAST>(ops, n, v, row, col0, nvalid, row_ok, st);
+  }
+};
+
+// Apply chain `ops[0..n)` with program P (the interpreter when P is Interp).
+template <class P>
+__device__ __forceinline__ void run_chain(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
+                                          int nvalid, bool row_ok, const Staged32& st) {
+  if constexpr (P::kGeneric) {
+    if (n <= 0) return;
+    if (fast)
+      P::template run<true>(ops, n, v, row, col0, nvalid, row_ok, st);
+    else
+      P::template run<false>(ops, n, v, row, col0, nvalid, row_ok, st);
+  } else {
+    if (fast)
+      P::template run<true>(ops, v, row, col0, nvalid, row_ok, st);
+    else
+      P::template run<false>(ops, v, row, col0, nvalid, row_ok, st);
+  }
+}
+template <class P>
+__device__ __forceinline__ void run_chain(bool fast, const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
+                                          int nvalid, bool row_ok) {
+  Staged32 none;
+  none.use_res = false;
+  none.vec_idx = -1;
+  run_chain<P>(fast, ops, n, v, row, col0, nvalid, row_ok, none);
 }
 
 }  // namespace kf

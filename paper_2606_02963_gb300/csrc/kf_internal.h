@@ -8,15 +8,29 @@
 
 namespace kf {
 
+// Compiled chain programs selectable by signature id (0 = interpreter).
+using ProgGeluChain = Prog<KF_OP_BIAS, KF_OP_GELU_TANH, KF_OP_SCALE, KF_OP_RESIDUAL_ADD>;  // bias, GELU, scale, +R
+using ProgBias = Prog<KF_OP_BIAS>;
+using ProgSilu = Prog<KF_OP_SILU>;
+using ProgScale = Prog<KF_OP_SCALE>;
+enum ChainSig : int {
+  kSigGeneric = 0,
+  kSigBiasGeluScaleRes = 1,  // store:      pre = ProgGeluChain
+  kSigBiasNormSilu = 2,      // GroupNorm:  pre = ProgBias, post = ProgSilu
+  kSigScaleLse = 3,          // row LSE:    pre = ProgScale, post = none
+};
+
 // Tensor-core GEMM launchers.  `bn` selects the tile width among the compiled
 // variants; returns cudaErrorInvalidValue for a variant that is not built.
 // `cta2` selects the CTA-pair variants (256-row tiles, cluster of 2, grid even).
+// `sig` selects a compiled chain program when one is built for (mode, bn,
+// cta2), else the interpreter variant runs.
 bool tc_dense_has(int mode, int bn, bool cta2);
 bool tc_dense2_has(int mode, int bn);
 bool tc_grouped_has(int mode, int bn);
-cudaError_t tc_dense_launch(int mode, int bn, bool cta2, const CUtensorMap& a, const CUtensorMap& b,
+cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,
                             const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
-cudaError_t tc_dense2_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
                              int sub_tiles, int grid, cudaStream_t s);
 cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
                               int grid, cudaStream_t s);

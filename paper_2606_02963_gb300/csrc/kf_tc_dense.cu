@@ -48,9 +48,9 @@ bool tc_dense_has(int mode, int bn, bool cta2) {
   return false;
 }
 
-cudaError_t tc_dense_launch(int mode, int bn, bool cta2, const CUtensorMap& a, const CUtensorMap& b,
+cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,
                             const TcParams& p, int sub, int grid, cudaStream_t s) {
-  if (cta2) return tc_dense2_launch(mode, bn, a, b, p, sub, grid, s);
+  if (cta2) return tc_dense2_launch(mode, bn, sig, a, b, p, sub, grid, s);
 #define X(M_, B_, S_) \
   if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, p, sub, grid, s);
   KF_DENSE_VARIANTS(X)

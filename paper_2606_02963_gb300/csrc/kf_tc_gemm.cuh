@@ -54,7 +54,7 @@ struct TcCfg {
   static constexpr int kTmemCols = 2 * kAccStride;
   static constexpr int kBarBytes = (8 * (2 * STAGES + 5) + 63) / 64 * 64;  // keeps what follows 64-B aligned
   // flags + row-statistics exchange (4 KB) + per-warp 2 KB transpose buffers
-  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16 + kEpiWarps * 2048;
+  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16 + kEpiWarps * 1024;
   static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
   static constexpr int kSmemUse = STAGES * kStageBytes + kBarBytes + kMiscBytes + kTableBytes;
   // pad to > half of the SM's shared memory so that at most one such CTA is
@@ -69,7 +69,9 @@ struct UnitInfo {
   int32_t m0, m_end, n0, g, n_blk;
 };
 
-template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2>
+// PRE / POST: compiled op programs (Prog<...>) for the chain before / after the
+// reduction, or Interp for arbitrary chains.
+template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2, class PRE = Interp, class POST = Interp>
 __global__ void __launch_bounds__(kThreads, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ TcParams p, const int32_t sub_tiles) {
@@ -318,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const bool fast = p.fast != 0;
     float4* xch = reinterpret_cast<float4*>(misc + 16);  // [2 halves][4 quadrants][32 lanes]
-    uint8_t* stage = reinterpret_cast<uint8_t*>(misc) + 64 + 2 * 4 * 32 * 16 + ew * 2048;  // this warp's tile buffer
+    uint8_t* stage = reinterpret_cast<uint8_t*>(misc) + 64 + 2 * 4 * 32 * 16 + ew * 1024;  // this warp's tile buffer
     const bool res_staged = MODE == kModeStore && p.res_op >= 0;
     const bool vec_staged = MODE == kModeStore && p.vec_op >= 0;
     const bool c_tiles = p.c_dtype == KF_BF16 && p.c_vec_ok != 0;
@@ -430,22 +432,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (sg.vec_idx >= 0) pack16(bq, sg.vec);
             issue_chunk(c + 2);
             tmem_ld32(tb + c * 32, v);
-            apply_chain32_rt(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok, sg);
+            run_chain<PRE>(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok, sg);
           } else if constexpr (MODE == kModeSwiglu) {
             float gt[32];
             tmem_ld32(tb + c * 32, gt);
             tmem_ld32(tb + Cfg::kOutN + c * 32, v);
             if (fast) {
+              // fp32 hardware tanh: h feeds the down GEMM, which sums 2880 of
+              // them, so it keeps more precision than a direct bf16 output needs
 #pragma unroll
               for (int j = 0; j < 32; ++j) v[j] = gt[j] * f_sigmoid_fast(gt[j]) * v[j];
             } else {
 #pragma unroll
               for (int j = 0; j < 32; ++j) v[j] = gt[j] * f_sigmoid(gt[j]) * v[j];
             }
-            apply_chain32_rt(fast, p.post, p.n_post, v, grow, col0, nvalid, row_ok);
+            run_chain<POST>(fast, p.post, p.n_post, v, grow, col0, nvalid, row_ok);
           } else {
             tmem_ld32(tb + c * 32, v);
-            apply_chain32_rt(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+            run_chain<PRE>(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
           }
           if constexpr (MODE == kModeScatter) {
             if (wr) {
@@ -482,7 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           float v[32];
           tmem_ld32(tb + c * 32, v);
-          apply_chain32_rt(false, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+          run_chain<PRE>(false, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
           float cm = -INFINITY;
 #pragma unroll
           for (int j = 0; j < 32; ++j)
@@ -516,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         auto finish_chunk = [&](uint32_t taddr, int32_t col0, float mean, float rstd) {
           float v[32];
           tmem_ld32(taddr, v);
-          apply_chain32_rt(false, p.pre, p.n_pre, v, grow, col0, 32, row_ok);
+          run_chain<PRE>(false, p.pre, p.n_pre, v, grow, col0, 32, row_ok);
 #pragma unroll
           for (int j8 = 0; j8 < 4; ++j8) {
             float ga[8], be[8];
@@ -530,7 +534,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               v[8 * j8 + j] = z;
             }
           }
-          apply_chain32_rt(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
+          run_chain<POST>(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
           if (c_tiles)
             store_tile32_bf16(stage, lane, v,
                               reinterpret_cast<__nv_bfloat16*>(p.C) + static_cast<int64_t>(wrow0) * p.ldc + col0, p.ldc,
@@ -549,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             float v[32];
             tmem_ld32(tb + c * 32, v);
-            apply_chain32_rt(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+            run_chain<PRE>(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
             float sum = 0.0f;
 #pragma unroll
             for (int j = 0; j < 32; ++j) sum += v[j];
