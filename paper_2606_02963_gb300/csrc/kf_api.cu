@@ -78,6 +78,22 @@ kf_status make_map(CUtensorMap* m, const void* base, uint64_t k, uint64_t rows, 
   return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
 }
 
+// Output tensor map for the epilogue's TMA stores: bf16 [rows x cols] (row
+// stride in bytes), box 16 columns x 32 rows, 32-byte swizzle (the layout of the
+// epilogue's tile buffers).
+kf_status make_map_out(CUtensorMap* m, void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes) {
+  auto fn = encode_fn();
+  if (!fn) return KF_ERR_CUDA;
+  std::memset(m, 0, sizeof(*m));
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {16, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_32B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 int elt_size(int dt) { return dt == KF_BF16 ? 2 : 4; }
 bool float_dtype(int dt) { return dt == KF_F32 || dt == KF_BF16; }
@@ -331,7 +347,9 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   p.fast = g.c_dtype == KF_BF16 && pl.mode != kModeScatter;
   const int64_t ub = ((g.rows_total + kBM - 1) / kBM + g.G) * p.tiles_n;
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
-  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, p, grid, s));
+  CUtensorMap mc;  // grouped outputs are masked per group: plain stores, no TMA map
+  std::memset(&mc, 0, sizeof(mc));
+  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, mc, p, grid, s));
 }
 
 }  // namespace
@@ -464,6 +482,13 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   p.c_vec_ok = aligned16(Y) && (ldy * elt_size(yt)) % 16 == 0;
   if (pl.mode == kModeLse) p.lse_part = static_cast<float2*>(workspace);
   fill_params_common(p, pl, di.err);
+  CUtensorMap mc;
+  std::memset(&mc, 0, sizeof(mc));
+  if ((pl.mode == kModeStore || pl.mode == kModeGroupNorm) && yt == KF_BF16 && p.c_vec_ok) {
+    st = make_map_out(&mc, Y, static_cast<uint64_t>(N), static_cast<uint64_t>(M), static_cast<uint64_t>(ldy) * 2);
+    if (st != KF_OK) return st;
+    p.c_tma = 1;
+  }
   p.fast = yt == KF_BF16 && pl.mode != kModeLse;  // bf16 results: reduced-precision activations suffice
   const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
   // a compiled chain program, if the chain matches one (bf16 operands staged)
@@ -474,7 +499,7 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     sig = kSigBiasNormSilu;
   else if (pl.mode == kModeLse && ProgScale::matches(pl.pre, pl.n_pre))
     sig = kSigScaleLse;
-  st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, p, sub, grid, s));
+  st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, p, sub, grid, s));
   if (st != KF_OK || pl.mode != kModeLse) return st;
   LseCombineParams cp;
   std::memset(&cp, 0, sizeof(cp));

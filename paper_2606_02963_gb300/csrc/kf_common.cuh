@@ -9,6 +9,7 @@
 #include <cstdint>
 
 #include "../../include/kf.h"
+#include "kf_ptx.cuh"
 
 namespace kf {
 
@@ -72,6 +73,7 @@ struct TcParams {
   int32_t fast;         // reduced-precision activations (result stored as bf16)
   int32_t res_op;       // index in pre[] of a bf16 RESIDUAL_ADD staged by coalesced loads, or -1
   int32_t vec_op;       // index in pre[] of a bf16 BIAS / MUL whose vector is loaded ahead, or -1
+  int32_t c_tma;        // output tiles leave through TMA stores (dense, bf16, aligned)
 };
 
 // ---------------------------------------------------------------- loads/stores
@@ -211,6 +213,38 @@ __device__ __forceinline__ void store_tile32_bf16(uint8_t* stage, int lane, cons
         *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(gbase) + r * ld + 16 * half + 8 * u) = w;
     }
     __syncwarp();
+  }
+}
+
+// Store the lane's 32 values (row `lane`) as bf16 through TMA: each 16-column
+// half goes into one of the warp's two 1 KB buffers (the 32-byte-swizzle layout
+// of xpose_off, which is what the tensor map's SWIZZLE_32B expects) and leaves
+// as a {16 x 32} box at (x + 16*half, y).  Rows/columns outside the tensor are
+// clipped by TMA.  A buffer is rewritten only after the store that last read it
+// has finished reading (at most one other group in flight).
+__device__ __forceinline__ void store_tile32_tma(uint8_t* stage2, int lane, const float (&v)[32], const CUtensorMap* map,
+                                                 int32_t x, int32_t y) {
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    uint8_t* buf = stage2 + half * 1024;
+    if (lane == 0) bulk_wait_group_read<1>();
+    __syncwarp();
+#pragma unroll
+    for (int uu = 0; uu < 2; ++uu) {
+      const int c = 16 * half + 8 * uu;
+      uint4 w;
+      w.x = pack_bf16x2(v[c + 0], v[c + 1]);
+      w.y = pack_bf16x2(v[c + 2], v[c + 3]);
+      w.z = pack_bf16x2(v[c + 4], v[c + 5]);
+      w.w = pack_bf16x2(v[c + 6], v[c + 7]);
+      *reinterpret_cast<uint4*>(buf + xpose_off(lane, uu)) = w;
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(map, buf, x + 16 * half, y);
+      bulk_commit_group();
+    }
   }
 }
 

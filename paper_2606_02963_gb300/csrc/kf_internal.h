@@ -29,11 +29,11 @@ bool tc_dense_has(int mode, int bn, bool cta2);
 bool tc_dense2_has(int mode, int bn);
 bool tc_grouped_has(int mode, int bn);
 cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,
-                            const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
-cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
-                             int sub_tiles, int grid, cudaStream_t s);
-cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
-                              int grid, cudaStream_t s);
+                            const CUtensorMap& c, const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
+cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
+                             const CUtensorMap& c, const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
+cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                              const TcParams& p, int grid, cudaStream_t s);
 
 // SIMT kernels.
 struct SimtParams {

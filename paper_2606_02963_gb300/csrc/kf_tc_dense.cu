@@ -9,7 +9,7 @@ namespace kf {
 namespace {
 
 template <int BN, int STAGES, int MODE>
-cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int sub, int grid,
+cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int sub, int grid,
                        cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, false>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, false>;
@@ -22,7 +22,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const TcParam
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, p, sub);
+  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, p, sub);
   return cudaGetLastError();
 }
 
@@ -49,10 +49,10 @@ bool tc_dense_has(int mode, int bn, bool cta2) {
 }
 
 cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,
-                            const TcParams& p, int sub, int grid, cudaStream_t s) {
-  if (cta2) return tc_dense2_launch(mode, bn, sig, a, b, p, sub, grid, s);
+                            const CUtensorMap& c, const TcParams& p, int sub, int grid, cudaStream_t s) {
+  if (cta2) return tc_dense2_launch(mode, bn, sig, a, b, c, p, sub, grid, s);
 #define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, p, sub, grid, s);
+  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, p, sub, grid, s);
   KF_DENSE_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;

@@ -10,7 +10,7 @@ namespace kf {
 namespace {
 
 template <int BN, int STAGES, int MODE, class PRE = Interp, class POST = Interp>
-cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int sub, int grid,
+cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int sub, int grid,
                         cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, true>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, true, PRE, POST>;
@@ -36,7 +36,7 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const TcPara
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, a, b, p, static_cast<int32_t>(sub));
+  return cudaLaunchKernelEx(&cfg, kern, a, b, c, p, static_cast<int32_t>(sub));
 }
 
 }  // namespace
@@ -45,10 +45,10 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const TcPara
 #define KF_DENSE2_VARIANTS(X) \
   X(kModeStore, 128, 8)       \
   X(kModeStore, 192, 7)       \
-  X(kModeStore, 224, 7)       \
+  X(kModeStore, 224, 6)       \
   X(kModeStore, 256, 6)       \
   X(kModeLse, 128, 8)         \
-  X(kModeLse, 224, 7)         \
+  X(kModeLse, 224, 6)         \
   X(kModeLse, 256, 6)         \
   X(kModeGroupNorm, 256, 6)
 
@@ -62,20 +62,20 @@ bool tc_dense2_has(int mode, int bn) {
 
 // Chain-program variants: (mode, BN, stages, signature, PRE, POST)
 #define KF_DENSE2_PROG_VARIANTS(X)                                              \
-  X(kModeStore, 224, 7, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 224, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
   X(kModeStore, 256, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
   X(kModeGroupNorm, 256, 6, kSigBiasNormSilu, ProgBias, ProgSilu)               \
-  X(kModeLse, 224, 7, kSigScaleLse, ProgScale, Interp)                          \
+  X(kModeLse, 224, 6, kSigScaleLse, ProgScale, Interp)                          \
   X(kModeLse, 256, 6, kSigScaleLse, ProgScale, Interp)
 
-cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p,
                              int sub, int grid, cudaStream_t s) {
 #define Y(M_, B_, S_, G_, PRE_, POST_) \
-  if (mode == M_ && bn == B_ && sig == G_) return launch_pair<B_, S_, M_, PRE_, POST_>(a, b, p, sub, grid, s);
+  if (mode == M_ && bn == B_ && sig == G_) return launch_pair<B_, S_, M_, PRE_, POST_>(a, b, c, p, sub, grid, s);
   KF_DENSE2_PROG_VARIANTS(Y)
 #undef Y
 #define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_pair<B_, S_, M_>(a, b, p, sub, grid, s);
+  if (mode == M_ && bn == B_) return launch_pair<B_, S_, M_>(a, b, c, p, sub, grid, s);
   KF_DENSE2_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;

@@ -28,6 +28,15 @@
 
 namespace kf {
 
+template <class P>
+struct IsBiasProg {
+  static constexpr bool value = false;
+};
+template <>
+struct IsBiasProg<Prog<KF_OP_BIAS>> {
+  static constexpr bool value = true;
+};
+
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kEpiWarps = 8;
@@ -53,10 +62,14 @@ struct TcCfg {
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
   static constexpr int kBarBytes = (8 * (2 * STAGES + 5) + 63) / 64 * 64;  // keeps what follows 64-B aligned
-  // flags + row-statistics exchange (4 KB) + per-warp 2 KB transpose buffers
-  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16 + kEpiWarps * 1024;
+  // per-warp 2 x 1 KB tile buffers (1 KB aligned, right after the stages)
+  static constexpr int kStagingBytes = kEpiWarps * 2048;
+  // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
+  static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiWarps * 3 * 4 * 32 * 4 : 0;
+  // flags + row-statistics exchange (4 KB)
+  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16;
   static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
-  static constexpr int kSmemUse = STAGES * kStageBytes + kBarBytes + kMiscBytes + kTableBytes;
+  static constexpr int kSmemUse = STAGES * kStageBytes + kStagingBytes + kGnCacheBytes + kBarBytes + kMiscBytes + kTableBytes;
   // pad to > half of the SM's shared memory so that at most one such CTA is
   // resident per SM (tensor-memory allocation then never has to wait)
   static constexpr int kSmemBytes = 1024 + (kSmemUse > 120 * 1024 ? kSmemUse : 120 * 1024);
@@ -74,24 +87,28 @@ struct UnitInfo {
 template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2, class PRE = Interp, class POST = Interp>
 __global__ void __launch_bounds__(kThreads, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                      const __grid_constant__ TcParams p, const int32_t sub_tiles) {
+                      const __grid_constant__ CUtensorMap tmC, const __grid_constant__ TcParams p,
+                      const int32_t sub_tiles) {
   using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CTA2>;
+  constexpr bool PRE_IS_BIAS = IsBiasProg<PRE>::value;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* smB = sm;                                // B stages first: any over-read stays inside the CTA
   uint8_t* smA = sm + STAGES * Cfg::kBBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + STAGES * Cfg::kStageBytes);
+  uint8_t* staging = sm + STAGES * Cfg::kStageBytes;           // epilogue tile buffers
+  float* gn_cache = reinterpret_cast<float*>(staging + Cfg::kStagingBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::kStagingBytes + Cfg::kGnCacheBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* accf = bars + 2 * STAGES;
   uint64_t* acce = bars + 2 * STAGES + 2;
   uint64_t* drain = bars + 2 * STAGES + 4;
-  uint32_t* misc = reinterpret_cast<uint32_t*>(sm + STAGES * Cfg::kStageBytes + Cfg::kBarBytes);
+  uint32_t* misc = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(bars) + Cfg::kBarBytes);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   int32_t* total_s = reinterpret_cast<int32_t*>(misc + 2);
   volatile int* zero_flag = reinterpret_cast<volatile int*>(misc + 3);
-  int32_t* off_s = reinterpret_cast<int32_t*>(sm + STAGES * Cfg::kStageBytes + Cfg::kBarBytes + Cfg::kMiscBytes);
+  int32_t* off_s = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(misc) + Cfg::kMiscBytes);
   int32_t* ustart_s = off_s + (kMaxGroups + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -320,10 +337,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const bool fast = p.fast != 0;
     float4* xch = reinterpret_cast<float4*>(misc + 16);  // [2 halves][4 quadrants][32 lanes]
-    uint8_t* stage = reinterpret_cast<uint8_t*>(misc) + 64 + 2 * 4 * 32 * 16 + ew * 1024;  // this warp's tile buffer
+    uint8_t* stage = staging + ew * 2048;  // this warp's two 1 KB tile buffers
+    float* gcache = gn_cache + ew * (3 * 4 * 32);  // GroupNorm: [bias | gamma | beta][4 chunks][32]
     const bool res_staged = MODE == kModeStore && p.res_op >= 0;
     const bool vec_staged = MODE == kModeStore && p.vec_op >= 0;
     const bool c_tiles = p.c_dtype == KF_BF16 && p.c_vec_ok != 0;
+    const bool c_tma = p.c_tma != 0;
     int32_t tl = 0;
     bool ok = true;
 
@@ -465,6 +484,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                   if (j < nvalid) atomicAdd(dstp + j, v[j] * rs);
               }
             }
+          } else if (c_tma) {
+            store_tile32_tma(stage, lane, v, &tmC, col0, wrow0);
           } else if (c_tiles && nvalid == 32) {
             store_tile32_bf16(stage, lane, v,
                               reinterpret_cast<__nv_bfloat16*>(p.C) + static_cast<int64_t>(wrow0) * p.ldc + col0, p.ldc,
@@ -517,25 +538,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int32_t gs = p.norm.groups;  // group size (columns), multiple of 32
         const float eps = p.norm.eps;
         // normalise + affine + post chain + store one 32-column chunk
-        auto finish_chunk = [&](uint32_t taddr, int32_t col0, float mean, float rstd) {
+        // bias / gamma / beta of this warp's chunks of one accumulator, loaded
+        // once into the warp's cache (coalesced, lane j = column j) so the
+        // normalize pass reads them from shared memory
+        const bool pre_bias = PRE_IS_BIAS;  // compiled program: the pre-chain is one bias op
+        auto fill_cache = [&](int32_t colbase, int c0, int c1, int step) {
+          int slot = 0;
+          for (int c = c0; c < c1 && slot < 4; c += step, ++slot) {
+            const int32_t col = colbase + c * 32 + lane;
+            float* g = gcache + slot * 32 + lane;
+            if (pre_bias) g[0] = ld_elem(p.pre[0].p0, p.pre[0].p_dtype, col);
+            g[4 * 32] = p.norm.p0 ? ld_elem(p.norm.p0, p.norm.p_dtype, col) : 1.0f;
+            g[8 * 32] = p.norm.p1 ? ld_elem(p.norm.p1, p.norm.p_dtype, col) : 0.0f;
+          }
+          __syncwarp();
+        };
+        auto finish_chunk = [&](uint32_t taddr, int32_t col0, float mean, float rstd, int slot) {
           float v[32];
           tmem_ld32(taddr, v);
-          run_chain<PRE>(false, p.pre, p.n_pre, v, grow, col0, 32, row_ok);
+          if (pre_bias) {
 #pragma unroll
-          for (int j8 = 0; j8 < 4; ++j8) {
-            float ga[8], be[8];
-            if (p.norm.p0) ld8(p.norm.p0, p.norm.p_dtype, col0 + 8 * j8, p.norm.vec_ok != 0, ga);
-            if (p.norm.p1) ld8(p.norm.p1, p.norm.p_dtype, col0 + 8 * j8, p.norm.vec_ok != 0, be);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              float z = (v[8 * j8 + j] - mean) * rstd;
-              if (p.norm.p0) z *= ga[j];
-              if (p.norm.p1) z += be[j];
-              v[8 * j8 + j] = z;
-            }
+            for (int j = 0; j < 32; ++j) v[j] += gcache[slot * 32 + j];
+          } else {
+            run_chain<PRE>(false, p.pre, p.n_pre, v, grow, col0, 32, row_ok);
           }
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            v[j] = (v[j] - mean) * rstd * gcache[(4 + slot) * 32 + j] + gcache[(8 + slot) * 32 + j];
           run_chain<POST>(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
-          if (c_tiles)
+          if (c_tma)
+            store_tile32_tma(stage, lane, v, &tmC, col0, wrow0);
+          else if (c_tiles)
             store_tile32_bf16(stage, lane, v,
                               reinterpret_cast<__nv_bfloat16*>(p.C) + static_cast<int64_t>(wrow0) * p.ldc + col0, p.ldc,
                               wrows);
@@ -575,10 +608,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             float n, mean, m2;
             moments(tb + gi * gs, g0, 0, nch, 1, n, mean, m2);
             const float rstd = rsqrtf(m2 / n + eps);
+            fill_cache(g0, 0, nch, 1);
             for (int c = 0; c < nch; ++c) {
               __syncwarp();
-              finish_chunk(tb + gi * gs + c * 32, g0 + c * 32, mean, rstd);
+              finish_chunk(tb + gi * gs + c * 32, g0 + c * 32, mean, rstd, c);
             }
+            __syncwarp();
           }
           release_acc(tl);
           ++tl;
@@ -607,10 +642,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float rstd = rsqrtf(tq / tn + eps);
           for (int st = 0; st < sub_tiles; ++st) {
             const uint32_t tb = tmem + lane_off + ((tl + st) & 1) * Cfg::kAccStride;
-            for (int c = h; c < BN / 32; c += 2) {
+            fill_cache(ui.n0 + st * BN, h, BN / 32, 2);
+            int slot = 0;
+            for (int c = h; c < BN / 32; c += 2, ++slot) {
               __syncwarp();
-              finish_chunk(tb + c * 32, ui.n0 + st * BN + c * 32, tm, rstd);
+              finish_chunk(tb + c * 32, ui.n0 + st * BN + c * 32, tm, rstd, slot);
             }
+            __syncwarp();
             release_acc(tl + st);
           }
           tl += sub_tiles;
@@ -620,6 +658,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ---------------------------------------------------------------- teardown
+  if (warp >= 2 && lane == 0) bulk_wait_group_all();  // this warp's TMA stores have completed
   tc_fence_before();
   __syncwarp();  // lane 0 of the producer / MMA warps arrives after lanes 1-31
   __syncthreads();

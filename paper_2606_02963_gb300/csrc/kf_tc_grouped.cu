@@ -7,7 +7,7 @@ namespace kf {
 namespace {
 
 template <int BN, int STAGES, int MODE>
-cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid, cudaStream_t s) {
+cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int grid, cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, true, false>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, false>;
   static bool configured[64] = {};  // the attribute is per device
@@ -19,7 +19,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const TcParam
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, p, 1);
+  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, p, 1);
   return cudaGetLastError();
 }
 
@@ -44,10 +44,10 @@ bool tc_grouped_has(int mode, int bn) {
   return false;
 }
 
-cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p,
+cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p,
                               int grid, cudaStream_t s) {
 #define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, p, grid, s);
+  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, p, grid, s);
   KF_GROUPED_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;
