@@ -131,6 +131,21 @@ class Clocks:
         return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def reduce_max_over_ranks(values, device, world):
+    """Max of each timing over all ranks (the job is as slow as its slowest rank)."""
+    if world <= 1:
+        return list(values)
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return t.tolist()
+
+
+def whole_job_tflops(flops_per_rank_step, ms_per_step, world):
+    """Whole-job throughput: every rank runs its own replica of the step (weak
+    scaling), so the job does world x flops per (max over ranks) step time."""
+    return world * flops_per_rank_step / (ms_per_step * 1e-3) / 1e12
+
+
 def time_steps(fn, steps, warmup, flush, stream, host_slack=True):
     """Mean device time (ms) of fn() over `steps` calls; L2 flushed before each.
     With host_slack, a ~100 us device-side sleep follows the flush so that the
@@ -248,12 +263,9 @@ def run_kf(args, rank, world, dev):
         ms = time_steps(step, args.steps, args.warmup, flush, stream)
     clocks = clk.summary()
     ms_e2e = time_steps(e2e_step, max(3, args.steps // 2), args.warmup, flush, stream, host_slack=False)
-    if world > 1:
-        t = torch.tensor([ms, ms_e2e], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, ms_e2e = t.tolist()
-    value = world * flops / (ms * 1e-3) / 1e12
-    e2e_value = world * flops / (ms_e2e * 1e-3) / 1e12
+    ms, ms_e2e = reduce_max_over_ranks([ms, ms_e2e], dev, world)
+    value = whole_job_tflops(flops, ms, world)
+    e2e_value = whole_job_tflops(flops, ms_e2e, world)
     ms_eager = time_steps(eager_dense(MAIN, d), args.steps, args.warmup, flush, stream)
     ms_cublas = time_steps(lambda: torch.matmul(d["X"], d["W"].t()), args.steps, args.warmup, flush, stream)
     traffic = stored_traffic("dense_store_gelu_1024x4096x4096")

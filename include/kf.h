@@ -82,7 +82,8 @@ typedef enum kf_op_kind {
                               of the fp32 additions is not fixed).                     */
   KF_OP_MISH = 11,         /* v * tanh(log(1 + exp(v)))                                */
   KF_OP_LEAKY_RELU = 12,   /* v > 0 ? v : scalar * v                                   */
-  KF_OP_MUL = 13           /* v *= p0[col]                          (p0: [N])        */
+  KF_OP_MUL = 13,          /* v *= p0[col]                          (p0: [N])        */
+  KF_OP_ROW_SCALE = 14     /* v *= p0[row]                 (p0: fp32, one per row)     */
 } kf_op_kind;
 
 typedef struct kf_epilogue_op {
@@ -177,6 +178,17 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
                      int64_t H, int64_t I, int32_t E, int32_t k, void* workspace, size_t workspace_bytes,
                      int32_t* topk_ids_out, float* topk_w_out, void* stream);
 size_t kf_moe_ffn_workspace(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k);
+
+/* kf_moe_ffn with flags.  KF_MOE_DETERMINISTIC: the down GEMM writes each routed
+ * row's weighted output (fp32 [T*k x H], in the workspace) and a finalize kernel
+ * sums each token's k rows in slot order, so Y is bit-identical from run to run
+ * (the default scatter-add uses fp32 atomics, whose summation order is not
+ * fixed).  Needs kf_moe_ffn_workspace_ex(..., flags) bytes. */
+#define KF_MOE_DETERMINISTIC 1u
+kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
+                        int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace,
+                        size_t workspace_bytes, int32_t* topk_ids_out, float* topk_w_out, void* stream);
+size_t kf_moe_ffn_workspace_ex(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags);
 
 /*
  * kf_fused_gemm_lse_noalloc -- kf_fused_gemm for row log-sum-exp chains, without

@@ -19,7 +19,7 @@ FP contraction):
 
 Chains are lists of ``(kind, params)``: kinds ``bias, scale, relu, gelu_tanh,
 silu, sigmoid, residual_add, row_logsumexp, groupnorm, swiglu,
-row_scale_scatter_add, mish, leaky_relu, mul``; params ``p0, p1`` (tensors),
+row_scale_scatter_add, mish, leaky_relu, mul, row_scale``; params ``p0, p1`` (tensors),
 ``scalar, eps, groups``.
 """
 from __future__ import annotations
@@ -46,7 +46,7 @@ ORC_F32, ORC_BF16 = 0, 1
 KINDS = {
     "bias": 0, "scale": 1, "relu": 2, "gelu_tanh": 3, "silu": 4, "sigmoid": 5,
     "residual_add": 6, "row_logsumexp": 7, "groupnorm": 8, "swiglu": 9,
-    "row_scale_scatter_add": 10, "mish": 11, "leaky_relu": 12, "mul": 13,
+    "row_scale_scatter_add": 10, "mish": 11, "leaky_relu": 12, "mul": 13, "row_scale": 14,
 }
 
 

@@ -51,6 +51,7 @@ enum {
   ORC_MISH = 11,         /* s * tanh(log(1 + exp(s)))                     */
   ORC_LEAKY_RELU = 12,   /* s > 0 ? s : scalar * s                        */
   ORC_MUL = 13,          /* s_j *= p0[j]                                  */
+  ORC_ROW_SCALE = 14,    /* s_ij *= p0[i]                                 */
 };
 
 typedef struct {
@@ -113,6 +114,7 @@ static double orc_pointwise(const orc_op *op, double v, int64_t i, int64_t j) {
     case ORC_MISH: return v * tanh(orc_softplus(v));
     case ORC_LEAKY_RELU: return v > 0.0 ? v : op->scalar * v;
     case ORC_MUL: return v * orc_load(op->p0, op->p_dtype, j);
+    case ORC_ROW_SCALE: return v * orc_load(op->p0, op->p_dtype, i);
     default: return NAN;
   }
 }
@@ -120,7 +122,7 @@ static double orc_pointwise(const orc_op *op, double v, int64_t i, int64_t j) {
 static int orc_is_pointwise(int kind) {
   return kind == ORC_BIAS || kind == ORC_SCALE || kind == ORC_RELU || kind == ORC_GELU_TANH ||
          kind == ORC_SILU || kind == ORC_SIGMOID || kind == ORC_RESIDUAL_ADD || kind == ORC_MISH ||
-         kind == ORC_LEAKY_RELU || kind == ORC_MUL;
+         kind == ORC_LEAKY_RELU || kind == ORC_MUL || kind == ORC_ROW_SCALE;
 }
 
 /* GroupNorm of one row (PyTorch convention: biased variance, contiguous groups

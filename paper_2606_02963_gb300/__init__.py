@@ -27,14 +27,15 @@ KF_F32, KF_BF16, KF_I32 = 0, 1, 2
 OPS = {
     "bias": 0, "scale": 1, "relu": 2, "gelu_tanh": 3, "silu": 4, "sigmoid": 5,
     "residual_add": 6, "row_logsumexp": 7, "groupnorm": 8, "swiglu": 9,
-    "row_scale_scatter_add": 10, "mish": 11, "leaky_relu": 12, "mul": 13,
+    "row_scale_scatter_add": 10, "mish": 11, "leaky_relu": 12, "mul": 13, "row_scale": 14,
 }
+KF_MOE_DETERMINISTIC = 1
 # every entry point declared in include/kf.h
 ABI_SYMBOLS = (
     "kf_fused_gemm", "kf_fused_gemm_workspace", "kf_moe_route", "kf_grouped_gemm",
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
-    "kf_fused_gemm_lse_noalloc_max_bytes",
+    "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex",
 )
 
 
@@ -78,6 +79,10 @@ def lib() -> ctypes.CDLL:
     L.kf_moe_ffn.argtypes = [P, P, P, P, P, I64, I64, I64, I32, I32, P, SZ, P, P, P]
     L.kf_moe_ffn_workspace.argtypes = [I64, I64, I64, I32, I32]
     L.kf_moe_ffn_workspace.restype = SZ
+    L.kf_moe_ffn_ex.argtypes = [P, P, P, P, P, I64, I64, I64, I32, I32, ctypes.c_uint32, P, SZ, P, P, P]
+    L.kf_moe_ffn_ex.restype = I32
+    L.kf_moe_ffn_workspace_ex.argtypes = [I64, I64, I64, I32, I32, ctypes.c_uint32]
+    L.kf_moe_ffn_workspace_ex.restype = SZ
     L.kf_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
     L.kf_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
     L.kf_fused_gemm_lse_noalloc.argtypes = [P, I32, I64, P, I32, I64, P, I32, I64, I64, I64, EP, P]
@@ -236,15 +241,16 @@ def grouped_gemm(A: torch.Tensor, B: torch.Tensor, offsets: torch.Tensor, N: int
     return out
 
 
-def moe_ffn_workspace_bytes(T: int, H: int, I: int, E: int, k: int) -> int:
-    return lib().kf_moe_ffn_workspace(T, H, I, E, k)
+def moe_ffn_workspace_bytes(T: int, H: int, I: int, E: int, k: int, deterministic: bool = False) -> int:
+    return lib().kf_moe_ffn_workspace_ex(T, H, I, E, k, KF_MOE_DETERMINISTIC if deterministic else 0)
 
 
 def moe_ffn(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tensor, W_down: torch.Tensor, k: int,
             out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
-            return_routing: bool = False, stream=None):
-    """Routed MoE expert FFN (kf_moe_ffn): route, gate/up + SwiGLU, down + scale +
-    scatter-add, bf16 output.  With ``return_routing`` also returns (ids, w)."""
+            return_routing: bool = False, deterministic: bool = False, stream=None):
+    """Routed MoE expert FFN (kf_moe_ffn_ex): route, gate/up + SwiGLU, down +
+    scale + scatter-add (or, deterministic, per-row outputs summed in slot order),
+    bf16 output.  With ``return_routing`` also returns (ids, w)."""
     T, H = X.shape
     E, I2, _ = W_gu.shape
     I = I2 // 2
@@ -254,14 +260,15 @@ def moe_ffn(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tensor, W_down: t
     if out is None:
         out = torch.empty(T, H, dtype=torch.bfloat16, device=X.device)
     L = lib()
-    ws, ws_bytes = _workspace(L.kf_moe_ffn_workspace(T, H, I, E, k), X.device, workspace)
+    flags = KF_MOE_DETERMINISTIC if deterministic else 0
+    ws, ws_bytes = _workspace(L.kf_moe_ffn_workspace_ex(T, H, I, E, k, flags), X.device, workspace)
     ids = w = None
     if return_routing:
         ids = torch.empty(T, k, dtype=torch.int32, device=X.device)
         w = torch.empty(T, k, dtype=torch.float32, device=X.device)
-    st = L.kf_moe_ffn(X.data_ptr(), logits.data_ptr(), W_gu.data_ptr(), W_down.data_ptr(), out.data_ptr(), T, H, I,
-                      E, k, _ptr(ws), ws_bytes, _ptr(ids), _ptr(w), _stream(stream))
-    _check(st, "kf_moe_ffn")
+    st = L.kf_moe_ffn_ex(X.data_ptr(), logits.data_ptr(), W_gu.data_ptr(), W_down.data_ptr(), out.data_ptr(), T, H,
+                         I, E, k, flags, _ptr(ws), ws_bytes, _ptr(ids), _ptr(w), _stream(stream))
+    _check(st, "kf_moe_ffn_ex")
     return (out, ids, w) if return_routing else out
 
 

@@ -103,7 +103,7 @@ bool is_scalar_op(int k) {
          k == KF_OP_MISH || k == KF_OP_LEAKY_RELU;
 }
 bool is_pointwise_op(int k) {
-  return is_scalar_op(k) || k == KF_OP_BIAS || k == KF_OP_MUL || k == KF_OP_RESIDUAL_ADD;
+  return is_scalar_op(k) || k == KF_OP_BIAS || k == KF_OP_MUL || k == KF_OP_RESIDUAL_ADD || k == KF_OP_ROW_SCALE;
 }
 
 struct ChainPlan {
@@ -132,6 +132,9 @@ kf_status to_devop(const kf_epilogue_op& o, int64_t N, DevOp* d) {
     case KF_OP_MUL:
       if (!o.p0 || !float_dtype(o.p_dtype)) return KF_ERR_INVALID_ARG;
       d->vec_ok = aligned16(o.p0);
+      return KF_OK;
+    case KF_OP_ROW_SCALE:
+      if (!o.p0 || o.p_dtype != KF_F32) return KF_ERR_INVALID_ARG;
       return KF_OK;
     case KF_OP_RESIDUAL_ADD:
       if (!o.p0 || !float_dtype(o.p_dtype) || o.ld < N) return KF_ERR_INVALID_ARG;
@@ -523,7 +526,7 @@ kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int
   kf_status st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, topk_ids, topk_w, s));
   if (st != KF_OK) return st;
   return cuda_status(route_sort_launch(topk_ids, topk_w, static_cast<int32_t>(T), E, k, offsets, sorted_token,
-                                       sorted_w, s));
+                                       sorted_w, nullptr, s));
 }
 
 size_t kf_grouped_gemm_workspace(int64_t rows_total, int64_t N, int64_t K, int32_t G, int32_t gathered,
@@ -572,9 +575,10 @@ kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows
 //   topk_ids i32 [T k] | topk_w f32 [T k] | offsets i32 [E+1] | sorted_token i32 [T k]
 //   | sorted_w f32 [T k] | Xg bf16 [T k, H] | h bf16 [T k, I] | Yacc f32 [T, H]
 struct MoeLayout {
-  size_t ids, w, off, st, sw, xg, h, yacc, total;
+  size_t ids, w, off, st, sw, xg, h, yacc, pos, yp, total;
 };
-static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k) {
+// deterministic mode adds: pair_pos i32 [T k] | Yp f32 [T k, H]
+static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags = 0) {
   MoeLayout L;
   const size_t P = static_cast<size_t>(T) * static_cast<size_t>(k);
   size_t o = 0;
@@ -591,25 +595,44 @@ static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t 
   L.xg = take(P * static_cast<size_t>(H) * 2);
   L.h = take(P * static_cast<size_t>(I) * 2);
   L.yacc = take(static_cast<size_t>(T) * static_cast<size_t>(H) * 4);
+  L.pos = L.yp = 0;
+  if (flags & KF_MOE_DETERMINISTIC) {
+    L.pos = take(P * 4);
+    L.yp = take(P * static_cast<size_t>(H) * 4);
+  }
   L.total = o;
   return L;
 }
 
 size_t kf_moe_ffn_workspace(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k) {
+  return kf_moe_ffn_workspace_ex(T, H, I, E, k, 0);
+}
+
+size_t kf_moe_ffn_workspace_ex(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags) {
   if (T < 0 || H < 1 || I < 1 || E < 1 || k < 1) return 0;
-  return moe_layout(T, H, I, E, k).total;
+  return moe_layout(T, H, I, E, k, flags).total;
 }
 
 kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
                      int64_t H, int64_t I, int32_t E, int32_t k, void* workspace, size_t ws_bytes,
                      int32_t* topk_ids_out, float* topk_w_out, void* stream) {
+  return kf_moe_ffn_ex(X, logits, W_gu, W_down, Y, T, H, I, E, k, 0, workspace, ws_bytes, topk_ids_out, topk_w_out,
+                       stream);
+}
+
+kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
+                        int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace, size_t ws_bytes,
+                        int32_t* topk_ids_out, float* topk_w_out, void* stream) {
+  if (flags & ~KF_MOE_DETERMINISTIC) return KF_ERR_INVALID_ARG;
+  const bool det = (flags & KF_MOE_DETERMINISTIC) != 0;
   if (T < 0 || H < 1 || I < 1 || E < 1 || E > 256 || k < 1 || k > E) return KF_ERR_INVALID_ARG;
   if (T * k > INT32_MAX || H > INT32_MAX || I > INT32_MAX) return KF_ERR_INVALID_ARG;
   if (!X || !logits || !W_gu || !W_down || !Y) return KF_ERR_INVALID_ARG;
   if (!aligned16(X) || !aligned16(W_gu) || !aligned16(W_down) || !aligned16(Y) || H % 8 != 0 || I % 8 != 0)
     return KF_ERR_MISALIGNED;
+  if (det && H % 4 != 0) return KF_ERR_MISALIGNED;
   if (T == 0) return KF_OK;
-  const MoeLayout L = moe_layout(T, H, I, E, k);
+  const MoeLayout L = moe_layout(T, H, I, E, k, flags);
   if (!workspace || !aligned16(workspace) || ws_bytes < L.total) return KF_ERR_WORKSPACE;
   DevInfo di;
   kf_status st = device_info(&di);
@@ -626,7 +649,10 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
   auto* yacc = reinterpret_cast<float*>(ws + L.yacc);
   const int64_t P = T * k;
 
-  st = kf_moe_route(logits, T, E, k, ids, w, off, stok, sw, stream);
+  int32_t* pos = det ? reinterpret_cast<int32_t*>(ws + L.pos) : nullptr;
+  st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, ids, w, s));
+  if (st != KF_OK) return st;
+  st = cuda_status(route_sort_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos, s));
   if (st != KF_OK) return st;
   // gate/up: h = silu(Xg W_gate[e]^T) * (Xg W_up[e]^T), rows gathered by token
   {
@@ -640,9 +666,25 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
     st = grouped_core(g, pl, xg, s, di);
     if (st != KF_OK) return st;
   }
-  // down: Yacc[token] += w * (h W_down[e]^T)
-  if (cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
-  {
+  if (det) {
+    // down: Yp[r] = w_r * (h_r W_down[e]^T), then a fixed-order sum per token
+    kf_epilogue_op op{};
+    op.kind = KF_OP_ROW_SCALE;
+    op.p0 = sw;
+    op.p_dtype = KF_F32;
+    kf_epilogue epi{1, &op};
+    ChainPlan pl;
+    st = plan_chain(&epi, H, true, &pl);
+    if (st != KF_OK) return st;
+    float* yp = reinterpret_cast<float*>(ws + L.yp);
+    GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yp, KF_F32, H};
+    st = grouped_core(g, pl, nullptr, s, di);
+    if (st != KF_OK) return st;
+    st = cuda_status(moe_finalize_launch(yp, pos, T, k, H, Y, s));
+    if (st != KF_OK) return st;
+  } else {
+    // down: Yacc[token] += w * (h W_down[e]^T), then bf16
+    if (cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
     kf_epilogue_op op{};
     op.kind = KF_OP_ROW_SCALE_SCATTER_ADD;
     op.p0 = sw;
@@ -656,9 +698,9 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yacc, KF_F32, H};
     st = grouped_core(g, pl, nullptr, s, di);
     if (st != KF_OK) return st;
+    st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s));
+    if (st != KF_OK) return st;
   }
-  st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s));
-  if (st != KF_OK) return st;
   if (topk_ids_out &&
       cudaMemcpyAsync(topk_ids_out, ids, static_cast<size_t>(P) * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
     return KF_ERR_CUDA;

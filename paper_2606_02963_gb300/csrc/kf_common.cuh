@@ -434,6 +434,11 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] *= s;
       } break;
+      case KF_OP_ROW_SCALE: {
+        const float s = row_ok ? reinterpret_cast<const float*>(op.p0)[row] : 0.0f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] *= s;
+      } break;
       case KF_OP_RELU: {
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.0f);

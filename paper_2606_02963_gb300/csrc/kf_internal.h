@@ -61,7 +61,10 @@ cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s);
 cudaError_t route_topk_launch(const float* logits, int32_t T, int32_t E, int32_t k, int32_t* ids, float* w,
                               cudaStream_t s);
 cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
-                              int32_t* offsets, int32_t* sorted_token, float* sorted_w, cudaStream_t s);
+                              int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
+                              cudaStream_t s);
+cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_t T, int32_t k, int64_t H, void* Y,
+                                cudaStream_t s);
 cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
                                int64_t K, void* out, uint32_t* err, cudaStream_t s);
 cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s);

@@ -21,6 +21,7 @@ __device__ __forceinline__ float apply_chain1(const DevOp* ops, int n, float v, 
       case KF_OP_BIAS: v += ld_elem(op.p0, op.p_dtype, col); break;
       case KF_OP_MUL: v *= ld_elem(op.p0, op.p_dtype, col); break;
       case KF_OP_RESIDUAL_ADD: v += ld_elem(op.p0, op.p_dtype, row * op.ld + col); break;
+      case KF_OP_ROW_SCALE: v *= reinterpret_cast<const float*>(op.p0)[row]; break;
       default: v = apply_scalar_op(op, v); break;
     }
   }
@@ -196,7 +197,8 @@ constexpr int kSortWarps = 32;
 __global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32_t* __restrict__ ids,
                                                                      const float* __restrict__ w, int32_t P,
                                                                      int32_t E, int32_t k, int32_t* offsets,
-                                                                     int32_t* sorted_token, float* sorted_w) {
+                                                                     int32_t* sorted_token, float* sorted_w,
+                                                                     int32_t* pair_pos) {
   extern __shared__ int32_t cnt[];  // [kSortWarps][E]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kSortWarps * E; i += blockDim.x) cnt[i] = 0;
@@ -229,6 +231,7 @@ __global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32
       const int32_t pos = cnt[warp * E + e] + rank;
       sorted_token[pos] = p / k;
       sorted_w[pos] = w[p];
+      if (pair_pos) pair_pos[p] = pos;
     }
     __syncwarp();
     if (valid && rank == 0) cnt[warp * E + e] += __popc(peers);
@@ -237,10 +240,44 @@ __global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32
 }
 
 cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
-                              int32_t* offsets, int32_t* sorted_token, float* sorted_w, cudaStream_t s) {
+                              int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
+                              cudaStream_t s) {
   const int32_t P = T * k;
   const size_t smem = sizeof(int32_t) * kSortWarps * E;
-  route_sort_kernel<<<1, kSortWarps * 32, smem, s>>>(ids, w, P, E, k, offsets, sorted_token, sorted_w);
+  route_sort_kernel<<<1, kSortWarps * 32, smem, s>>>(ids, w, P, E, k, offsets, sorted_token, sorted_w, pair_pos);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------ deterministic MoE finalize
+// Y[t, :] = bf16( sum_{j = 0..k-1} Yp[pair_pos[t*k + j], :] ), slot order fixed.
+__global__ void moe_finalize_kernel(const float4* __restrict__ Yp, const int32_t* __restrict__ pair_pos, int64_t T,
+                                    int32_t k, int64_t h4, uint2* __restrict__ Y) {
+  const int64_t total = T * h4;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t t = i / h4, c = i % h4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int32_t j = 0; j < k; ++j) {
+      const float4 y = Yp[static_cast<int64_t>(pair_pos[t * k + j]) * h4 + c];
+      acc.x += y.x;
+      acc.y += y.y;
+      acc.z += y.z;
+      acc.w += y.w;
+    }
+    uint2 o;
+    o.x = pack_bf16x2(acc.x, acc.y);
+    o.y = pack_bf16x2(acc.z, acc.w);
+    Y[i] = o;
+  }
+}
+
+cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_t T, int32_t k, int64_t H, void* Y,
+                                cudaStream_t s) {
+  if (T == 0) return cudaSuccess;
+  const int64_t h4 = H / 4, total = T * h4;
+  const int blocks = static_cast<int>(std::min<int64_t>((total + 255) / 256, 148 * 8));
+  moe_finalize_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const float4*>(Yp), pair_pos, T, k, h4,
+                                             reinterpret_cast<uint2*>(Y));
   return cudaGetLastError();
 }
 

@@ -31,7 +31,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
 // Compiled variants: (mode, BN) -> stages
 #define KF_DENSE_VARIANTS(X) \
   X(kModeStore, 128, 6)      \
-  X(kModeStore, 192, 5)      \
+  X(kModeStore, 192, 4)      \
   X(kModeStore, 224, 4)      \
   X(kModeStore, 256, 4)      \
   X(kModeLse, 128, 6)        \

@@ -62,8 +62,11 @@ struct TcCfg {
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
   static constexpr int kBarBytes = (8 * (2 * STAGES + 5) + 63) / 64 * 64;  // keeps what follows 64-B aligned
-  // per-warp 2 x 1 KB tile buffers (1 KB aligned, right after the stages)
-  static constexpr int kStagingBytes = kEpiWarps * 2048;
+  // per-warp 1 KB tile buffers (1 KB aligned, right after the stages): two for
+  // the asynchronous TMA stores, plus (store mode) one for the residual
+  // transposition, which must not reuse a buffer a TMA store may still read
+  static constexpr int kWarpStaging = (MODE == kModeStore) ? 3072 : 2048;
+  static constexpr int kStagingBytes = kEpiWarps * kWarpStaging;
   // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
   static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiWarps * 3 * 4 * 32 * 4 : 0;
   // flags + row-statistics exchange (4 KB)
@@ -337,7 +340,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const bool fast = p.fast != 0;
     float4* xch = reinterpret_cast<float4*>(misc + 16);  // [2 halves][4 quadrants][32 lanes]
-    uint8_t* stage = staging + ew * 2048;  // this warp's two 1 KB tile buffers
+    uint8_t* stage = staging + ew * Cfg::kWarpStaging;  // this warp's 1 KB tile buffers
+    uint8_t* rstage = stage + 2048;                     // store mode: residual transposition
     float* gcache = gn_cache + ew * (3 * 4 * 32);  // GroupNorm: [bias | gamma | beta][4 chunks][32]
     const bool res_staged = MODE == kModeStore && p.res_op >= 0;
     const bool vec_staged = MODE == kModeStore && p.vec_op >= 0;
@@ -447,7 +451,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             Staged32 sg;
             sg.use_res = res_staged && nvalid == 32;
             sg.vec_idx = (vec_staged && nvalid == 32) ? p.vec_op : -1;
-            if (sg.use_res) tile32_finish(stage, lane, rq, sg.res);
+            if (sg.use_res) tile32_finish(rstage, lane, rq, sg.res);
             if (sg.vec_idx >= 0) pack16(bq, sg.vec);
             issue_chunk(c + 2);
             tmem_ld32(tb + c * 32, v);

@@ -33,7 +33,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
   X(kModeScatter, 192, 5)      \
   X(kModeScatter, 256, 4)      \
   X(kModeStore, 128, 6)        \
-  X(kModeStore, 192, 5)        \
+  X(kModeStore, 192, 4)        \
   X(kModeStore, 256, 4)
 
 bool tc_grouped_has(int mode, int bn) {

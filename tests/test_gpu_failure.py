@@ -1,0 +1,64 @@
+"""Failure detection without a GPU fault: every device-side wait of the tensor-core
+kernels has a wall-clock limit.  With the limit set to 1 ns the first wait that
+is not already satisfied gives up; the kernel records a timeout bit in the
+device error word, drains its in-flight copies and MMAs, frees tensor memory and
+returns.  The host reads KF_ERR_DEVICE_TIMEOUT, and the context stays usable: the
+next (normal) call is correct."""
+import numpy as np
+import pytest
+import torch
+
+import kf_workloads
+import oracle
+import paper_2606_02963_gb300 as kf
+from tests._util import check_bf16, wl_chain, chain_to
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def _problem():
+    inp = kf_workloads.generate("bf16_gelu_scale_residual", seed=21, M=512, N=1024, K=512)
+    return inp, {k: v.to(DEV) for k, v in inp.items()}
+
+
+@pytest.mark.parametrize("M", [100, 512])  # single-CTA tiles and CTA pairs
+def test_wait_timeout_is_reported_and_context_survives(M):
+    inp, d = _problem()
+    X, R = d["X"][:M], d["R"][:M]
+    chain = chain_to(wl_chain("bf16_gelu_scale_residual", inp), DEV)
+    chain[-1] = ("residual_add", {"p0": R})
+    assert kf.get_device_error()[0] == kf.KF_OK
+    try:
+        kf.set_wait_timeout_ns(1)
+        kf.fused_gemm(X, d["W"], chain)
+        st, raw = kf.get_device_error()
+    finally:
+        kf.set_wait_timeout_ns(0)
+    assert st == kf.KF_ERR_DEVICE_TIMEOUT, (st, hex(raw))
+    assert raw & 0x7
+    # the error word was cleared by the read, and the next call is correct
+    assert kf.get_device_error()[0] == kf.KF_OK
+    Y = kf.fused_gemm(X, d["W"], chain)
+    torch.cuda.synchronize()
+    ref_chain = wl_chain("bf16_gelu_scale_residual", inp)
+    ref = oracle.fused_gemm(inp["X"][:M], inp["W"], ref_chain)
+    check_bf16(Y, ref, "after timeout")
+    assert kf.get_device_error()[0] == kf.KF_OK
+
+
+def test_grouped_wait_timeout_is_reported():
+    g = torch.Generator().manual_seed(3)
+    A = torch.randn(300, 128, generator=g).to(torch.bfloat16).to(DEV)
+    B = (torch.randn(3, 256, 128, generator=g) * 0.1).to(torch.bfloat16).to(DEV)
+    off = torch.tensor([0, 100, 100, 300], dtype=torch.int32, device=DEV)
+    try:
+        kf.set_wait_timeout_ns(1)
+        kf.grouped_gemm(A, B, off, 256, [])
+        st, raw = kf.get_device_error()
+    finally:
+        kf.set_wait_timeout_ns(0)
+    assert st == kf.KF_ERR_DEVICE_TIMEOUT, (st, hex(raw))
+    C = kf.grouped_gemm(A, B, off, 256, [])
+    ref = oracle.grouped_gemm(A.cpu(), B.cpu(), off.cpu().numpy(), 256, [])
+    check_bf16(C, ref, "grouped after timeout")

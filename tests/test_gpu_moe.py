@@ -126,3 +126,32 @@ def test_moe_ffn_full_size(T, n_check):
     check_bf16(out[toks], ref, f"moe T={T}")
     assert torch.isfinite(out.float()).all()
     _no_device_error()
+
+
+@pytest.mark.parametrize("T", [64, 500])
+def test_moe_ffn_deterministic_mode(T):
+    """Fixed-order finalize: bit-identical across runs, and within tolerance of
+    the oracle (the atomic scatter-add mode is checked above)."""
+    m = kf_workloads.moe_generate(T, seed=T + 7, H=2880, I=2880, E=32, k=4)
+    d = {k: v.to(DEV) for k, v in m.items()}
+    y1 = kf.moe_ffn(d["X"], d["logits"], d["W_gu"], d["W_down"], 4, deterministic=True)
+    y2 = kf.moe_ffn(d["X"], d["logits"], d["W_gu"], d["W_down"], 4, deterministic=True)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
+    r = oracle.moe_route(m["logits"], 4)
+    toks = sorted(set([0, T - 1] + list(np.random.default_rng(2).choice(T, 12, replace=False))))
+    ref = oracle.moe_ffn(m["X"], m["W_gu"], m["W_down"], r["topk_ids"], r["topk_w"], tokens=toks)
+    check_bf16(y1[toks], ref, f"deterministic moe T={T}")
+    _no_device_error()
+
+
+def test_grouped_row_scale_store():
+    sizes = [5, 0, 70]
+    N, K = 256, 64
+    rows, off, B, g = _groups(sizes, K, N, seed=31)
+    A = torch.randn(rows, K, generator=g).to(torch.bfloat16)
+    sc = torch.rand(rows, generator=g)
+    C = kf.grouped_gemm(A.to(DEV), B.to(DEV), off.to(DEV), N, [("row_scale", {"p0": sc.to(DEV)})],
+                        out_dtype=torch.float32)
+    ref = oracle.grouped_gemm(A, B, off.numpy(), N, [("row_scale", {"p0": sc})])
+    check_f32(C, ref, "row scale")

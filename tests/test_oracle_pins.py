@@ -338,3 +338,12 @@ def test_grouped_single_group_equals_dense():
     dense = oracle.fused_gemm(X, W, chain)
     grp = oracle.grouped_gemm(X, W[None], np.array([0, 7], np.int32), 9, chain)
     assert np.array_equal(dense, grp)
+
+
+def test_row_scale_multiplies_each_row():
+    g = torch.Generator().manual_seed(13)
+    X = bf16(torch.randint(-3, 4, (5, 8), generator=g).float())
+    W = bf16(torch.randint(-3, 4, (6, 8), generator=g).float())
+    sc = torch.tensor([1.0, -2.0, 0.5, 0.0, 3.0])
+    Y = oracle.fused_gemm(X, W, [("row_scale", {"p0": sc})])
+    assert np.array_equal(Y, (f64(X) @ f64(W).T) * sc.double().numpy()[:, None])
