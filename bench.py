@@ -48,7 +48,7 @@ def _peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
 
 
-KERNEL_FILES = ("kf_ptx.cuh", "kf_common.cuh", "kf_tc_gemm.cuh", "kf_tc_dense.cu")
+KERNEL_FILES = ("kf_ptx.cuh", "kf_common.cuh", "kf_tc_gemm.cuh", "kf_internal.h", "kf_tc_dense.cu", "kf_tc_dense2.cu")
 
 
 def kernel_source_hash() -> str:
