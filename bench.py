@@ -367,6 +367,28 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
     return res
 
 
+def profile_workload(name, dev, reps):
+    """Run one workload through the public API `reps` times (no timing): the
+    command that ncu launch lists and captures of that workload are taken on."""
+    import paper_2606_02963_gb300 as kf
+    if name.startswith("moe_T"):
+        T, E, k, H, I = int(name[5:]), 32, 4, 2880, 2880
+        g = torch.Generator("cpu").manual_seed(0)
+        X = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
+        logits = torch.randn(T, E, generator=g).to(dev)
+        gd = torch.Generator(dev).manual_seed(1)
+        Wgu = (torch.randn(E, 2 * I, H, generator=gd, device=dev) * 0.02).to(torch.bfloat16)
+        Wd = (torch.randn(E, H, I, generator=gd, device=dev) * 0.02).to(torch.bfloat16)
+        for _ in range(reps):
+            kf.moe_ffn(X, logits, Wgu, Wd, k)
+    else:
+        wl, inp, d, chain = dense_setup(name, dev)
+        for _ in range(reps):
+            kf.fused_gemm(d["X"], d["W"], chain)
+    torch.cuda.synchronize()
+    print(f"profiled {name} x{reps}")
+
+
 def run_reference(args, rank, world):
     """The oracle as it stands on the host cores, on bounded row samples of the
     headline workload (one sample per step)."""
@@ -408,6 +430,9 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=8.0)
     ap.add_argument("--ref-rows", type=int, default=16)
+    ap.add_argument("--profile-workload", default=None,
+                    help="run one workload's calls --steps times, untimed (the command ncu captures of it use): "
+                         "bf16_gelu_scale_residual, bf16_scale_rowlse, bf16_groupnorm_swish, moe_T64 or moe_T4096")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -420,6 +445,9 @@ def main():
         return
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    if args.profile_workload:
+        profile_workload(args.profile_workload, dev, args.steps)
+        return
     if world > 1:
         torch.distributed.init_process_group("nccl", device_id=dev)
     line = run_kf(args, rank, world, dev)

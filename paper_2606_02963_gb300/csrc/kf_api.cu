@@ -454,9 +454,15 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   // CTA pairs (256-row tiles, tcgen05.mma.cta_group::2) unless one 128-row
   // tile already covers M
   const bool cta2 = M > kBM && di.nsm >= 2;
+  // GroupNorm over 512-column groups: clusters of two CTA pairs, one 256-column
+  // half of each group per pair, so each CTA double-buffers its accumulators
+  const bool quad = cta2 && pl.mode == kModeGroupNorm && pl.gs == 512 && di.nsm >= 4 && tc_dense4_has(pl.mode, 256);
   int bn = 0, sub = 1;
   int64_t tiles_n = 0;
-  if (pl.mode == kModeGroupNorm) {
+  if (quad) {
+    bn = 256;
+    tiles_n = N / 512;
+  } else if (pl.mode == kModeGroupNorm) {
     bn = 256;
     sub = pl.gs == 512 ? 2 : 1;
     tiles_n = (N + bn * sub - 1) / (bn * sub);
@@ -502,7 +508,10 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     sig = kSigBiasNormSilu;
   else if (pl.mode == kModeLse && ProgScale::matches(pl.pre, pl.n_pre))
     sig = kSigScaleLse;
-  st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, p, sub, grid, s));
+  if (quad)
+    st = cuda_status(tc_dense4_launch(pl.mode, bn, sig, ma, mb, mc, p, s));
+  else
+    st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, p, sub, grid, s));
   if (st != KF_OK || pl.mode != kModeLse) return st;
   LseCombineParams cp;
   std::memset(&cp, 0, sizeof(cp));

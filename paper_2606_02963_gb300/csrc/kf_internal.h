@@ -34,6 +34,12 @@ cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, co
                              const CUtensorMap& c, const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
 cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                               const TcParams& p, int grid, cudaStream_t s);
+// GroupNorm over 512-column groups on clusters of two CTA pairs (one 256-column
+// half of the group per pair); units = 256-row x 512-column blocks, the grid is
+// sized inside from the number of co-resident clusters.
+bool tc_dense4_has(int mode, int bn);
+cudaError_t tc_dense4_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
+                             const CUtensorMap& c, const TcParams& p, cudaStream_t s);
 
 // SIMT kernels.
 struct SimtParams {

@@ -207,17 +207,50 @@ __global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32
   const int32_t beg = min(P, warp * chunk), end = min(P, beg + chunk);
   for (int32_t p = beg + lane; p < end; p += 32) atomicAdd(&cnt[warp * E + ids[p]], 1);
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int32_t run = 0;
-    for (int e = 0; e < E; ++e) {
-      offsets[e] = run;
-      for (int ww = 0; ww < kSortWarps; ++ww) {
-        const int32_t c = cnt[ww * E + e];
-        cnt[ww * E + e] = run;  // becomes the first slot of (warp ww, expert e)
-        run += c;
+  // Scan the (expert, warp) counts in expert-major, warp-minor order.  Thread e
+  // sums its expert's column; warp 0 scans the E totals (lane l owns experts
+  // l*per .. l*per+per-1, then a shuffle scan across lanes); thread e then turns
+  // its column into each warp's first slot for expert e.
+  __shared__ int32_t tot[kMaxExperts];
+  if (threadIdx.x < E) {
+    int32_t t = 0;
+    for (int ww = 0; ww < kSortWarps; ++ww) t += cnt[ww * E + threadIdx.x];
+    tot[threadIdx.x] = t;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int per = (E + 31) / 32;
+    int32_t local = 0;
+    for (int i = 0; i < per; ++i) {
+      const int e = lane * per + i;
+      if (e < E) local += tot[e];
+    }
+    int32_t incl = local;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int32_t o = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += o;
+    }
+    int32_t run = incl - local;  // exclusive prefix of this lane's first expert
+    for (int i = 0; i < per; ++i) {
+      const int e = lane * per + i;
+      if (e < E) {
+        const int32_t t = tot[e];
+        tot[e] = run;
+        offsets[e] = run;
+        run += t;
       }
     }
-    offsets[E] = run;
+    if (lane == 31) offsets[E] = run;
+  }
+  __syncthreads();
+  if (threadIdx.x < E) {
+    int32_t run = tot[threadIdx.x];
+    for (int ww = 0; ww < kSortWarps; ++ww) {
+      const int32_t c = cnt[ww * E + threadIdx.x];
+      cnt[ww * E + threadIdx.x] = run;  // first slot of (warp ww, expert e)
+      run += c;
+    }
   }
   __syncthreads();
   const uint32_t lt_mask = (1u << lane) - 1u;

@@ -2,7 +2,10 @@
 // a cluster of two CTAs computes a 256-row tile with tcgen05.mma.cta_group::2
 // (each CTA stages its own 128 rows of A and half of the B rows), which halves
 // the operand bytes each SM streams per MMA and lets a 6-8 stage ring cover the
-// TMA round trip.
+// TMA round trip.  GroupNorm over 512-column groups also runs on clusters of
+// two such pairs, one 256-column half of the group each.
+#include <algorithm>
+
 #include "kf_internal.h"
 #include "kf_tc_gemm.cuh"
 
@@ -12,8 +15,8 @@ namespace {
 template <int BN, int STAGES, int MODE, class PRE = Interp, class POST = Interp>
 cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int sub, int grid,
                         cudaStream_t s) {
-  using Cfg = TcCfg<BN, STAGES, MODE, false, true>;
-  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, true, PRE, POST>;
+  using Cfg = TcCfg<BN, STAGES, MODE, false, kClPair>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClPair, PRE, POST>;
   static bool configured[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -39,7 +42,55 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtens
   return cudaLaunchKernelEx(&cfg, kern, a, b, c, p, static_cast<int32_t>(sub));
 }
 
+// Cluster of four (two CTA pairs).  The persistent grid holds as many clusters
+// as can be resident at once (a cluster needs four free SMs of one GPC), at
+// most one per unit.
+template <int BN, int STAGES, int MODE, class PRE = Interp, class POST = Interp>
+cudaError_t launch_quad(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p,
+                        cudaStream_t s) {
+  using Cfg = TcCfg<BN, STAGES, MODE, false, kClQuad>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClQuad, PRE, POST>;
+  static int max_clusters[64] = {};  // per device; 0 = not yet queried
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 4;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (max_clusters[dev] == 0) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    int nc = 0;
+    cfg.gridDim = dim3(4, 1, 1);
+    e = cudaOccupancyMaxActiveClusters(&nc, kern, &cfg);
+    if (e != cudaSuccess) return e;
+    if (nc < 1) return cudaErrorInvalidConfiguration;
+    max_clusters[dev] = nc;
+  }
+  const int clusters = std::min(p.total_units, max_clusters[dev]);
+  if (clusters < 1) return cudaSuccess;
+  cfg.gridDim = dim3(4 * clusters, 1, 1);
+  return cudaLaunchKernelEx(&cfg, kern, a, b, c, p, static_cast<int32_t>(1));
+}
+
 }  // namespace
+
+bool tc_dense4_has(int mode, int bn) { return mode == kModeGroupNorm && bn == 256; }
+
+cudaError_t tc_dense4_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
+                             const CUtensorMap& c, const TcParams& p, cudaStream_t s) {
+  if (mode != kModeGroupNorm || bn != 256) return cudaErrorInvalidValue;
+  if (sig == kSigBiasNormSilu) return launch_quad<256, 6, kModeGroupNorm, ProgBias, ProgSilu>(a, b, c, p, s);
+  return launch_quad<256, 6, kModeGroupNorm>(a, b, c, p, s);  // any other chain: interpreter
+}
 
 // Compiled CTA-pair variants: (mode, BN) -> stages
 #define KF_DENSE2_VARIANTS(X) \

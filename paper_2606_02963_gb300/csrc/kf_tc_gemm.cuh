@@ -47,10 +47,21 @@ __host__ __device__ constexpr int pow2_at_least(int x) {
   return x <= 32 ? 32 : x <= 64 ? 64 : x <= 128 ? 128 : x <= 256 ? 256 : 512;
 }
 
-template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2>
+// Cluster layouts (CL): kClOne = single CTA, 128-row tiles; kClPair = a CTA
+// pair (cluster of 2) computing 256-row tiles with tcgen05.mma.cta_group::2;
+// kClQuad = a cluster of two such pairs whose tiles are the two 256-column
+// halves of one 512-column unit (GroupNorm: one group per unit).
+constexpr int kClOne = 0;
+constexpr int kClPair = 1;
+constexpr int kClQuad = 2;
+
+template <int BN, int STAGES, int MODE, bool GROUPED, int CL>
 struct TcCfg {
+  static constexpr bool CTA2 = CL != kClOne;  // tcgen05 CTA-pair MMAs
+  static constexpr bool kQuad = CL == kClQuad;
   static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN");
   static_assert(!(GROUPED && CTA2), "grouped GEMMs use single-CTA tiles");
+  static_assert(!kQuad || (MODE == kModeGroupNorm && BN == 256), "quad clusters split 512-column groups");
   static constexpr int kOutN = (MODE == kModeSwiglu) ? BN / 2 : BN;  // output columns of a (sub)tile
   // With CTA pairs each CTA stages its own 128 rows of A and half of the BN rows of B.
   static constexpr int kBRows = CTA2 ? BN / 2 : BN;
@@ -61,7 +72,7 @@ struct TcCfg {
   // accumulator buffer b starts at TMEM column b * kAccStride
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
-  static constexpr int kBarBytes = (8 * (2 * STAGES + 5) + 63) / 64 * 64;  // keeps what follows 64-B aligned
+  static constexpr int kBarBytes = (8 * (2 * STAGES + 7) + 63) / 64 * 64;  // keeps what follows 64-B aligned
   // per-warp 1 KB tile buffers (1 KB aligned, right after the stages): two for
   // the asynchronous TMA stores, plus (store mode) one for the residual
   // transposition, which must not reuse a buffer a TMA store may still read
@@ -69,8 +80,9 @@ struct TcCfg {
   static constexpr int kStagingBytes = kEpiWarps * kWarpStaging;
   // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
   static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiWarps * 3 * 4 * 32 * 4 : 0;
-  // flags + row-statistics exchange (4 KB)
-  static constexpr int kMiscBytes = 64 + 2 * 4 * 32 * 16;
+  // flags + row-statistics exchange between the two warps of a quadrant (2 KB)
+  // + (quad) the other pair's per-row statistics, two slots (2 KB)
+  static constexpr int kMiscBytes = 64 + 2 * kBM * 8 + (kQuad ? 2 * kBM * 8 : 0);
   static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
   static constexpr int kSmemUse = STAGES * kStageBytes + kStagingBytes + kGnCacheBytes + kBarBytes + kMiscBytes + kTableBytes;
   // pad to > half of the SM's shared memory so that at most one such CTA is
@@ -87,12 +99,14 @@ struct UnitInfo {
 
 // PRE / POST: compiled op programs (Prog<...>) for the chain before / after the
 // reduction, or Interp for arbitrary chains.
-template <int BN, int STAGES, int MODE, bool GROUPED, bool CTA2, class PRE = Interp, class POST = Interp>
+template <int BN, int STAGES, int MODE, bool GROUPED, int CL, class PRE = Interp, class POST = Interp>
 __global__ void __launch_bounds__(kThreads, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, const __grid_constant__ TcParams p,
                       const int32_t sub_tiles) {
-  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CTA2>;
+  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CL>;
+  constexpr bool CTA2 = Cfg::CTA2;
+  constexpr bool QUAD = Cfg::kQuad;
   constexpr bool PRE_IS_BIAS = IsBiasProg<PRE>::value;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -106,6 +120,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* accf = bars + 2 * STAGES;
   uint64_t* acce = bars + 2 * STAGES + 2;
   uint64_t* drain = bars + 2 * STAGES + 4;
+  uint64_t* xbar = bars + 2 * STAGES + 5;  // quad: the other pair's statistics have landed (2 slots)
   uint32_t* misc = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(bars) + Cfg::kBarBytes);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
@@ -116,10 +131,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const uint32_t rank = CTA2 ? cluster_ctarank() : 0u;  // 0 = leader of the CTA pair (issues the MMAs)
-  const bool leader = rank == 0;
-  const int32_t unit0 = CTA2 ? static_cast<int32_t>(blockIdx.x >> 1) : static_cast<int32_t>(blockIdx.x);
-  const int32_t unit_step = CTA2 ? static_cast<int32_t>(gridDim.x >> 1) : static_cast<int32_t>(gridDim.x);
+  // CTA pairs are the cluster ranks that differ in bit 0; the even rank leads
+  // (issues the MMAs, owns the barriers both CTAs' copies complete on)
+  const uint32_t rank = CTA2 ? cluster_ctarank() : 0u;
+  const uint32_t prank = rank & 1u;       // position in the pair: 128-row half
+  const uint32_t lead_rank = rank & ~1u;  // cluster rank of the pair's leader
+  const uint16_t pair_mask = static_cast<uint16_t>(0x3u << (rank & 2u));
+  const bool leader = prank == 0;
+  constexpr int kUnitShift = QUAD ? 2 : (CTA2 ? 1 : 0);
+  const int32_t unit0 = static_cast<int32_t>(blockIdx.x >> kUnitShift);
+  const int32_t unit_step = static_cast<int32_t>(gridDim.x >> kUnitShift);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -131,6 +152,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&acce[a], kEpiWarps * (CTA2 ? 2 : 1));
     }
     mbar_init(drain, 1);
+    if constexpr (QUAD) {
+      mbar_init(&xbar[0], kBM);  // one arrival per row of the other pair's CTA
+      mbar_init(&xbar[1], kBM);
+    }
     *abort_flag = 0;
     *zero_flag = 0;
     *total_s = GROUPED ? 0 : p.total_units;
@@ -210,9 +235,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int32_t mb = u % p.tiles_m;
       r.n_blk = u / p.tiles_m;
       r.g = 0;
-      r.m0 = mb * Cfg::kRowsPerUnit + static_cast<int32_t>(rank) * kBM;  // this CTA's 128 rows
+      r.m0 = mb * Cfg::kRowsPerUnit + static_cast<int32_t>(prank) * kBM;  // this CTA's 128 rows
       r.m_end = min(p.M, r.m0 + kBM);
-      r.n0 = r.n_blk * Cfg::kOutN * sub_tiles;
+      if constexpr (QUAD)
+        r.n0 = r.n_blk * 2 * BN + static_cast<int32_t>(rank >> 1) * BN;  // this pair's 256 columns
+      else
+        r.n0 = r.n_blk * Cfg::kOutN * sub_tiles;
     }
     return r;
   };
@@ -225,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int32_t u = unit0; ok && u < total; u += unit_step) {
         const UnitInfo ui = decode(u);
         for (int s = 0; ok && s < sub_tiles; ++s) {
-          const int32_t nb0 = ui.n0 + s * BN + static_cast<int32_t>(rank) * Cfg::kBRows;
+          const int32_t nb0 = ui.n0 + s * BN + static_cast<int32_t>(prank) * Cfg::kBRows;
           for (int32_t kb = 0; kb < p.num_kb; ++kb) {
             const int st = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1;
@@ -240,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if constexpr (CTA2) {
               // both CTAs' copies complete on the leader's full barrier
               if (leader) mbar_arrive_expect_tx(&full[st], Cfg::kTxBytes);
-              const uint32_t fb = mapa_shared(smem_u32(&full[st]), 0);
+              const uint32_t fb = mapa_shared(smem_u32(&full[st]), lead_rank);
               tma_load_2d_pair(a, &tmA, fb, kb * kBK, ui.m0);
               tma_load_3d_pair(b, &tmB, fb, kb * kBK, nb0, ui.g);
             } else {
@@ -303,14 +331,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_mma_bf16(d, ad, bd, Cfg::kIdesc, (kb | kk) != 0 ? 1u : 0u);
             }
             if constexpr (CTA2)
-              tc_commit_pair_mc(&empty[st], 0x3);  // frees the slot in both CTAs
+              tc_commit_pair_mc(&empty[st], pair_mask);  // frees the slot in both CTAs
             else
               tc_commit(&empty[st]);
             ++it;
           }
           if (!ok) break;
           if constexpr (CTA2)
-            tc_commit_pair_mc(&accf[acc], 0x3);
+            tc_commit_pair_mc(&accf[acc], pair_mask);
           else
             tc_commit(&accf[acc]);
           ++tl;
@@ -339,7 +367,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int32_t row_in_tile = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const bool fast = p.fast != 0;
-    float4* xch = reinterpret_cast<float4*>(misc + 16);  // [2 halves][4 quadrants][32 lanes]
+    float2* xch = reinterpret_cast<float2*>(misc + 16);  // [2 halves][128 rows]
+    float2* xs = xch + 2 * kBM;                           // quad: [2 slots][128 rows] from CTA rank ^ 2
     uint8_t* stage = staging + ew * Cfg::kWarpStaging;  // this warp's 1 KB tile buffers
     uint8_t* rstage = stage + 2048;                     // store mode: residual transposition
     float* gcache = gn_cache + ew * (3 * 4 * 32);  // GroupNorm: [bias | gamma | beta][4 chunks][32]
@@ -366,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) {
         if (CTA2 && !leader)
-          mbar_arrive_remote(mapa_shared(smem_u32(&acce[t & 1]), 0));
+          mbar_arrive_remote(mapa_shared(smem_u32(&acce[t & 1]), lead_rank));
         else
           mbar_arrive(&acce[t & 1]);
       }
@@ -527,10 +556,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         release_acc(tl);
         ++tl;
         // merge the two halves of the row: half 1 hands (m, s) to half 0
-        if (h == 1) xch[q * 32 + lane] = make_float4(m, s, 0.f, 0.f);
+        if (h == 1) xch[row_in_tile] = make_float2(m, s);
         pair_sync();
         if (h == 0) {
-          const float4 o = xch[q * 32 + lane];
+          const float2 o = xch[row_in_tile];
           const float nm = fmaxf(m, o.x);
           float ss = 0.0f;
           if (nm != -INFINITY)
@@ -546,29 +575,61 @@ __global__ void __launch_bounds__(kThreads, 1)
         // once into the warp's cache (coalesced, lane j = column j) so the
         // normalize pass reads them from shared memory
         const bool pre_bias = PRE_IS_BIAS;  // compiled program: the pre-chain is one bias op
-        auto fill_cache = [&](int32_t colbase, int c0, int c1, int step) {
-          int slot = 0;
-          for (int c = c0; c < c1 && slot < 4; c += step, ++slot) {
+        // the vectors of the warp's 4 chunks c0, c0 + step, ... (lane j = column j
+        // of each chunk) are loaded into registers first, all at once, and
+        // parked in the cache later: one memory round trip instead of twelve
+        float vb[4], vg[4], vt[4];
+        auto issue_vecs = [&](int32_t colbase, int c0, int c1, int step) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int c = c0 + i * step;
             const int32_t col = colbase + c * 32 + lane;
-            float* g = gcache + slot * 32 + lane;
-            if (pre_bias) g[0] = ld_elem(p.pre[0].p0, p.pre[0].p_dtype, col);
-            g[4 * 32] = p.norm.p0 ? ld_elem(p.norm.p0, p.norm.p_dtype, col) : 1.0f;
-            g[8 * 32] = p.norm.p1 ? ld_elem(p.norm.p1, p.norm.p_dtype, col) : 0.0f;
+            const bool in = c < c1;
+            vb[i] = (in && pre_bias) ? ld_elem(p.pre[0].p0, p.pre[0].p_dtype, col) : 0.0f;
+            vg[i] = (in && p.norm.p0) ? ld_elem(p.norm.p0, p.norm.p_dtype, col) : 1.0f;
+            vt[i] = (in && p.norm.p1) ? ld_elem(p.norm.p1, p.norm.p_dtype, col) : 0.0f;
+          }
+        };
+        auto park_vecs = [&]() {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            gcache[i * 32 + lane] = vb[i];
+            gcache[(4 + i) * 32 + lane] = vg[i];
+            gcache[(8 + i) * 32 + lane] = vt[i];
           }
           __syncwarp();
+        };
+        auto fill_cache = [&](int32_t colbase, int c0, int c1, int step) {
+          __syncwarp();  // the previous chunks' reads of the cache are done
+          issue_vecs(colbase, c0, c1, step);
+          park_vecs();
         };
         auto finish_chunk = [&](uint32_t taddr, int32_t col0, float mean, float rstd, int slot) {
           float v[32];
           tmem_ld32(taddr, v);
+          const float4* cb = reinterpret_cast<const float4*>(gcache + slot * 32);
+          const float4* cg = reinterpret_cast<const float4*>(gcache + (4 + slot) * 32);
+          const float4* ct = reinterpret_cast<const float4*>(gcache + (8 + slot) * 32);
           if (pre_bias) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] += gcache[slot * 32 + j];
+            for (int k = 0; k < 8; ++k) {
+              const float4 b = cb[k];
+              v[4 * k] += b.x;
+              v[4 * k + 1] += b.y;
+              v[4 * k + 2] += b.z;
+              v[4 * k + 3] += b.w;
+            }
           } else {
             run_chain<PRE>(false, p.pre, p.n_pre, v, grow, col0, 32, row_ok);
           }
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            v[j] = (v[j] - mean) * rstd * gcache[(4 + slot) * 32 + j] + gcache[(8 + slot) * 32 + j];
+          for (int k = 0; k < 8; ++k) {
+            const float4 g = cg[k], t = ct[k];
+            v[4 * k] = (v[4 * k] - mean) * rstd * g.x + t.x;
+            v[4 * k + 1] = (v[4 * k + 1] - mean) * rstd * g.y + t.y;
+            v[4 * k + 2] = (v[4 * k + 2] - mean) * rstd * g.z + t.z;
+            v[4 * k + 3] = (v[4 * k + 3] - mean) * rstd * g.w + t.w;
+          }
           run_chain<POST>(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
           if (c_tma)
             store_tile32_tma(stage, lane, v, &tmC, col0, wrow0);
@@ -582,15 +643,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         // (count, mean, M2) of this thread's chunks c0, c0+step, ... < c1 in one pass over
         // TMEM: exact two-pass moments of each 32-value chunk in registers, merged
         // chunk by chunk with Chan's formula.
-        auto moments = [&](uint32_t tb, int32_t colbase, int c0, int c1, int step, float& n, float& mean, float& m2) {
+        // With `cached`, a bias pre-chain reads the chunks' bias from the cache
+        // (parked for chunks c0, c0 + step, ... in order).
+        auto moments = [&](uint32_t tb, int32_t colbase, int c0, int c1, int step, float& n, float& mean, float& m2,
+                           bool cached) {
           n = 0.0f;
           mean = 0.0f;
           m2 = 0.0f;
-          for (int c = c0; c < c1; c += step) {
+          int slot = 0;
+          for (int c = c0; c < c1; c += step, ++slot) {
             __syncwarp();
             float v[32];
             tmem_ld32(tb + c * 32, v);
-            run_chain<PRE>(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+            if (cached && pre_bias) {
+              const float4* cb = reinterpret_cast<const float4*>(gcache + slot * 32);
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const float4 b = cb[k];
+                v[4 * k] += b.x;
+                v[4 * k + 1] += b.y;
+                v[4 * k + 2] += b.z;
+                v[4 * k + 3] += b.w;
+              }
+            } else {
+              run_chain<PRE>(false, p.pre, p.n_pre, v, grow, colbase + c * 32, 32, row_ok);
+            }
             float sum = 0.0f;
 #pragma unroll
             for (int j = 0; j < 32; ++j) sum += v[j];
@@ -601,7 +678,64 @@ __global__ void __launch_bounds__(kThreads, 1)
             chan(n, mean, m2, 32.0f, cmean, cq, n, mean, m2);
           }
         };
-        if (gs < BN) {
+        if (QUAD || (gs == BN && sub_tiles == 1)) {
+          // One accumulator holds this CTA's columns of the group: the whole
+          // group (gs = BN), or (quad) one 256-column half of a 512-column group
+          // whose other half CTA rank ^ 2 holds for the same rows.  The
+          // quadrant's two warps split the chunks and merge their moments; with
+          // quad, half 0 then sends (mean, M2) of this CTA's 256 columns to the
+          // other CTA through distributed shared memory, and both CTAs merge the
+          // two column halves in the same order (the lower half first), so both
+          // normalise with identical statistics.  Slot tl & 1 is written for tile
+          // tl only after the other CTA has passed tile tl - 1, which it reached
+          // after reading slot tl & 1 for tile tl - 2.
+          issue_vecs(ui.n0, h, BN / 32, 2);  // in flight across the wait
+          if (!pair_vote(wait_acc(tl))) { ok = false; break; }
+          park_vecs();
+          const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
+          float n, mean, m2;
+          moments(tb, ui.n0, h, BN / 32, 2, n, mean, m2, true);
+          xch[h * kBM + row_in_tile] = make_float2(mean, m2);
+          pair_sync();
+          const float2 o = xch[(h ^ 1) * kBM + row_in_tile];
+          pair_sync();
+          float tn, tm, tq;
+          if (h == 0)
+            chan(n, mean, m2, n, o.x, o.y, tn, tm, tq);
+          else
+            chan(n, o.x, o.y, n, mean, m2, tn, tm, tq);
+          if constexpr (QUAD) {
+            const float cn = tn, cm = tm, cq = tq;
+            const int slot = tl & 1;
+            const uint32_t other = rank ^ 2u;
+            if (h == 0) {
+              st_cluster_f2(mapa_shared(smem_u32(xs + slot * kBM + row_in_tile), other), cm, cq);
+              mbar_arrive_remote(mapa_shared(smem_u32(&xbar[slot]), other));
+            }
+            bool got = mbar_wait_cluster(&xbar[slot], (tl >> 1) & 1, abort_flag, p.wait_ns);
+            got = __all_sync(0xffffffffu, got);
+            if (!pair_vote(got)) {
+              *abort_flag = 1;
+              if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+              ok = false;
+              break;
+            }
+            const float2 r = xs[slot * kBM + row_in_tile];
+            if ((rank >> 1) == 0)
+              chan(cn, cm, cq, cn, r.x, r.y, tn, tm, tq);
+            else
+              chan(cn, r.x, r.y, cn, cm, cq, tn, tm, tq);
+          }
+          const float rstd = rsqrtf(tq / tn + eps);
+          int cs = 0;
+          for (int c = h; c < BN / 32; c += 2, ++cs) {
+            __syncwarp();
+            finish_chunk(tb + c * 32, ui.n0 + c * 32, tm, rstd, cs);
+          }
+          __syncwarp();
+          release_acc(tl);
+          ++tl;
+        } else if (gs < BN) {
           // several whole groups per tile: half h takes groups h, h+2, ...
           if (!wait_acc(tl)) { ok = false; break; }
           const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
@@ -610,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int32_t g0 = ui.n0 + gi * gs;
             if (g0 >= p.N) break;
             float n, mean, m2;
-            moments(tb + gi * gs, g0, 0, nch, 1, n, mean, m2);
+            moments(tb + gi * gs, g0, 0, nch, 1, n, mean, m2, false);
             const float rstd = rsqrtf(m2 / n + eps);
             fill_cache(g0, 0, nch, 1);
             for (int c = 0; c < nch; ++c) {
@@ -629,20 +763,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!pair_vote(wait_acc(tl + st))) { ok = false; break; }
             const uint32_t tb = tmem + lane_off + ((tl + st) & 1) * Cfg::kAccStride;
             float nb, mb, qb;
-            moments(tb, ui.n0 + st * BN, h, BN / 32, 2, nb, mb, qb);
+            moments(tb, ui.n0 + st * BN, h, BN / 32, 2, nb, mb, qb, false);
             chan(n, mean, m2, nb, mb, qb, n, mean, m2);
           }
           if (!ok) break;
-          xch[(h * 4 + q) * 32 + lane] = make_float4(n, mean, m2, 0.f);
+          // the two halves hold equally many columns: only (mean, M2) travel
+          xch[h * kBM + row_in_tile] = make_float2(mean, m2);
           pair_sync();
-          const float4 o = xch[((h ^ 1) * 4 + q) * 32 + lane];
+          const float2 o = xch[(h ^ 1) * kBM + row_in_tile];
           pair_sync();
           // both halves merge in the same order (half 0 first) -> identical stats
           float tn, tm, tq;
           if (h == 0)
-            chan(n, mean, m2, o.x, o.y, o.z, tn, tm, tq);
+            chan(n, mean, m2, n, o.x, o.y, tn, tm, tq);
           else
-            chan(o.x, o.y, o.z, n, mean, m2, tn, tm, tq);
+            chan(n, o.x, o.y, n, mean, m2, tn, tm, tq);
           const float rstd = rsqrtf(tq / tn + eps);
           for (int st = 0; st < sub_tiles; ++st) {
             const uint32_t tb = tmem + lane_off + ((tl + st) & 1) * Cfg::kAccStride;

@@ -8,8 +8,8 @@ namespace {
 
 template <int BN, int STAGES, int MODE>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int grid, cudaStream_t s) {
-  using Cfg = TcCfg<BN, STAGES, MODE, true, false>;
-  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, false>;
+  using Cfg = TcCfg<BN, STAGES, MODE, true, kClOne>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, kClOne>;
   static bool configured[64] = {};  // the attribute is per device
   int dev = 0;
   cudaGetDevice(&dev);

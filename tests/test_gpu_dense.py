@@ -161,6 +161,19 @@ def test_groupnorm_swish(N, groups):
     _no_device_error()
 
 
+@pytest.mark.parametrize("post", ["silu", "gelu_tanh"])  # compiled program / interpreter
+def test_groupnorm_512_many_units_per_cluster(post):
+    # 4 ragged 256-row tiles x 24 groups of 512 = 96 units: more than the clusters
+    # of four that fit at once, so every cluster reuses its statistics slots
+    inp = kf_workloads.generate("bf16_groupnorm_swish", seed=17, M=1000, N=12288, K=136)
+    chain = [("bias", {"p0": inp["b"]}),
+             ("groupnorm", {"groups": 24, "eps": 1e-5, "p0": inp["gamma"], "p1": inp["beta"]}),
+             (post, {})]
+    Y = kf.fused_gemm(inp["X"].to(DEV), inp["W"].to(DEV), chain_to(chain, DEV))
+    check_bf16(Y, oracle.fused_gemm(inp["X"], inp["W"], chain), f"gn 512 x96 {post}")
+    _no_device_error()
+
+
 def test_groupnorm_no_affine_unit_moments():
     inp = kf_workloads.generate("bf16_groupnorm_swish", seed=9, M=130, N=1024, K=64, dist="unscaled")
     chain = [("groupnorm", {"groups": 2, "eps": 1e-5})]
