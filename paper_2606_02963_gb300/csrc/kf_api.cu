@@ -94,6 +94,22 @@ kf_status make_map_out(CUtensorMap* m, void* base, uint64_t cols, uint64_t rows,
   return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
 }
 
+// bf16 [rows x cols] map with 32 x 32 boxes in the 64-byte swizzle: the
+// residual-tile kernels load the residual and store the output through it.
+kf_status make_map_blk64(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes) {
+  auto fn = encode_fn();
+  if (!fn) return KF_ERR_CUDA;
+  std::memset(m, 0, sizeof(*m));
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 int elt_size(int dt) { return dt == KF_BF16 ? 2 : 4; }
 bool float_dtype(int dt) { return dt == KF_F32 || dt == KF_BF16; }
@@ -502,8 +518,20 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
   // a compiled chain program, if the chain matches one (bf16 operands staged)
   int sig = kSigGeneric;
-  if (pl.mode == kModeStore && ProgGeluChain::matches(pl.pre, pl.n_pre) && p.vec_op == 0 && p.res_op == 3)
+  CUtensorMap mr;
+  std::memset(&mr, 0, sizeof(mr));
+  // bias-GELU-scale-residual on CTA pairs: the residual tile goes through shared
+  // memory (TMA in, in-place result, TMA out) -- needs TMA-able residual and
+  // output and whole 8-column bias units
+  if (pl.mode == kModeStore && ProgGeluChain::matches(pl.pre, pl.n_pre) && p.vec_op == 0 && p.res_op == 3 && cta2 &&
+      p.c_tma && N % 8 == 0 && tc_dense2_has_prog(pl.mode, bn, kSigBiasGeluScaleRes)) {
     sig = kSigBiasGeluScaleRes;
+    const DevOp& ro = pl.pre[3];
+    st = make_map_blk64(&mr, ro.p0, static_cast<uint64_t>(N), static_cast<uint64_t>(M), static_cast<uint64_t>(ro.ld) * 2);
+    if (st != KF_OK) return st;
+    st = make_map_blk64(&mc, Y, static_cast<uint64_t>(N), static_cast<uint64_t>(M), static_cast<uint64_t>(ldy) * 2);
+    if (st != KF_OK) return st;
+  }
   else if (pl.mode == kModeGroupNorm && ProgBias::matches(pl.pre, pl.n_pre) && ProgSilu::matches(pl.post, pl.n_post))
     sig = kSigBiasNormSilu;
   else if (pl.mode == kModeLse && ProgScale::matches(pl.pre, pl.n_pre))
@@ -511,7 +539,7 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   if (quad)
     st = cuda_status(tc_dense4_launch(pl.mode, bn, sig, ma, mb, mc, p, s));
   else
-    st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, p, sub, grid, s));
+    st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, mr, p, sub, grid, s));
   if (st != KF_OK || pl.mode != kModeLse) return st;
   LseCombineParams cp;
   std::memset(&cp, 0, sizeof(cp));

@@ -186,6 +186,14 @@ __device__ __forceinline__ void st32(void* p, int dt, int64_t i0, int nvalid, bo
 __device__ __forceinline__ uint32_t xpose_off(int row, int unit) {
   return static_cast<uint32_t>(row * 32 + ((unit ^ ((row >> 2) & 1)) << 4));
 }
+// 64-byte-swizzled block of 32 bf16 columns (64 B per row): the 16-byte unit u
+// of row r sits at unit u ^ ((r >> 1) & 3), the layout TMA's SWIZZLE_64B mode
+// reads and writes.  One row per lane: each 16-byte access of a warp touches
+// every bank group once per 8 rows (no conflicts beyond the 4 wavefronts that
+// 512 bytes need).
+__device__ __forceinline__ uint32_t sw64_off(int row, int unit) {
+  return static_cast<uint32_t>(row * 64 + ((unit ^ ((row >> 1) & 3)) << 4));
+}
 
 // Store the lane's 32 values (row `lane`) as bf16 to rows [0, rows) of the
 // 32 x 32 block at `gbase` (row stride ld elements).
@@ -581,6 +589,7 @@ template <int... KINDS>
 struct Prog {
   static constexpr int kLen = sizeof...(KINDS);
   static constexpr bool kGeneric = false;
+  static constexpr bool kHasRes = ((KINDS == KF_OP_RESIDUAL_ADD) || ... || false);
   template <bool FAST>
   __device__ __forceinline__ static void run(const DevOp* ops, float (&v)[32], int64_t row, int64_t col0, int nvalid,
                                              bool row_ok, const Staged32& st) {
@@ -598,6 +607,7 @@ struct Prog {
 };
 struct Interp {
   static constexpr bool kGeneric = true;
+  static constexpr bool kHasRes = false;
   template <bool FAST>
   __device__ __forceinline__ static void run(const DevOp* ops, int n, float (&v)[32], int64_t row, int64_t col0,
                                              int nvalid, bool row_ok, const Staged32& st) {

@@ -15,7 +15,7 @@ using ProgSilu = Prog<KF_OP_SILU>;
 using ProgScale = Prog<KF_OP_SCALE>;
 enum ChainSig : int {
   kSigGeneric = 0,
-  kSigBiasGeluScaleRes = 1,  // store:      pre = ProgGeluChain
+  kSigBiasGeluScaleRes = 1,  // store:      pre = ProgGeluChain (CTA pairs: residual tile)
   kSigBiasNormSilu = 2,      // GroupNorm:  pre = ProgBias, post = ProgSilu
   kSigScaleLse = 3,          // row LSE:    pre = ProgScale, post = none
 };
@@ -27,11 +27,16 @@ enum ChainSig : int {
 // cta2), else the interpreter variant runs.
 bool tc_dense_has(int mode, int bn, bool cta2);
 bool tc_dense2_has(int mode, int bn);
+bool tc_dense2_has_prog(int mode, int bn, int sig);  // a compiled chain program for (mode, bn, sig)
 bool tc_grouped_has(int mode, int bn);
+// `c` is the output map of the TMA stores, `r` the residual map of the
+// residual-tile variants (unused by the others).
 cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,
-                            const CUtensorMap& c, const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
+                            const CUtensorMap& c, const CUtensorMap& r, const TcParams& p, int sub_tiles, int grid,
+                            cudaStream_t s);
 cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
-                             const CUtensorMap& c, const TcParams& p, int sub_tiles, int grid, cudaStream_t s);
+                             const CUtensorMap& c, const CUtensorMap& r, const TcParams& p, int sub_tiles, int grid,
+                             cudaStream_t s);
 cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                               const TcParams& p, int grid, cudaStream_t s);
 // GroupNorm over 512-column groups on clusters of two CTA pairs (one 256-column

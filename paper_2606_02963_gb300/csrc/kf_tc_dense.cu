@@ -9,8 +9,8 @@ namespace kf {
 namespace {
 
 template <int BN, int STAGES, int MODE>
-cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int sub, int grid,
-                       cudaStream_t s) {
+cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& r,
+                       const TcParams& p, int sub, int grid, cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, kClOne>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClOne>;
   static bool configured[64] = {};  // the attribute is per device
@@ -22,7 +22,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, p, sub);
+  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, r, p, sub);
   return cudaGetLastError();
 }
 
@@ -49,10 +49,11 @@ bool tc_dense_has(int mode, int bn, bool cta2) {
 }
 
 cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,
-                            const CUtensorMap& c, const TcParams& p, int sub, int grid, cudaStream_t s) {
-  if (cta2) return tc_dense2_launch(mode, bn, sig, a, b, c, p, sub, grid, s);
+                            const CUtensorMap& c, const CUtensorMap& r, const TcParams& p, int sub, int grid,
+                            cudaStream_t s) {
+  if (cta2) return tc_dense2_launch(mode, bn, sig, a, b, c, r, p, sub, grid, s);
 #define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, p, sub, grid, s);
+  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, r, p, sub, grid, s);
   KF_DENSE_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;

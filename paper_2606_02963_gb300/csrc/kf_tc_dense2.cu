@@ -13,9 +13,9 @@ namespace kf {
 namespace {
 
 template <int BN, int STAGES, int MODE, class PRE = Interp, class POST = Interp>
-cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int sub, int grid,
-                        cudaStream_t s) {
-  using Cfg = TcCfg<BN, STAGES, MODE, false, kClPair>;
+cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& r,
+                        const TcParams& p, int sub, int grid, cudaStream_t s) {
+  using Cfg = TcCfg<BN, STAGES, MODE, false, kClPair, kResTileFor<MODE, false, kClPair, PRE>>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClPair, PRE, POST>;
   static bool configured[64] = {};
   int dev = 0;
@@ -39,7 +39,7 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtens
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, a, b, c, p, static_cast<int32_t>(sub));
+  return cudaLaunchKernelEx(&cfg, kern, a, b, c, r, p, static_cast<int32_t>(sub));
 }
 
 // Cluster of four (two CTA pairs).  The persistent grid holds as many clusters
@@ -78,7 +78,8 @@ cudaError_t launch_quad(const CUtensorMap& a, const CUtensorMap& b, const CUtens
   const int clusters = std::min(p.total_units, max_clusters[dev]);
   if (clusters < 1) return cudaSuccess;
   cfg.gridDim = dim3(4 * clusters, 1, 1);
-  return cudaLaunchKernelEx(&cfg, kern, a, b, c, p, static_cast<int32_t>(1));
+  static const CUtensorMap none = {};  // GroupNorm stages no residual tile
+  return cudaLaunchKernelEx(&cfg, kern, a, b, c, none, p, static_cast<int32_t>(1));
 }
 
 }  // namespace
@@ -112,21 +113,33 @@ bool tc_dense2_has(int mode, int bn) {
 }
 
 // Chain-program variants: (mode, BN, stages, signature, PRE, POST)
+// (the residual-tile variants give BN x 256 B of shared memory to the residual
+// tile, so their rings are one or two stages shorter)
 #define KF_DENSE2_PROG_VARIANTS(X)                                              \
-  X(kModeStore, 224, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
-  X(kModeStore, 256, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 128, 7, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 192, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 224, 5, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 256, 4, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
   X(kModeGroupNorm, 256, 6, kSigBiasNormSilu, ProgBias, ProgSilu)               \
   X(kModeLse, 224, 6, kSigScaleLse, ProgScale, Interp)                          \
   X(kModeLse, 256, 6, kSigScaleLse, ProgScale, Interp)
 
-cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p,
-                             int sub, int grid, cudaStream_t s) {
+bool tc_dense2_has_prog(int mode, int bn, int sig) {
 #define Y(M_, B_, S_, G_, PRE_, POST_) \
-  if (mode == M_ && bn == B_ && sig == G_) return launch_pair<B_, S_, M_, PRE_, POST_>(a, b, c, p, sub, grid, s);
+  if (mode == M_ && bn == B_ && sig == G_) return true;
+  KF_DENSE2_PROG_VARIANTS(Y)
+#undef Y
+  return false;
+}
+
+cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                             const CUtensorMap& r, const TcParams& p, int sub, int grid, cudaStream_t s) {
+#define Y(M_, B_, S_, G_, PRE_, POST_) \
+  if (mode == M_ && bn == B_ && sig == G_) return launch_pair<B_, S_, M_, PRE_, POST_>(a, b, c, r, p, sub, grid, s);
   KF_DENSE2_PROG_VARIANTS(Y)
 #undef Y
 #define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_pair<B_, S_, M_>(a, b, c, p, sub, grid, s);
+  if (mode == M_ && bn == B_) return launch_pair<B_, S_, M_>(a, b, c, r, p, sub, grid, s);
   KF_DENSE2_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;

@@ -55,13 +55,22 @@ constexpr int kClOne = 0;
 constexpr int kClPair = 1;
 constexpr int kClQuad = 2;
 
-template <int BN, int STAGES, int MODE, bool GROUPED, int CL>
+// Residual tile: dense CTA-pair store kernels whose compiled chain adds a bf16
+// residual stage the whole residual tile in shared memory by TMA (each epilogue
+// warp loads its own rows x chunks before it waits for the accumulator), add it
+// from there, write the bf16 result in place and send each 32 x 32 block out
+// with one TMA store.
+template <int MODE, bool GROUPED, int CL, class PRE>
+constexpr bool kResTileFor = MODE == kModeStore && !GROUPED && CL == kClPair && PRE::kHasRes;
+
+template <int BN, int STAGES, int MODE, bool GROUPED, int CL, bool RT = false>
 struct TcCfg {
   static constexpr bool CTA2 = CL != kClOne;  // tcgen05 CTA-pair MMAs
   static constexpr bool kQuad = CL == kClQuad;
   static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN");
   static_assert(!(GROUPED && CTA2), "grouped GEMMs use single-CTA tiles");
   static_assert(!kQuad || (MODE == kModeGroupNorm && BN == 256), "quad clusters split 512-column groups");
+  static_assert(!RT || (MODE == kModeStore && !GROUPED && CL == kClPair), "residual tile: dense CTA-pair store");
   static constexpr int kOutN = (MODE == kModeSwiglu) ? BN / 2 : BN;  // output columns of a (sub)tile
   // With CTA pairs each CTA stages its own 128 rows of A and half of the BN rows of B.
   static constexpr int kBRows = CTA2 ? BN / 2 : BN;
@@ -72,11 +81,14 @@ struct TcCfg {
   // accumulator buffer b starts at TMEM column b * kAccStride
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
-  static constexpr int kBarBytes = (8 * (2 * STAGES + 7) + 63) / 64 * 64;  // keeps what follows 64-B aligned
+  static constexpr int kBarBytes = (8 * (2 * STAGES + 7 + kEpiWarps) + 63) / 64 * 64;  // keeps what follows 64-B aligned
   // per-warp 1 KB tile buffers (1 KB aligned, right after the stages): two for
   // the asynchronous TMA stores, plus (store mode) one for the residual
   // transposition, which must not reuse a buffer a TMA store may still read
-  static constexpr int kWarpStaging = (MODE == kModeStore) ? 3072 : 2048;
+  // (residual tile: 256 B per warp, the bias of its chunks)
+  static constexpr int kWarpStaging = RT ? 256 : ((MODE == kModeStore) ? 3072 : 2048);
+  // residual tile: BN / 32 chunks x 128 rows x 64 B (64-byte swizzle), 2 KB per warp and chunk
+  static constexpr int kResTileBytes = RT ? BN * 256 : 0;
   static constexpr int kStagingBytes = kEpiWarps * kWarpStaging;
   // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
   static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiWarps * 3 * 4 * 32 * 4 : 0;
@@ -84,7 +96,8 @@ struct TcCfg {
   // + (quad) the other pair's per-row statistics, two slots (2 KB)
   static constexpr int kMiscBytes = 64 + 2 * kBM * 8 + (kQuad ? 2 * kBM * 8 : 0);
   static constexpr int kTableBytes = GROUPED ? 8 * (kMaxGroups + 1) : 0;
-  static constexpr int kSmemUse = STAGES * kStageBytes + kStagingBytes + kGnCacheBytes + kBarBytes + kMiscBytes + kTableBytes;
+  static constexpr int kSmemUse =
+      STAGES * kStageBytes + kResTileBytes + kStagingBytes + kGnCacheBytes + kBarBytes + kMiscBytes + kTableBytes;
   // pad to > half of the SM's shared memory so that at most one such CTA is
   // resident per SM (tensor-memory allocation then never has to wait)
   static constexpr int kSmemBytes = 1024 + (kSmemUse > 120 * 1024 ? kSmemUse : 120 * 1024);
@@ -102,9 +115,10 @@ struct UnitInfo {
 template <int BN, int STAGES, int MODE, bool GROUPED, int CL, class PRE = Interp, class POST = Interp>
 __global__ void __launch_bounds__(kThreads, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                      const __grid_constant__ CUtensorMap tmC, const __grid_constant__ TcParams p,
-                      const int32_t sub_tiles) {
-  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CL>;
+                      const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmR,
+                      const __grid_constant__ TcParams p, const int32_t sub_tiles) {
+  constexpr bool RT = kResTileFor<MODE, GROUPED, CL, PRE>;
+  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CL, RT>;
   constexpr bool CTA2 = Cfg::CTA2;
   constexpr bool QUAD = Cfg::kQuad;
   constexpr bool PRE_IS_BIAS = IsBiasProg<PRE>::value;
@@ -112,7 +126,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* smB = sm;                                // B stages first: any over-read stays inside the CTA
   uint8_t* smA = sm + STAGES * Cfg::kBBytes;
-  uint8_t* staging = sm + STAGES * Cfg::kStageBytes;           // epilogue tile buffers
+  uint8_t* rtile = sm + STAGES * Cfg::kStageBytes;             // residual tile (RT)
+  uint8_t* staging = rtile + Cfg::kResTileBytes;                // epilogue tile buffers
   float* gn_cache = reinterpret_cast<float*>(staging + Cfg::kStagingBytes);
   uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::kStagingBytes + Cfg::kGnCacheBytes);
   uint64_t* full = bars;
@@ -121,6 +136,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* acce = bars + 2 * STAGES + 2;
   uint64_t* drain = bars + 2 * STAGES + 4;
   uint64_t* xbar = bars + 2 * STAGES + 5;  // quad: the other pair's statistics have landed (2 slots)
+  uint64_t* rbar = bars + 2 * STAGES + 7;  // residual tile: warp ew's rows have landed (kEpiWarps)
   uint32_t* misc = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(bars) + Cfg::kBarBytes);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
@@ -156,6 +172,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&xbar[0], kBM);  // one arrival per row of the other pair's CTA
       mbar_init(&xbar[1], kBM);
     }
+    if constexpr (RT)
+      for (int w = 0; w < kEpiWarps; ++w) mbar_init(&rbar[w], 1);
     *abort_flag = 0;
     *zero_flag = 0;
     *total_s = GROUPED ? 0 : p.total_units;
@@ -165,6 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    if constexpr (RT) tma_prefetch_desc(&tmR);
   }
   if (warp == 1) {
     __syncwarp();
@@ -378,6 +397,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool c_tma = p.c_tma != 0;
     int32_t tl = 0;
     bool ok = true;
+    // residual tile state: the warp's bias cache, the bias vector, whether a
+    // residual load is in flight and the phase of its barrier
+    uint8_t* bcache = staging + ew * Cfg::kWarpStaging;
+    const __nv_bfloat16* rt_bias_ptr =
+        RT ? reinterpret_cast<const __nv_bfloat16*>(p.pre[p.vec_op < 0 ? 0 : p.vec_op].p0) : nullptr;
+    bool rt_pending = false;
+    uint32_t rt_phase = 0;
 
     auto wait_acc = [&](int32_t t) -> bool {
       bool w = mbar_wait(&accf[t & 1], (t >> 1) & 1, abort_flag, p.wait_ns);
@@ -433,7 +459,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int32_t wrow0 = ui.m0 + q * 32;                      // first row of this warp's 32
       const int wrows = max(0, min(32, ui.m_end - wrow0));       // rows of them that exist
       // pull this unit's residual rows toward L2 while its mainloop runs
-      if (res_staged && row_ok) {
+      if (!RT && res_staged && row_ok) {
         const DevOp& ro = p.pre[p.res_op];
         const __nv_bfloat16* rp = reinterpret_cast<const __nv_bfloat16*>(ro.p0) + static_cast<int64_t>(grow) * ro.ld;
         for (int c = h + 2; c < Cfg::kOutN / 32; c += 2)
@@ -453,8 +479,43 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (vec_staged) vec32_issue(p.pre[p.vec_op].p0, col0, bq);
         };
-        if constexpr (MODE == kModeStore) issue_chunk(h);
+        // residual tile: this warp's chunks of the residual (TMA) and of the bias
+        // (one 16-byte unit per lane 0..15) are requested before the wait
+        uint4 rt_bias = make_uint4(0u, 0u, 0u, 0u);
+        if constexpr (RT) {
+          if (lane < 16) {
+            const int c = h + 2 * (lane >> 2);
+            const int32_t col = ui.n0 + c * 32 + (lane & 3) * 8;
+            if (c < Cfg::kOutN / 32 && col + 8 <= p.N) rt_bias = ldg_v4_pinned(rt_bias_ptr + col);
+          }
+          if (lane == 0) {
+            bulk_wait_group_read<0>();  // this warp's stores of the previous tile have read its blocks
+            uint32_t bytes = 0;
+            for (int c = h; c < Cfg::kOutN / 32; c += 2)
+              if (ui.n0 + c * 32 < p.N) bytes += 2048;
+            mbar_arrive_expect_tx(&rbar[ew], bytes);
+            for (int c = h; c < Cfg::kOutN / 32; c += 2)
+              if (ui.n0 + c * 32 < p.N) tma_load_2d(rtile + c * 8192 + q * 2048, &tmR, &rbar[ew], ui.n0 + c * 32, wrow0);
+          }
+          rt_pending = true;
+        } else if constexpr (MODE == kModeStore) {
+          issue_chunk(h);
+        }
         if (!wait_acc(tl)) { ok = false; break; }
+        if constexpr (RT) {
+          if (lane < 16) *reinterpret_cast<uint4*>(bcache + (lane >> 2) * 64 + (lane & 3) * 16) = rt_bias;
+          bool got = mbar_wait(&rbar[ew], rt_phase, abort_flag, p.wait_ns);
+          got = __all_sync(0xffffffffu, got);
+          if (!got) {
+            *abort_flag = 1;
+            if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+            ok = false;
+            break;
+          }
+          rt_pending = false;
+          rt_phase ^= 1u;
+          __syncwarp();
+        }
         const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
         float rs = 0.0f;
         int32_t dst = 0;
@@ -475,7 +536,45 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (nvalid <= 0) break;  // uniform across the warp
           __syncwarp();
           float v[32];
-          if constexpr (MODE == kModeStore) {
+          if constexpr (RT) {
+            // residual from the tile (64-byte swizzle, row = lane), bias from the
+            // warp's cache; the result overwrites the residual in place
+            uint8_t* blk = rtile + c * 8192 + q * 2048;
+            const uint4* bc = reinterpret_cast<const uint4*>(bcache + ((c - h) >> 1) * 64);
+            Staged32 sg;
+            sg.use_res = true;
+            sg.vec_idx = p.vec_op;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const uint4 r = *reinterpret_cast<const uint4*>(blk + sw64_off(lane, u));
+              const uint4 b = bc[u];
+              sg.res[4 * u] = r.x;
+              sg.res[4 * u + 1] = r.y;
+              sg.res[4 * u + 2] = r.z;
+              sg.res[4 * u + 3] = r.w;
+              sg.vec[4 * u] = b.x;
+              sg.vec[4 * u + 1] = b.y;
+              sg.vec[4 * u + 2] = b.z;
+              sg.vec[4 * u + 3] = b.w;
+            }
+            tmem_ld32(tb + c * 32, v);
+            run_chain<PRE>(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok, sg);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              uint4 w;
+              w.x = pack_bf16x2(v[8 * u + 0], v[8 * u + 1]);
+              w.y = pack_bf16x2(v[8 * u + 2], v[8 * u + 3]);
+              w.z = pack_bf16x2(v[8 * u + 4], v[8 * u + 5]);
+              w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
+              *reinterpret_cast<uint4*>(blk + sw64_off(lane, u)) = w;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmC, blk, col0, wrow0);  // rows / columns outside Y are clipped
+              bulk_commit_group();
+            }
+          } else if constexpr (MODE == kModeStore) {
             // operands of this chunk were issued one chunk ahead; issue the next
             Staged32 sg;
             sg.use_res = res_staged && nvalid == 32;
@@ -503,7 +602,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld32(tb + c * 32, v);
             run_chain<PRE>(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
           }
-          if constexpr (MODE == kModeScatter) {
+          if constexpr (RT) {
+            // stored above
+          } else if constexpr (MODE == kModeScatter) {
             if (wr) {
               float* dstp = reinterpret_cast<float*>(p.C) + static_cast<int64_t>(dst) * p.ldc + col0;
               if (nvalid == 32 && p.c_vec_ok) {
@@ -793,6 +894,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           tl += sub_tiles;
         }
       }
+    }
+    // a residual load still in flight after an abort lands before the CTA exits
+    if constexpr (RT) {
+      if (rt_pending && lane == 0) mbar_wait(&rbar[ew], rt_phase, zero_flag, p.drain_ns);
     }
   }
 

@@ -19,7 +19,8 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, p, 1);
+  static const CUtensorMap none = {};  // grouped variants stage no residual tile
+  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, none, p, 1);
   return cudaGetLastError();
 }
 

@@ -96,6 +96,25 @@ def test_gelu_scale_residual_chain_sweep(dist):
     _no_device_error()
 
 
+@pytest.mark.parametrize("in_place", [False, True])
+def test_gelu_chain_more_tiles_than_cta_pairs(in_place):
+    # 4 ragged 256-row tiles x 20 column tiles of 224 = 80 tiles: more than the
+    # CTA pairs of the grid, so pairs run a second tile and reload their
+    # residual tile in shared memory after the first tile's stores
+    inp = kf_workloads.generate("bf16_gelu_scale_residual", seed=14, M=1000, N=4480, K=136, dist="unscaled")
+    chain = wl_chain("bf16_gelu_scale_residual", inp)
+    ref = oracle.fused_gemm(inp["X"], inp["W"], chain)
+    gchain = chain_to(chain, DEV)
+    if in_place:
+        R = inp["R"].to(DEV).clone()
+        gchain[-1] = ("residual_add", {"p0": R})
+        Y = kf.fused_gemm(inp["X"].to(DEV), inp["W"].to(DEV), gchain, out=R)
+    else:
+        Y = kf.fused_gemm(inp["X"].to(DEV), inp["W"].to(DEV), gchain)
+    check_bf16(Y, ref, f"80 tiles, in place {in_place}")
+    _no_device_error()
+
+
 def test_residual_in_place():
     inp = kf_workloads.generate("bf16_gelu_scale_residual", seed=8, M=256, N=256, K=128)
     chain = wl_chain("bf16_gelu_scale_residual", inp)
