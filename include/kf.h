@@ -113,8 +113,13 @@ typedef struct kf_epilogue {
  *   fp32; element-wise chains only).
  *   bf16 path: X, W must be 16-byte aligned with ldx, ldw multiples of 8, else
  *   KF_ERR_MISALIGNED.  M == 0 or N == 0 is a no-op; K must be >= 1.
- *   workspace: kf_fused_gemm_workspace() bytes (0 unless the chain holds a row
- *   log-sum-exp, which keeps per-tile row partials there).
+ *   workspace: kf_fused_gemm_workspace() bytes.  Required for a row
+ *   log-sum-exp (per-tile row partials live there).  Optional for GroupNorm over
+ *   512-column groups with M > 128: with it, pairs of CTA pairs exchange per-row
+ *   statistics through it (all SMs work; the launch is cooperative); with a
+ *   smaller or no workspace, clusters of four CTAs exchange them on chip (fewer
+ *   SMs can be used).  Same results either way.  0 otherwise.  Calls that share
+ *   one workspace must not overlap on the GPU.
  *   Y must not alias X or W; a RESIDUAL_ADD operand may alias Y (in place).
  */
 kf_status kf_fused_gemm(const void* X, int32_t x_dtype, int64_t ldx, const void* W, int32_t w_dtype,

@@ -4,6 +4,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <chrono>
 #include <cstring>
 #include <mutex>
 
@@ -301,6 +302,36 @@ uint32_t mode_box(int mode, int bn) { return mode == kModeSwiglu ? bn / 2 : bn; 
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// GroupNorm couples: statistics exchange area for up to kMaxCouples couples
+// ([couples][2 slots][2 halves][256 rows] float2, then [couples][2][2][8] flags)
+constexpr int kMaxCouples = 128;
+constexpr size_t kCoupleDataBytes = 2 * 2 * 256 * sizeof(float) * 2;
+constexpr size_t kCoupleFlagBytes = 2 * 2 * 8 * sizeof(unsigned long long);
+int couple_slots(int64_t M, int64_t N) {
+  const int64_t units = ((M + 255) / 256) * (N / 512);
+  return static_cast<int>(std::min<int64_t>(units, kMaxCouples));
+}
+size_t couple_ws_bytes(int64_t M, int64_t N) {
+  return align_up(static_cast<size_t>(couple_slots(M, N)) * (kCoupleDataBytes + kCoupleFlagBytes), 256);
+}
+// True when the chain normalises 512-column groups and M spans CTA pairs: the
+// case the couples (with a workspace) and clusters of four (without) serve.
+bool gn512_pairs(const kf_epilogue* epi, int64_t M, int64_t N) {
+  if (M <= 128 || !epi || !epi->ops) return false;
+  for (int i = 0; i < epi->num_ops; ++i)
+    if (epi->ops[i].kind == KF_OP_GROUPNORM)
+      return epi->ops[i].groups > 0 && N % epi->ops[i].groups == 0 && N / epi->ops[i].groups == 512;
+  return false;
+}
+// Per-call tag of the couples' flags: unique within the process, and seeded from
+// the clock so that flags left in reused memory by another process do not match.
+uint32_t next_epoch() {
+  static std::atomic<uint32_t> ctr{static_cast<uint32_t>(
+      std::chrono::steady_clock::now().time_since_epoch().count() * 2654435761ull)};
+  uint32_t e = ctr.fetch_add(1);
+  return e == 0 ? ctr.fetch_add(1) : e;
+}
+
 size_t lse_ws_bytes(int64_t M, int64_t N) {
   // upper bound over all tile widths (narrowest tile = most partials per row)
   return align_up(static_cast<size_t>(M) * static_cast<size_t>((N + 127) / 128) * sizeof(float2), 256);
@@ -418,6 +449,7 @@ size_t kf_fused_gemm_workspace(int64_t M, int64_t N, int64_t K, const kf_epilogu
   if (!epi || M <= 0 || N <= 0) return 0;
   for (int i = 0; i < epi->num_ops && epi->ops; ++i)
     if (epi->ops[i].kind == KF_OP_ROW_LOGSUMEXP) return lse_ws_bytes(M, N);
+  if (gn512_pairs(epi, M, N)) return couple_ws_bytes(M, N);  // optional: enables the couples
   return 0;
 }
 
@@ -473,6 +505,10 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   // GroupNorm over 512-column groups: clusters of two CTA pairs, one 256-column
   // half of each group per pair, so each CTA double-buffers its accumulators
   const bool quad = cta2 && pl.mode == kModeGroupNorm && pl.gs == 512 && di.nsm >= 4 && tc_dense4_has(pl.mode, 256);
+  // with a workspace for the statistics exchange: couples of CTA pairs instead
+  // (all co-resident pairs work; clusters of four leave SMs idle)
+  const bool couple = quad && tc_couple_has(pl.mode, 256) && workspace && aligned16(workspace) &&
+                      ws_bytes >= couple_ws_bytes(M, N);
   int bn = 0, sub = 1;
   int64_t tiles_n = 0;
   if (quad) {
@@ -536,7 +572,13 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     sig = kSigBiasNormSilu;
   else if (pl.mode == kModeLse && ProgScale::matches(pl.pre, pl.n_pre))
     sig = kSigScaleLse;
-  if (quad)
+  if (couple) {
+    const int slots = couple_slots(M, N);
+    p.gx_data = static_cast<float2*>(workspace);
+    p.gx_flag = reinterpret_cast<unsigned long long*>(static_cast<char*>(workspace) + slots * kCoupleDataBytes);
+    p.gx_epoch = next_epoch();
+    st = cuda_status(tc_couple_launch(pl.mode, bn, sig, ma, mb, mc, p, slots, s));
+  } else if (quad)
     st = cuda_status(tc_dense4_launch(pl.mode, bn, sig, ma, mb, mc, p, s));
   else
     st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, mr, p, sub, grid, s));

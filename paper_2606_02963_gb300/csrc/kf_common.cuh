@@ -74,6 +74,14 @@ struct TcParams {
   int32_t res_op;       // index in pre[] of a bf16 RESIDUAL_ADD staged by coalesced loads, or -1
   int32_t vec_op;       // index in pre[] of a bf16 BIAS / MUL whose vector is loaded ahead, or -1
   int32_t c_tma;        // output tiles leave through TMA stores (dense, bf16, aligned)
+  // GroupNorm on couples of CTA pairs: per-row statistics exchanged through
+  // global memory (workspace) -- [couples][2 slots][2 halves][256 rows] float2,
+  // then [couples][2 slots][2 halves][8 row blocks] uint64 flags tagged with
+  // (epoch << 32 | tile sequence + 1)
+  float2* gx_data;
+  unsigned long long* gx_flag;
+  uint32_t gx_epoch;
+  int32_t gx_couples;
 };
 
 // ---------------------------------------------------------------- loads/stores

@@ -42,6 +42,13 @@ cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUte
 // GroupNorm over 512-column groups on clusters of two CTA pairs (one 256-column
 // half of the group per pair); units = 256-row x 512-column blocks, the grid is
 // sized inside from the number of co-resident clusters.
+// GroupNorm over 512-column groups on couples of CTA pairs (cooperative grid):
+// the same split as the clusters of four, with the statistics exchanged through
+// global memory (p.gx_data / p.gx_flag, room for `max_couples` couples), so all
+// co-resident pairs work.
+bool tc_couple_has(int mode, int bn);
+cudaError_t tc_couple_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
+                             const CUtensorMap& c, const TcParams& p, int max_couples, cudaStream_t s);
 bool tc_dense4_has(int mode, int bn);
 cudaError_t tc_dense4_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
                              const CUtensorMap& c, const TcParams& p, cudaStream_t s);

@@ -221,6 +221,34 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
 // Arrive on an mbarrier of another CTA of the cluster (shared::cluster address).
+// Flag word in global memory shared with CTAs of other clusters (same grid,
+// co-resident by a cooperative launch).
+__device__ __forceinline__ void st_release_gpu_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_acquire_gpu_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ float2 ld_relaxed_gpu_f2(const float2* p) {
+  float2 v;
+  asm volatile("ld.relaxed.gpu.global.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(p) : "memory");
+  return v;
+}
+// Bounded wait until *flag == want (acquire).  Gives up after `limit_ns` of wall
+// time or when `*abort_flag` is raised.
+__device__ __forceinline__ bool flag_wait_gpu(const unsigned long long* flag, unsigned long long want,
+                                              const volatile int* abort_flag, uint64_t limit_ns) {
+  if (ld_acquire_gpu_u64(flag) == want) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    if (ld_acquire_gpu_u64(flag) == want) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
 // Store two floats into (possibly another CTA's) shared memory of the cluster.
 __device__ __forceinline__ void st_cluster_f2(uint32_t cluster_addr, float a, float b) {
   asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(cluster_addr), "f"(a), "f"(b) : "memory");

@@ -82,7 +82,62 @@ cudaError_t launch_quad(const CUtensorMap& a, const CUtensorMap& b, const CUtens
   return cudaLaunchKernelEx(&cfg, kern, a, b, c, none, p, static_cast<int32_t>(1));
 }
 
+// Couples of CTA pairs (clusters of 2) in one cooperative grid: the pairs of a
+// couple wait on each other's statistics, so every CTA must be resident at once,
+// which the cooperative launch guarantees (it fails rather than oversubscribe).
+template <int BN, int STAGES, int MODE, class PRE = Interp, class POST = Interp>
+cudaError_t launch_couple(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p_in,
+                          int max_couples, cudaStream_t s) {
+  using Cfg = TcCfg<BN, STAGES, MODE, false, kClCouple>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClCouple, PRE, POST>;
+  static int max_pairs[64] = {};  // per device; 0 = not yet queried
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeCooperative;
+  attr[1].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (max_pairs[dev] == 0) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    int nc = 0;
+    cfg.gridDim = dim3(2, 1, 1);
+    e = cudaOccupancyMaxActiveClusters(&nc, kern, &cfg);
+    if (e != cudaSuccess) return e;
+    if (nc < 2) return cudaErrorInvalidConfiguration;
+    max_pairs[dev] = nc;
+  }
+  const int couples = std::min(std::min(p_in.total_units, max_pairs[dev] / 2), max_couples);
+  if (couples < 1) return cudaSuccess;
+  TcParams p = p_in;
+  p.gx_couples = couples;
+  cfg.gridDim = dim3(4 * couples, 1, 1);
+  cfg.numAttrs = 2;
+  static const CUtensorMap none = {};
+  return cudaLaunchKernelEx(&cfg, kern, a, b, c, none, p, static_cast<int32_t>(1));
+}
+
 }  // namespace
+
+bool tc_couple_has(int mode, int bn) { return mode == kModeGroupNorm && bn == 256; }
+
+cudaError_t tc_couple_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
+                             const CUtensorMap& c, const TcParams& p, int max_couples, cudaStream_t s) {
+  if (mode != kModeGroupNorm || bn != 256) return cudaErrorInvalidValue;
+  if (sig == kSigBiasNormSilu)
+    return launch_couple<256, 6, kModeGroupNorm, ProgBias, ProgSilu>(a, b, c, p, max_couples, s);
+  return launch_couple<256, 6, kModeGroupNorm>(a, b, c, p, max_couples, s);  // any other chain: interpreter
+}
 
 bool tc_dense4_has(int mode, int bn) { return mode == kModeGroupNorm && bn == 256; }
 

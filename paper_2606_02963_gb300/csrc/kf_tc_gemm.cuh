@@ -54,6 +54,10 @@ __host__ __device__ constexpr int pow2_at_least(int x) {
 constexpr int kClOne = 0;
 constexpr int kClPair = 1;
 constexpr int kClQuad = 2;
+// kClCouple = CTA pairs (clusters of 2) of one cooperative grid taken two at a
+// time: the pairs of a couple hold the two 256-column halves of one 512-column
+// unit and swap per-row statistics through global memory (GroupNorm).
+constexpr int kClCouple = 3;
 
 // Residual tile: dense CTA-pair store kernels whose compiled chain adds a bf16
 // residual stage the whole residual tile in shared memory by TMA (each epilogue
@@ -70,6 +74,7 @@ struct TcCfg {
   static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN");
   static_assert(!(GROUPED && CTA2), "grouped GEMMs use single-CTA tiles");
   static_assert(!kQuad || (MODE == kModeGroupNorm && BN == 256), "quad clusters split 512-column groups");
+  static_assert(CL != kClCouple || (MODE == kModeGroupNorm && BN == 256), "couples split 512-column groups");
   static_assert(!RT || (MODE == kModeStore && !GROUPED && CL == kClPair), "residual tile: dense CTA-pair store");
   static constexpr int kOutN = (MODE == kModeSwiglu) ? BN / 2 : BN;  // output columns of a (sub)tile
   // With CTA pairs each CTA stages its own 128 rows of A and half of the BN rows of B.
@@ -121,6 +126,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CL, RT>;
   constexpr bool CTA2 = Cfg::CTA2;
   constexpr bool QUAD = Cfg::kQuad;
+  constexpr bool COUPLE = CL == kClCouple;
   constexpr bool PRE_IS_BIAS = IsBiasProg<PRE>::value;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -155,8 +161,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint16_t pair_mask = static_cast<uint16_t>(0x3u << (rank & 2u));
   const bool leader = prank == 0;
   constexpr int kUnitShift = QUAD ? 2 : (CTA2 ? 1 : 0);
-  const int32_t unit0 = static_cast<int32_t>(blockIdx.x >> kUnitShift);
-  const int32_t unit_step = static_cast<int32_t>(gridDim.x >> kUnitShift);
+  int32_t unit0 = static_cast<int32_t>(blockIdx.x >> kUnitShift);
+  int32_t unit_step = static_cast<int32_t>(gridDim.x >> kUnitShift);
+  uint32_t chalf = 0;  // couples: which 256-column half of the unit this pair holds
+  if constexpr (COUPLE) {
+    // pair i and pair i + couples form couple i (grid = 4 x couples CTAs)
+    const int32_t pi = static_cast<int32_t>(blockIdx.x >> 1), ncpl = static_cast<int32_t>(gridDim.x >> 2);
+    unit0 = pi % ncpl;
+    unit_step = ncpl;
+    chalf = static_cast<uint32_t>(pi / ncpl);
+  }
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -258,6 +272,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       r.m_end = min(p.M, r.m0 + kBM);
       if constexpr (QUAD)
         r.n0 = r.n_blk * 2 * BN + static_cast<int32_t>(rank >> 1) * BN;  // this pair's 256 columns
+      else if constexpr (COUPLE)
+        r.n0 = r.n_blk * 2 * BN + static_cast<int32_t>(chalf) * BN;
       else
         r.n0 = r.n_blk * Cfg::kOutN * sub_tiles;
     }
@@ -779,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             chan(n, mean, m2, 32.0f, cmean, cq, n, mean, m2);
           }
         };
-        if (QUAD || (gs == BN && sub_tiles == 1)) {
+        if (QUAD || COUPLE || (gs == BN && sub_tiles == 1)) {
           // One accumulator holds this CTA's columns of the group: the whole
           // group (gs = BN), or (quad) one 256-column half of a 512-column group
           // whose other half CTA rank ^ 2 holds for the same rows.  The
@@ -823,6 +839,39 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const float2 r = xs[slot * kBM + row_in_tile];
             if ((rank >> 1) == 0)
+              chan(cn, cm, cq, cn, r.x, r.y, tn, tm, tq);
+            else
+              chan(cn, r.x, r.y, cn, cm, cq, tn, tm, tq);
+          } else if constexpr (COUPLE) {
+            // the same through global memory: half 0 writes (mean, M2) of its rows,
+            // fences, and one lane publishes the warp's 32 rows with a release
+            // store of (epoch, tile + 1) to the rows' flag; the other pair's warps
+            // of the same rows wait for that exact value (acquire), then read.
+            // Slots alternate with the tile as above.
+            const float cn = tn, cm = tm, cq = tq;
+            const size_t slot = static_cast<size_t>(tl & 1);
+            const size_t mine = (static_cast<size_t>(unit0) * 2 + slot) * 2 + chalf;
+            const size_t other = (static_cast<size_t>(unit0) * 2 + slot) * 2 + (chalf ^ 1u);
+            const int32_t row_u = static_cast<int32_t>(prank) * kBM + row_in_tile;  // row within the unit
+            const int fl = static_cast<int>(prank) * 4 + q;                         // the warp's 32 rows
+            const unsigned long long want =
+                (static_cast<unsigned long long>(p.gx_epoch) << 32) | static_cast<uint32_t>(tl + 1);
+            if (h == 0) {
+              p.gx_data[mine * 256 + row_u] = make_float2(cm, cq);
+              __threadfence();
+              __syncwarp();
+              if (lane == 0) st_release_gpu_u64(p.gx_flag + mine * 8 + fl, want);
+            }
+            bool got = flag_wait_gpu(p.gx_flag + other * 8 + fl, want, abort_flag, p.wait_ns);
+            got = __all_sync(0xffffffffu, got);
+            if (!pair_vote(got)) {
+              *abort_flag = 1;
+              if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+              ok = false;
+              break;
+            }
+            const float2 r = ld_relaxed_gpu_f2(p.gx_data + other * 256 + row_u);
+            if (chalf == 0)
               chan(cn, cm, cq, cn, r.x, r.y, tn, tm, tq);
             else
               chan(cn, r.x, r.y, cn, cm, cq, tn, tm, tq);

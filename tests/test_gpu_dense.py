@@ -193,6 +193,33 @@ def test_groupnorm_512_many_units_per_cluster(post):
     _no_device_error()
 
 
+@pytest.mark.parametrize("M,N,groups", [(200, 1024, 2), (1000, 12288, 24)])
+def test_groupnorm_512_without_workspace(M, N, groups):
+    # no workspace: the statistics of a 512-column group are exchanged on chip
+    # by clusters of four; with one (the binding's default) by couples of CTA
+    # pairs through global memory -- both must match the oracle
+    import ctypes
+    inp = kf_workloads.generate("bf16_groupnorm_swish", seed=19, M=M, N=N, K=136)
+    chain = [("bias", {"p0": inp["b"]}),
+             ("groupnorm", {"groups": groups, "eps": 1e-5, "p0": inp["gamma"], "p1": inp["beta"]}),
+             ("silu", {})]
+    X, W = inp["X"].to(DEV), inp["W"].to(DEV)
+    keep = []
+    epi = kf.make_epilogue(chain_to(chain, DEV), keep)
+    L = kf.lib()
+    assert L.kf_fused_gemm_workspace(M, N, 136, ctypes.byref(epi)) > 0
+    Y = torch.empty(M, N, dtype=torch.bfloat16, device=DEV)
+    st = L.kf_fused_gemm(X.data_ptr(), kf.KF_BF16, 136, W.data_ptr(), kf.KF_BF16, 136, Y.data_ptr(), kf.KF_BF16, N,
+                         M, N, 136, ctypes.byref(epi), None, 0, None)
+    assert st == kf.KF_OK, kf.status_string(st)
+    torch.cuda.synchronize()
+    ref = oracle.fused_gemm(inp["X"], inp["W"], chain)
+    check_bf16(Y, ref, "gn 512, clusters of four")
+    Y2 = kf.fused_gemm(X, W, chain_to(chain, DEV))
+    check_bf16(Y2, ref, "gn 512, couples")
+    _no_device_error()
+
+
 def test_groupnorm_no_affine_unit_moments():
     inp = kf_workloads.generate("bf16_groupnorm_swish", seed=9, M=130, N=1024, K=64, dist="unscaled")
     chain = [("groupnorm", {"groups": 2, "eps": 1e-5})]
