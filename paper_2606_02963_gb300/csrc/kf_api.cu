@@ -279,11 +279,30 @@ int pick_dense_bn(int mode, int64_t M, int64_t N, int nsm, bool cta2) {
   return best;
 }
 
-// Output-column tile for the grouped variants: the widest compiled tile that
-// divides N, else the one wasting the fewest columns.
-int pick_grouped_outn(int mode, int64_t N) {
+// Output-column tile for the grouped variants.  Decode-like problems (at most
+// one 128-row tile per group on average) stream each group's weights once and
+// are bound by how evenly the tiles fall on the SMs: take the width with the
+// fewest tile-widths of weights on the busiest SM (+ a small fixed cost per
+// tile).  Otherwise the widest compiled tile that divides N, else the one
+// wasting the fewest columns.
+int pick_grouped_outn(int mode, int64_t N, int64_t rows_total, int32_t G, int nsm) {
   static const int cand[] = {256, 192, 128};
   int best = 0;
+  if (G > 0 && rows_total <= static_cast<int64_t>(G) * kBM && nsm > 0) {
+    const int64_t row_tiles = std::min<int64_t>(G, rows_total);  // one tile per touched group
+    int64_t best_cost = INT64_MAX;
+    for (int bn : cand) {
+      if (!tc_grouped_has(mode, bn)) continue;
+      const int outn = mode == kModeSwiglu ? bn / 2 : bn;
+      const int64_t units = row_tiles * ((N + outn - 1) / outn);
+      const int64_t cost = ((units + nsm - 1) / nsm) * (bn + 16);
+      if (cost < best_cost) {
+        best_cost = cost;
+        best = bn;
+      }
+    }
+    return best;
+  }
   int64_t best_waste = INT64_MAX;
   for (int bn : cand) {
     if (!tc_grouped_has(mode, bn)) continue;
@@ -358,16 +377,20 @@ size_t grouped_ws_bytes(int64_t rows_total, int64_t K, bool gathered) {
   return gathered ? align_up(static_cast<size_t>(rows_total) * static_cast<size_t>(K) * 2, 256) : 0;
 }
 
-kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cudaStream_t s, const DevInfo& di) {
+// `pdl`: the previous kernel in the stream is one of this library's (MoE chain),
+// so the launches here may be programmatic dependents of it.
+kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cudaStream_t s, const DevInfo& di,
+                       bool pdl) {
   const void* A = g.A;
   int64_t lda = g.lda;
   if (g.a_row_index) {
-    kf_status st = cuda_status(gather_rows_launch(g.A, g.lda, g.a_rows, g.a_row_index, g.rows_total, g.K, ws, di.err, s));
+    kf_status st =
+        cuda_status(gather_rows_launch(g.A, g.lda, g.a_rows, g.a_row_index, g.rows_total, g.K, ws, di.err, s, pdl));
     if (st != KF_OK) return st;
     A = ws;
     lda = g.K;
   }
-  const int bn = pick_grouped_outn(pl.mode, g.N);
+  const int bn = pick_grouped_outn(pl.mode, g.N, g.rows_total, g.G, di.nsm);
   if (bn == 0) return KF_ERR_UNSUPPORTED;
   const int outn = pl.mode == kModeSwiglu ? bn / 2 : bn;
   const int64_t nb = pl.mode == kModeSwiglu ? 2 * g.N : g.N;
@@ -399,7 +422,8 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
   CUtensorMap mc;  // grouped outputs are masked per group: plain stores, no TMA map
   std::memset(&mc, 0, sizeof(mc));
-  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, mc, p, grid, s));
+  // after the gather (when there is one) the GEMM follows a library kernel
+  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, mc, p, grid, s, pdl || g.a_row_index != nullptr));
 }
 
 }  // namespace
@@ -592,7 +616,7 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   cp.out_dtype = yt;
   cp.n_post = pl.n_post;
   for (int i = 0; i < pl.n_post; ++i) cp.post[i] = pl.post[i];
-  return cuda_status(lse_combine_launch(cp, s));
+  return cuda_status(lse_combine_launch(cp, s, true));
 }
 
 kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int32_t* topk_ids, float* topk_w,
@@ -605,7 +629,7 @@ kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int
   kf_status st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, topk_ids, topk_w, s));
   if (st != KF_OK) return st;
   return cuda_status(route_sort_launch(topk_ids, topk_w, static_cast<int32_t>(T), E, k, offsets, sorted_token,
-                                       sorted_w, nullptr, s));
+                                       sorted_w, nullptr, s, true));
 }
 
 size_t kf_grouped_gemm_workspace(int64_t rows_total, int64_t N, int64_t K, int32_t G, int32_t gathered,
@@ -647,7 +671,7 @@ kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows
   if (st != KF_OK) return st;
   GroupedArgs g{A, lda, a_row_index ? a_rows : rows_total, a_row_index, B, ldb,
                 G > 1 ? b_group_stride : nb * ldb, offsets, G, rows_total, N, K, C, ct, ldc};
-  return grouped_core(g, pl, workspace, static_cast<cudaStream_t>(stream), di);
+  return grouped_core(g, pl, workspace, static_cast<cudaStream_t>(stream), di, false);
 }
 
 // Workspace layout of kf_moe_ffn (each region 256-byte aligned):
@@ -729,9 +753,12 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
   const int64_t P = T * k;
 
   int32_t* pos = det ? reinterpret_cast<int32_t*>(ws + L.pos) : nullptr;
+  // the fp32 scatter target is cleared first, so that the kernels of the chain
+  // below follow one another directly (each a programmatic dependent of the last)
+  if (!det && cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
   st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, ids, w, s));
   if (st != KF_OK) return st;
-  st = cuda_status(route_sort_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos, s));
+  st = cuda_status(route_sort_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos, s, true));
   if (st != KF_OK) return st;
   // gate/up: h = silu(Xg W_gate[e]^T) * (Xg W_up[e]^T), rows gathered by token
   {
@@ -742,7 +769,7 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
     st = plan_chain(&epi, I, true, &pl);
     if (st != KF_OK) return st;
     GroupedArgs g{X, H, T, stok, W_gu, H, 2 * I * H, off, E, P, I, H, h, KF_BF16, I};
-    st = grouped_core(g, pl, xg, s, di);
+    st = grouped_core(g, pl, xg, s, di, true);
     if (st != KF_OK) return st;
   }
   if (det) {
@@ -757,13 +784,12 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
     if (st != KF_OK) return st;
     float* yp = reinterpret_cast<float*>(ws + L.yp);
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yp, KF_F32, H};
-    st = grouped_core(g, pl, nullptr, s, di);
+    st = grouped_core(g, pl, nullptr, s, di, true);
     if (st != KF_OK) return st;
-    st = cuda_status(moe_finalize_launch(yp, pos, T, k, H, Y, s));
+    st = cuda_status(moe_finalize_launch(yp, pos, T, k, H, Y, s, true));
     if (st != KF_OK) return st;
   } else {
     // down: Yacc[token] += w * (h W_down[e]^T), then bf16
-    if (cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
     kf_epilogue_op op{};
     op.kind = KF_OP_ROW_SCALE_SCATTER_ADD;
     op.p0 = sw;
@@ -775,9 +801,9 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
     st = plan_chain(&epi, H, true, &pl);
     if (st != KF_OK) return st;
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yacc, KF_F32, H};
-    st = grouped_core(g, pl, nullptr, s, di);
+    st = grouped_core(g, pl, nullptr, s, di, true);
     if (st != KF_OK) return st;
-    st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s));
+    st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s, true));
     if (st != KF_OK) return st;
   }
   if (topk_ids_out &&

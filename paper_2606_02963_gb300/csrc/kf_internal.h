@@ -4,9 +4,31 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <utility>
+
 #include "kf_common.cuh"
 
 namespace kf {
+
+// Launch `kern` on `s`; with `pdl` as a programmatic dependent of the previous
+// kernel in the stream (one of this library's): it may be scheduled while that
+// kernel finishes and waits for it with griddepcontrol.wait before reading its
+// results.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 // Compiled chain programs selectable by signature id (0 = interpreter).
 using ProgGeluChain = Prog<KF_OP_BIAS, KF_OP_GELU_TANH, KF_OP_SCALE, KF_OP_RESIDUAL_ADD>;  // bias, GELU, scale, +R
@@ -38,7 +60,7 @@ cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, co
                              const CUtensorMap& c, const CUtensorMap& r, const TcParams& p, int sub_tiles, int grid,
                              cudaStream_t s);
 cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
-                              const TcParams& p, int grid, cudaStream_t s);
+                              const TcParams& p, int grid, cudaStream_t s, bool pdl);
 // GroupNorm over 512-column groups on clusters of two CTA pairs (one 256-column
 // half of the group per pair); units = 256-row x 512-column blocks, the grid is
 // sized inside from the number of co-resident clusters.
@@ -74,17 +96,17 @@ struct LseCombineParams {
   int32_t n_post;
   DevOp post[kMaxOps];
 };
-cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s);
+cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s, bool pdl);
 
 cudaError_t route_topk_launch(const float* logits, int32_t T, int32_t E, int32_t k, int32_t* ids, float* w,
                               cudaStream_t s);
 cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
                               int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
-                              cudaStream_t s);
+                              cudaStream_t s, bool pdl);
 cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_t T, int32_t k, int64_t H, void* Y,
-                                cudaStream_t s);
+                                cudaStream_t s, bool pdl);
 cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
-                               int64_t K, void* out, uint32_t* err, cudaStream_t s);
-cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s);
+                               int64_t K, void* out, uint32_t* err, cudaStream_t s, bool pdl);
+cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s, bool pdl);
 
 }  // namespace kf

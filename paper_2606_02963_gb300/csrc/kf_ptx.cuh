@@ -221,6 +221,14 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
 // Arrive on an mbarrier of another CTA of the cluster (shared::cluster address).
+// Programmatic dependent launch: wait until the grids this one depends on have
+// completed and their writes are visible (no-op without such a dependency), and
+// let the next grid in the stream be scheduled now.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Flag word in global memory shared with CTAs of other clusters (same grid,
 // co-resident by a cooperative launch).
 __device__ __forceinline__ void st_release_gpu_u64(unsigned long long* p, unsigned long long v) {

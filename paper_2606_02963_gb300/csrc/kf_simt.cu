@@ -76,6 +76,8 @@ cudaError_t simt_gemm_f32_launch(const SimtParams& p, cudaStream_t s) {
 // ------------------------------------------------------- row log-sum-exp combine
 // (m, s) (+) (m', s') = (M, s e^{m-M} + s' e^{m'-M}),  out = M + log S.
 __global__ void lse_combine_kernel(const __grid_constant__ LseCombineParams p) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   const int warps = blockDim.x >> 5;
   const int row = blockIdx.x * warps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -110,10 +112,9 @@ __global__ void lse_combine_kernel(const __grid_constant__ LseCombineParams p) {
   }
 }
 
-cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s) {
+cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s, bool pdl) {
   const int warps = 8;
-  lse_combine_kernel<<<(p.M + warps - 1) / warps, warps * 32, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(lse_combine_kernel, dim3((p.M + warps - 1) / warps), dim3(warps * 32), 0, s, pdl, p);
 }
 
 // ------------------------------------------------------------------- routing
@@ -122,6 +123,8 @@ cudaError_t lse_combine_launch(const LseCombineParams& p, cudaStream_t s) {
 constexpr int kMaxExperts = 256;
 __global__ void route_topk_kernel(const float* __restrict__ logits, int32_t T, int32_t E, int32_t k,
                                   int32_t* __restrict__ ids, float* __restrict__ w) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   const int warps = blockDim.x >> 5;
   const int t = blockIdx.x * warps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -199,6 +202,8 @@ __global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32
                                                                      int32_t E, int32_t k, int32_t* offsets,
                                                                      int32_t* sorted_token, float* sorted_w,
                                                                      int32_t* pair_pos) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   extern __shared__ int32_t cnt[];  // [kSortWarps][E]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kSortWarps * E; i += blockDim.x) cnt[i] = 0;
@@ -274,17 +279,19 @@ __global__ void __launch_bounds__(kSortWarps * 32) route_sort_kernel(const int32
 
 cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
                               int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
-                              cudaStream_t s) {
+                              cudaStream_t s, bool pdl) {
   const int32_t P = T * k;
   const size_t smem = sizeof(int32_t) * kSortWarps * E;
-  route_sort_kernel<<<1, kSortWarps * 32, smem, s>>>(ids, w, P, E, k, offsets, sorted_token, sorted_w, pair_pos);
-  return cudaGetLastError();
+  return launch_k(route_sort_kernel, dim3(1), dim3(kSortWarps * 32), smem, s, pdl, ids, w, P, E, k, offsets,
+                  sorted_token, sorted_w, pair_pos);
 }
 
 // ------------------------------------------------ deterministic MoE finalize
 // Y[t, :] = bf16( sum_{j = 0..k-1} Yp[pair_pos[t*k + j], :] ), slot order fixed.
 __global__ void moe_finalize_kernel(const float4* __restrict__ Yp, const int32_t* __restrict__ pair_pos, int64_t T,
                                     int32_t k, int64_t h4, uint2* __restrict__ Y) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   const int64_t total = T * h4;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -305,13 +312,12 @@ __global__ void moe_finalize_kernel(const float4* __restrict__ Yp, const int32_t
 }
 
 cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_t T, int32_t k, int64_t H, void* Y,
-                                cudaStream_t s) {
+                                cudaStream_t s, bool pdl) {
   if (T == 0) return cudaSuccess;
   const int64_t h4 = H / 4, total = T * h4;
   const int blocks = static_cast<int>(std::min<int64_t>((total + 255) / 256, 148 * 8));
-  moe_finalize_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const float4*>(Yp), pair_pos, T, k, h4,
-                                             reinterpret_cast<uint2*>(Y));
-  return cudaGetLastError();
+  return launch_k(moe_finalize_kernel, dim3(blocks), dim3(256), 0, s, pdl, reinterpret_cast<const float4*>(Yp),
+                  pair_pos, T, k, h4, reinterpret_cast<uint2*>(Y));
 }
 
 // ----------------------------------------------------------------- row gather
@@ -320,6 +326,8 @@ cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_
 __global__ void gather_rows_kernel(const uint4* __restrict__ A, int64_t lda_v, int64_t a_rows,
                                    const int32_t* __restrict__ idx, int64_t rows, int64_t kv,
                                    uint4* __restrict__ out, uint32_t* err) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   const int64_t total = rows * kv;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -335,17 +343,18 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ A, int64_t lda_v, i
 }
 
 cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
-                               int64_t K, void* out, uint32_t* err, cudaStream_t s) {
+                               int64_t K, void* out, uint32_t* err, cudaStream_t s, bool pdl) {
   if (rows == 0) return cudaSuccess;
   const int64_t kv = K / 8, total = rows * kv;
   int blocks = static_cast<int>(std::min<int64_t>((total + 255) / 256, 148 * 16));
-  gather_rows_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4*>(A), lda / 8, a_rows, idx, rows, kv,
-                                            reinterpret_cast<uint4*>(out), err);
-  return cudaGetLastError();
+  return launch_k(gather_rows_kernel, dim3(blocks), dim3(256), 0, s, pdl, reinterpret_cast<const uint4*>(A), lda / 8,
+                  a_rows, idx, rows, kv, reinterpret_cast<uint4*>(out), err);
 }
 
 // ------------------------------------------------------------ fp32 -> bf16
 __global__ void cvt_f32_bf16_kernel(const float4* __restrict__ in, uint2* __restrict__ out, int64_t n4) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n4;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const float4 f = in[i];
@@ -356,19 +365,25 @@ __global__ void cvt_f32_bf16_kernel(const float4* __restrict__ in, uint2* __rest
   }
 }
 __global__ void cvt_f32_bf16_tail_kernel(const float* in, __nv_bfloat16* out, int64_t beg, int64_t n) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
   const int64_t i = beg + threadIdx.x;
   if (i < n) out[i] = __float2bfloat16_rn(in[i]);
 }
 
-cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s) {
+cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s, bool pdl) {
   const int64_t n4 = n / 4;
   if (n4 > 0) {
     int blocks = static_cast<int>(std::min<int64_t>((n4 + 255) / 256, 148 * 8));
-    cvt_f32_bf16_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const float4*>(in), reinterpret_cast<uint2*>(out),
-                                               n4);
+    cudaError_t e = launch_k(cvt_f32_bf16_kernel, dim3(blocks), dim3(256), 0, s, pdl,
+                             reinterpret_cast<const float4*>(in), reinterpret_cast<uint2*>(out), n4);
+    if (e != cudaSuccess) return e;
+    pdl = true;  // the tail follows the main kernel
   }
-  if (n % 4) cvt_f32_bf16_tail_kernel<<<1, 4, 0, s>>>(in, reinterpret_cast<__nv_bfloat16*>(out), n4 * 4, n);
-  return cudaGetLastError();
+  if (n % 4)
+    return launch_k(cvt_f32_bf16_tail_kernel, dim3(1), dim3(4), 0, s, pdl, in,
+                    reinterpret_cast<__nv_bfloat16*>(out), n4 * 4, n);
+  return cudaSuccess;
 }
 
 }  // namespace kf

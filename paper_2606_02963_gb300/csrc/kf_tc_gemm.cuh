@@ -209,6 +209,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_relinquish();
     }
   }
+  // Everything above is independent of other kernels' results; when this grid
+  // follows another of this library's kernels as a programmatic dependent (the
+  // MoE chain), wait for it here, before the group table, operands or epilogue
+  // inputs are read.  Without such a dependency the wait returns at once.
+  griddep_wait();
+  griddep_launch_dependents();
   if constexpr (GROUPED) {
     if (threadIdx.x == 64) {
       // Group table: validate the device-resident offsets and count work units

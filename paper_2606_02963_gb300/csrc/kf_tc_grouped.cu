@@ -7,7 +7,8 @@ namespace kf {
 namespace {
 
 template <int BN, int STAGES, int MODE>
-cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int grid, cudaStream_t s) {
+cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int grid, cudaStream_t s,
+                       bool pdl) {
   using Cfg = TcCfg<BN, STAGES, MODE, true, kClOne>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, kClOne>;
   static bool configured[64] = {};  // the attribute is per device
@@ -20,8 +21,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     configured[dev] = true;
   }
   static const CUtensorMap none = {};  // grouped variants stage no residual tile
-  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, none, p, 1);
-  return cudaGetLastError();
+  return launch_k(kern, dim3(grid), dim3(kThreads), Cfg::kSmemBytes, s, pdl, a, b, c, none, p, static_cast<int32_t>(1));
 }
 
 }  // namespace
@@ -46,9 +46,9 @@ bool tc_grouped_has(int mode, int bn) {
 }
 
 cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p,
-                              int grid, cudaStream_t s) {
+                              int grid, cudaStream_t s, bool pdl) {
 #define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, p, grid, s);
+  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, p, grid, s, pdl);
   KF_GROUPED_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;
