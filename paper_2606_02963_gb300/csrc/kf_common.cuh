@@ -372,6 +372,27 @@ __device__ __forceinline__ void tanh2_fast(float a, float b, float& ta, float& t
   ta = __low2float(h2);
   tb = __high2float(h2);
 }
+// GELU_tanh of two values in packed half precision, for results stored as
+// bf16: g = h + h tanh(x (c0 + c1 x^2)), h = x / 2, c0 = sqrt(2/pi),
+// c1 = 0.044715 c0 -- each step one f16x2 instruction.  f16 keeps 11
+// significant bits (bf16 keeps 8).  Past |x| ~ 150 the tanh argument overflows
+// to +-inf and tanh saturates at +-1, which is the function's limit.
+__device__ __forceinline__ void gelu2_f16(float& a, float& b) {
+  uint32_t x, g;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(x) : "f"(b), "f"(a));
+  asm("{\n\t.reg .b32 u, p, q, t, h;\n\t"
+      "mul.rn.f16x2 u, %1, %1;\n\t"
+      "fma.rn.f16x2 p, u, %2, %3;\n\t"
+      "mul.rn.f16x2 q, %1, p;\n\t"
+      "tanh.approx.f16x2 t, q;\n\t"
+      "mul.rn.f16x2 h, %1, %4;\n\t"
+      "fma.rn.f16x2 %0, h, t, h;\n\t}"
+      : "=r"(g)
+      : "r"(x), "r"(0x28912891u), "r"(0x3a623a62u), "r"(0x38003800u));  // c1, c0, 1/2 (f16 pairs)
+  const __half2 h2 = *reinterpret_cast<const __half2*>(&g);
+  a = __low2float(h2);
+  b = __high2float(h2);
+}
 __device__ __forceinline__ float f_gelu_tanh_fast(float x) {
   const float c = 0.7978845608028654f;
   const float hx = 0.5f * x;
@@ -461,16 +482,8 @@ __device__ __forceinline__ void apply_chain32(const DevOp* ops, int n, float (&v
       } break;
       case KF_OP_GELU_TANH: {
         if (FAST) {
-          const float c = 0.7978845608028654f;  // sqrt(2/pi)
 #pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            float t0, t1;
-            tanh2_fast(c * fmaf(0.044715f * v[j], v[j] * v[j], v[j]),
-                       c * fmaf(0.044715f * v[j + 1], v[j + 1] * v[j + 1], v[j + 1]), t0, t1);
-            const float h0 = 0.5f * v[j], h1 = 0.5f * v[j + 1];
-            v[j] = fmaf(h0, t0, h0);
-            v[j + 1] = fmaf(h1, t1, h1);
-          }
+          for (int j = 0; j < 32; j += 2) gelu2_f16(v[j], v[j + 1]);
         } else {
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = f_gelu_tanh(v[j]);
@@ -561,16 +574,8 @@ __device__ __forceinline__ void prog_op(const DevOp& op, float (&v)[32], int64_t
     for (int j = 0; j < 32; ++j) v[j] *= op.scalar;
   } else if constexpr (KIND == KF_OP_GELU_TANH) {
     if constexpr (FAST) {
-      const float c = 0.7978845608028654f;
 #pragma unroll
-      for (int j = 0; j < 32; j += 2) {
-        float t0, t1;
-        tanh2_fast(c * fmaf(0.044715f * v[j], v[j] * v[j], v[j]),
-                   c * fmaf(0.044715f * v[j + 1], v[j + 1] * v[j + 1], v[j + 1]), t0, t1);
-        const float h0 = 0.5f * v[j], h1 = 0.5f * v[j + 1];
-        v[j] = fmaf(h0, t0, h0);
-        v[j + 1] = fmaf(h1, t1, h1);
-      }
+      for (int j = 0; j < 32; j += 2) gelu2_f16(v[j], v[j + 1]);
     } else {
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = f_gelu_tanh(v[j]);
