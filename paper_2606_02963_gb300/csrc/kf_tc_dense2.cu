@@ -168,13 +168,13 @@ bool tc_dense2_has(int mode, int bn) {
 }
 
 // Chain-program variants: (mode, BN, stages, signature, PRE, POST)
-// (the residual-tile variants give BN x 256 B of shared memory to the residual
-// tile, so their rings are one or two stages shorter)
+// (the residual-tile variants keep the residual in two ring slots and need
+// only small per-warp buffers, so their rings are as deep as shared memory allows)
 #define KF_DENSE2_PROG_VARIANTS(X)                                              \
-  X(kModeStore, 128, 7, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
-  X(kModeStore, 192, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
-  X(kModeStore, 224, 5, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
-  X(kModeStore, 256, 4, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 128, 9, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 192, 7, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 224, 7, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
+  X(kModeStore, 256, 6, kSigBiasGeluScaleRes, ProgGeluChain, Interp)            \
   X(kModeGroupNorm, 256, 6, kSigBiasNormSilu, ProgBias, ProgSilu)               \
   X(kModeLse, 224, 6, kSigScaleLse, ProgScale, Interp)                          \
   X(kModeLse, 256, 6, kSigScaleLse, ProgScale, Interp)

@@ -60,10 +60,11 @@ constexpr int kClQuad = 2;
 constexpr int kClCouple = 3;
 
 // Residual tile: dense CTA-pair store kernels whose compiled chain adds a bf16
-// residual stage the whole residual tile in shared memory by TMA (each epilogue
-// warp loads its own rows x chunks before it waits for the accumulator), add it
-// from there, write the bf16 result in place and send each 32 x 32 block out
-// with one TMA store.
+// residual stage the unit's residual tile in shared memory by TMA, in the two
+// ring slots that follow the unit's last k-block (the producer loads them, the
+// MMA skips them), add it from there, write the bf16 result in place and send
+// each 32 x 32 block out with one TMA store; the last epilogue warp to finish
+// frees the two slots.
 template <int MODE, bool GROUPED, int CL, class PRE>
 constexpr bool kResTileFor = MODE == kModeStore && !GROUPED && CL == kClPair && PRE::kHasRes;
 
@@ -92,8 +93,13 @@ struct TcCfg {
   // transposition, which must not reuse a buffer a TMA store may still read
   // (residual tile: 256 B per warp, the bias of its chunks)
   static constexpr int kWarpStaging = RT ? 256 : ((MODE == kModeStore) ? 3072 : 2048);
-  // residual tile: BN / 32 chunks x 128 rows x 64 B (64-byte swizzle), 2 KB per warp and chunk
-  static constexpr int kResTileBytes = RT ? BN * 256 : 0;
+  // residual tile: BN / 32 chunks x 4 row blocks of 32 x 32 bf16 (2 KB, 64-byte
+  // swizzle), placed in the A then B regions of two ring slots
+  static constexpr int kResTileBytes = 0;
+  static constexpr int kResBlocksA = kABytes / 2048;
+  static constexpr int kResBlocksPerSlot = kABytes / 2048 + kBBytes / 2048;
+  static_assert(!RT || 2 * kResBlocksPerSlot >= (BN / 32) * 4, "residual tile fits two ring slots");
+  static_assert(!RT || STAGES >= 3, "residual tile needs two slots beside an operand slot");
   static constexpr int kStagingBytes = kEpiWarps * kWarpStaging;
   // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
   static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiWarps * 3 * 4 * 32 * 4 : 0;
@@ -132,8 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* smB = sm;                                // B stages first: any over-read stays inside the CTA
   uint8_t* smA = sm + STAGES * Cfg::kBBytes;
-  uint8_t* rtile = sm + STAGES * Cfg::kStageBytes;             // residual tile (RT)
-  uint8_t* staging = rtile + Cfg::kResTileBytes;                // epilogue tile buffers
+  uint8_t* staging = sm + STAGES * Cfg::kStageBytes;           // epilogue tile buffers
   float* gn_cache = reinterpret_cast<float*>(staging + Cfg::kStagingBytes);
   uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::kStagingBytes + Cfg::kGnCacheBytes);
   uint64_t* full = bars;
@@ -148,6 +153,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   int32_t* total_s = reinterpret_cast<int32_t*>(misc + 2);
   volatile int* zero_flag = reinterpret_cast<volatile int*>(misc + 3);
+  // residual tile: epilogue warps done with the unit's slots, one counter per
+  // accumulator parity (a warp runs at most one unit ahead of the slowest: the
+  // unit after next reuses this unit's accumulator, freed only after this count)
+  int* rdone = reinterpret_cast<int*>(misc + 4);
   int32_t* off_s = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(misc) + Cfg::kMiscBytes);
   int32_t* ustart_s = off_s + (kMaxGroups + 1);
 
@@ -190,6 +199,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int w = 0; w < kEpiWarps; ++w) mbar_init(&rbar[w], 1);
     *abort_flag = 0;
     *zero_flag = 0;
+    rdone[0] = 0;
+    rdone[1] = 0;
     *total_s = GROUPED ? 0 : p.total_units;
     fence_mbarrier_init();
     fence_proxy_async_smem();
@@ -250,6 +261,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const int32_t total = *total_s;
 
+  // residual block (chunk c, row block q) of a unit whose residual sits in ring
+  // slots s0, s1
+  auto res_block = [&](int s0, int s1, int c, int qq) -> uint8_t* {
+    const int bi = c * 4 + qq;
+    const int sl = bi < Cfg::kResBlocksPerSlot ? s0 : s1;
+    const int j = bi % Cfg::kResBlocksPerSlot;
+    return j < Cfg::kResBlocksA ? smA + sl * kABytes + j * 2048 : smB + sl * Cfg::kBBytes + (j - Cfg::kResBlocksA) * 2048;
+  };
+
   auto decode = [&](int32_t u) -> UnitInfo {
     UnitInfo r;
     if constexpr (GROUPED) {
@@ -289,7 +309,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      int32_t it = 0;
+      int32_t it = 0, rt_units = 0;
       bool ok = true;
       for (int32_t u = unit0; ok && u < total; u += unit_step) {
         const UnitInfo ui = decode(u);
@@ -324,9 +344,44 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             ++it;
           }
+          if constexpr (RT) {
+            // the unit's residual tile into the next two slots; each epilogue
+            // warp's blocks complete on its own barrier
+            int sr[2] = {0, 0};
+            for (int r = 0; ok && r < 2; ++r) {
+              const int st = it % STAGES;
+              const uint32_t ph = (it / STAGES) & 1;
+              if (!mbar_wait(&empty[st], ph ^ 1, abort_flag, p.wait_ns)) {
+                *abort_flag = 1;
+                atomicOr(p.err, kErrWaitProducer);
+                ok = false;
+                break;
+              }
+              if (leader) mbar_arrive(&full[st]);  // one phase per slot use, as for operand slots
+              sr[r] = st;
+              ++it;
+            }
+            if (!ok) break;
+            for (int w = 0; w < kEpiWarps; ++w) {
+              uint32_t bytes = 0;
+              for (int c = w >> 2; c < Cfg::kOutN / 32; c += 2)
+                if (ui.n0 + c * 32 < p.N) bytes += 2048;
+              mbar_arrive_expect_tx(&rbar[w], bytes);
+            }
+            for (int c = 0; c < Cfg::kOutN / 32 && ui.n0 + c * 32 < p.N; ++c)
+              for (int qq = 0; qq < 4; ++qq)
+                tma_load_2d(res_block(sr[0], sr[1], c, qq), &tmR, &rbar[(c & 1) * 4 + ((qq + 2) & 3)], ui.n0 + c * 32,
+                            ui.m0 + qq * 32);
+            ++rt_units;
+          }
         }
       }
       if (!ok) {
+        if constexpr (RT) {
+          // residual copies still in flight land before the CTA exits
+          if (rt_units > 0)
+            for (int w = 0; w < kEpiWarps; ++w) mbar_wait(&rbar[w], (rt_units - 1) & 1, zero_flag, p.drain_ns);
+        }
         if (!CTA2 || leader) {
           // wait (bounded) for the copies still in flight before the CTA exits
           for (int32_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
@@ -382,6 +437,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_commit_pair_mc(&accf[acc], pair_mask);
           else
             tc_commit(&accf[acc]);
+          if constexpr (RT) it += 2;  // the unit's residual slots are the epilogue's
           ++tl;
         }
       }
@@ -419,12 +475,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool c_tma = p.c_tma != 0;
     int32_t tl = 0;
     bool ok = true;
-    // residual tile state: the warp's bias cache, the bias vector, whether a
-    // residual load is in flight and the phase of its barrier
+    // residual tile state: the warp's bias cache, the bias vector and the phase
+    // of the warp's residual barrier
     uint8_t* bcache = staging + ew * Cfg::kWarpStaging;
     const __nv_bfloat16* rt_bias_ptr =
         RT ? reinterpret_cast<const __nv_bfloat16*>(p.pre[p.vec_op < 0 ? 0 : p.vec_op].p0) : nullptr;
-    bool rt_pending = false;
     uint32_t rt_phase = 0;
 
     auto wait_acc = [&](int32_t t) -> bool {
@@ -501,8 +556,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (vec_staged) vec32_issue(p.pre[p.vec_op].p0, col0, bq);
         };
-        // residual tile: this warp's chunks of the residual (TMA) and of the bias
-        // (one 16-byte unit per lane 0..15) are requested before the wait
+        // residual tile: this warp's chunks of the bias (one 16-byte unit per lane
+        // 0..15) are requested before the wait; the producer loads the residual
         uint4 rt_bias = make_uint4(0u, 0u, 0u, 0u);
         if constexpr (RT) {
           if (lane < 16) {
@@ -510,16 +565,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int32_t col = ui.n0 + c * 32 + (lane & 3) * 8;
             if (c < Cfg::kOutN / 32 && col + 8 <= p.N) rt_bias = ldg_v4_pinned(rt_bias_ptr + col);
           }
-          if (lane == 0) {
-            bulk_wait_group_read<0>();  // this warp's stores of the previous tile have read its blocks
-            uint32_t bytes = 0;
-            for (int c = h; c < Cfg::kOutN / 32; c += 2)
-              if (ui.n0 + c * 32 < p.N) bytes += 2048;
-            mbar_arrive_expect_tx(&rbar[ew], bytes);
-            for (int c = h; c < Cfg::kOutN / 32; c += 2)
-              if (ui.n0 + c * 32 < p.N) tma_load_2d(rtile + c * 8192 + q * 2048, &tmR, &rbar[ew], ui.n0 + c * 32, wrow0);
-          }
-          rt_pending = true;
         } else if constexpr (MODE == kModeStore) {
           issue_chunk(h);
         }
@@ -534,10 +579,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
           }
-          rt_pending = false;
           rt_phase ^= 1u;
           __syncwarp();
         }
+        // ring slots holding this unit's residual tile (after its k-blocks)
+        const int32_t rt_pos = tl * (p.num_kb + 2) + p.num_kb;
+        const int rt_s0 = rt_pos % STAGES, rt_s1 = (rt_pos + 1) % STAGES;
         const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
         float rs = 0.0f;
         int32_t dst = 0;
@@ -561,7 +608,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if constexpr (RT) {
             // residual from the tile (64-byte swizzle, row = lane), bias from the
             // warp's cache; the result overwrites the residual in place
-            uint8_t* blk = rtile + c * 8192 + q * 2048;
+            uint8_t* blk = res_block(rt_s0, rt_s1, c, q);
             const uint4* bc = reinterpret_cast<const uint4*>(bcache + ((c - h) >> 1) * 64);
             Staged32 sg;
             sg.use_res = true;
@@ -648,6 +695,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                               wrows);
           } else {
             if (row_ok) st32(p.C, p.c_dtype, static_cast<int64_t>(grow) * p.ldc + col0, nvalid, p.c_vec_ok != 0, v);
+          }
+        }
+        if constexpr (RT) {
+          // this warp's stores have read its blocks: the last warp to get here
+          // frees the unit's two residual slots
+          if (lane == 0) {
+            bulk_wait_group_read<0>();
+            __threadfence_block();
+            if (atomicAdd(&rdone[tl & 1], 1) == kEpiWarps - 1) {
+              rdone[tl & 1] = 0;
+              __threadfence_block();
+              mbar_arrive(&empty[rt_s0]);
+              mbar_arrive(&empty[rt_s1]);
+            }
           }
         }
         release_acc(tl);
@@ -949,10 +1010,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           tl += sub_tiles;
         }
       }
-    }
-    // a residual load still in flight after an abort lands before the CTA exits
-    if constexpr (RT) {
-      if (rt_pending && lane == 0) mbar_wait(&rbar[ew], rt_phase, zero_flag, p.drain_ns);
     }
   }
 
