@@ -22,7 +22,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  kern<<<grid, kThreads, Cfg::kSmemBytes, s>>>(a, b, c, r, p, sub);
+  kern<<<grid, Cfg::kThr, Cfg::kSmemBytes, s>>>(a, b, c, r, p, sub);
   return cudaGetLastError();
 }
 

@@ -39,8 +39,8 @@ struct IsBiasProg<Prog<KF_OP_BIAS>> {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;
-constexpr int kEpiWarps = 8;
-constexpr int kThreads = 64 + 32 * kEpiWarps;  // TMA warp, MMA warp, 8 epilogue warps
+constexpr int kEpiWarps = 8;  // epilogue warps of the variants without a residual tile
+constexpr int kThreads = 64 + 32 * kEpiWarps;  // TMA warp, MMA warp, epilogue warps
 constexpr int kABytes = kBM * kBK * 2;
 
 __host__ __device__ constexpr int pow2_at_least(int x) {
@@ -67,10 +67,18 @@ constexpr int kClCouple = 3;
 // frees the two slots.
 template <int MODE, bool GROUPED, int CL, class PRE>
 constexpr bool kResTileFor = MODE == kModeStore && !GROUPED && CL == kClPair && PRE::kHasRes;
+// The residual-tile variants need few registers per thread (no operands staged
+// in registers), so they run 12 epilogue warps (3 per TMEM lane quadrant) in
+// 448 threads; the others 8 (2 per quadrant) in 320.
+template <int MODE, bool GROUPED, int CL, class PRE>
+constexpr int kThreadsFor = 64 + 32 * (kResTileFor<MODE, GROUPED, CL, PRE> ? 12 : kEpiWarps);
 
 template <int BN, int STAGES, int MODE, bool GROUPED, int CL, bool RT = false>
 struct TcCfg {
   static constexpr bool CTA2 = CL != kClOne;  // tcgen05 CTA-pair MMAs
+  static constexpr int kEpiW = RT ? 12 : kEpiWarps;  // epilogue warps
+  static constexpr int kH = kEpiW / 4;               // epilogue warps per TMEM lane quadrant
+  static constexpr int kThr = 64 + 32 * kEpiW;
   static constexpr bool kQuad = CL == kClQuad;
   static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN");
   static_assert(!(GROUPED && CTA2), "grouped GEMMs use single-CTA tiles");
@@ -87,7 +95,7 @@ struct TcCfg {
   // accumulator buffer b starts at TMEM column b * kAccStride
   static constexpr int kAccStride = pow2_at_least(BN);
   static constexpr int kTmemCols = 2 * kAccStride;
-  static constexpr int kBarBytes = (8 * (2 * STAGES + 7 + kEpiWarps) + 63) / 64 * 64;  // keeps what follows 64-B aligned
+  static constexpr int kBarBytes = (8 * (2 * STAGES + 7 + kEpiW) + 63) / 64 * 64;  // keeps what follows 64-B aligned
   // per-warp 1 KB tile buffers (1 KB aligned, right after the stages): two for
   // the asynchronous TMA stores, plus (store mode) one for the residual
   // transposition, which must not reuse a buffer a TMA store may still read
@@ -100,9 +108,9 @@ struct TcCfg {
   static constexpr int kResBlocksPerSlot = kABytes / 2048 + kBBytes / 2048;
   static_assert(!RT || 2 * kResBlocksPerSlot >= (BN / 32) * 4, "residual tile fits two ring slots");
   static_assert(!RT || STAGES >= 3, "residual tile needs two slots beside an operand slot");
-  static constexpr int kStagingBytes = kEpiWarps * kWarpStaging;
+  static constexpr int kStagingBytes = kEpiW * kWarpStaging;
   // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
-  static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiWarps * 3 * 4 * 32 * 4 : 0;
+  static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiW * 3 * 4 * 32 * 4 : 0;
   // flags + row-statistics exchange between the two warps of a quadrant (2 KB)
   // + (quad) the other pair's per-row statistics, two slots (2 KB)
   static constexpr int kMiscBytes = 64 + 2 * kBM * 8 + (kQuad ? 2 * kBM * 8 : 0);
@@ -124,7 +132,7 @@ struct UnitInfo {
 // PRE / POST: compiled op programs (Prog<...>) for the chain before / after the
 // reduction, or Interp for arbitrary chains.
 template <int BN, int STAGES, int MODE, bool GROUPED, int CL, class PRE = Interp, class POST = Interp>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmR,
                       const __grid_constant__ TcParams p, const int32_t sub_tiles) {
@@ -147,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* acce = bars + 2 * STAGES + 2;
   uint64_t* drain = bars + 2 * STAGES + 4;
   uint64_t* xbar = bars + 2 * STAGES + 5;  // quad: the other pair's statistics have landed (2 slots)
-  uint64_t* rbar = bars + 2 * STAGES + 7;  // residual tile: warp ew's rows have landed (kEpiWarps)
+  uint64_t* rbar = bars + 2 * STAGES + 7;  // residual tile: warp ew's rows have landed (one per epilogue warp)
   uint32_t* misc = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(bars) + Cfg::kBarBytes);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
@@ -188,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&accf[a], 1);
-      mbar_init(&acce[a], kEpiWarps * (CTA2 ? 2 : 1));
+      mbar_init(&acce[a], Cfg::kEpiW * (CTA2 ? 2 : 1));
     }
     mbar_init(drain, 1);
     if constexpr (QUAD) {
@@ -196,7 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&xbar[1], kBM);
     }
     if constexpr (RT)
-      for (int w = 0; w < kEpiWarps; ++w) mbar_init(&rbar[w], 1);
+      for (int w = 0; w < Cfg::kEpiW; ++w) mbar_init(&rbar[w], 1);
     *abort_flag = 0;
     *zero_flag = 0;
     rdone[0] = 0;
@@ -362,15 +370,15 @@ __global__ void __launch_bounds__(kThreads, 1)
               ++it;
             }
             if (!ok) break;
-            for (int w = 0; w < kEpiWarps; ++w) {
+            for (int w = 0; w < Cfg::kEpiW; ++w) {
               uint32_t bytes = 0;
-              for (int c = w >> 2; c < Cfg::kOutN / 32; c += 2)
+              for (int c = w >> 2; c < Cfg::kOutN / 32; c += Cfg::kH)
                 if (ui.n0 + c * 32 < p.N) bytes += 2048;
               mbar_arrive_expect_tx(&rbar[w], bytes);
             }
             for (int c = 0; c < Cfg::kOutN / 32 && ui.n0 + c * 32 < p.N; ++c)
               for (int qq = 0; qq < 4; ++qq)
-                tma_load_2d(res_block(sr[0], sr[1], c, qq), &tmR, &rbar[(c & 1) * 4 + ((qq + 2) & 3)], ui.n0 + c * 32,
+                tma_load_2d(res_block(sr[0], sr[1], c, qq), &tmR, &rbar[(c % Cfg::kH) * 4 + ((qq + 2) & 3)], ui.n0 + c * 32,
                             ui.m0 + qq * 32);
             ++rt_units;
           }
@@ -380,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if constexpr (RT) {
           // residual copies still in flight land before the CTA exits
           if (rt_units > 0)
-            for (int w = 0; w < kEpiWarps; ++w) mbar_wait(&rbar[w], (rt_units - 1) & 1, zero_flag, p.drain_ns);
+            for (int w = 0; w < Cfg::kEpiW; ++w) mbar_wait(&rbar[w], (rt_units - 1) & 1, zero_flag, p.drain_ns);
         }
         if (!CTA2 || leader) {
           // wait (bounded) for the copies still in flight before the CTA exits
@@ -561,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint4 rt_bias = make_uint4(0u, 0u, 0u, 0u);
         if constexpr (RT) {
           if (lane < 16) {
-            const int c = h + 2 * (lane >> 2);
+            const int c = h + Cfg::kH * (lane >> 2);
             const int32_t col = ui.n0 + c * 32 + (lane & 3) * 8;
             if (c < Cfg::kOutN / 32 && col + 8 <= p.N) rt_bias = ldg_v4_pinned(rt_bias_ptr + col);
           }
@@ -599,7 +607,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        for (int c = h; c < Cfg::kOutN / 32; c += 2) {
+        for (int c = h; c < Cfg::kOutN / 32; c += Cfg::kH) {
           const int32_t col0 = ui.n0 + c * 32;
           const int nvalid = min(32, p.N - col0);
           if (nvalid <= 0) break;  // uniform across the warp
@@ -609,7 +617,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // residual from the tile (64-byte swizzle, row = lane), bias from the
             // warp's cache; the result overwrites the residual in place
             uint8_t* blk = res_block(rt_s0, rt_s1, c, q);
-            const uint4* bc = reinterpret_cast<const uint4*>(bcache + ((c - h) >> 1) * 64);
+            const uint4* bc = reinterpret_cast<const uint4*>(bcache + ((c - h) / Cfg::kH) * 64);
             Staged32 sg;
             sg.use_res = true;
             sg.vec_idx = p.vec_op;
@@ -703,7 +711,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) {
             bulk_wait_group_read<0>();
             __threadfence_block();
-            if (atomicAdd(&rdone[tl & 1], 1) == kEpiWarps - 1) {
+            if (atomicAdd(&rdone[tl & 1], 1) == Cfg::kEpiW - 1) {
               rdone[tl & 1] = 0;
               __threadfence_block();
               mbar_arrive(&empty[rt_s0]);

@@ -21,7 +21,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     configured[dev] = true;
   }
   static const CUtensorMap none = {};  // grouped variants stage no residual tile
-  return launch_k(kern, dim3(grid), dim3(kThreads), Cfg::kSmemBytes, s, pdl, a, b, c, none, p, static_cast<int32_t>(1));
+  return launch_k(kern, dim3(grid), dim3(Cfg::kThr), Cfg::kSmemBytes, s, pdl, a, b, c, none, p, static_cast<int32_t>(1));
 }
 
 }  // namespace
