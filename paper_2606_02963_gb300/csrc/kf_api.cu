@@ -465,6 +465,7 @@ kf_status kf_get_device_error(void* stream, uint32_t* raw) {
   if (raw) *raw = v;
   if (v & (kErrWaitProducer | kErrWaitMma | kErrWaitEpilogue)) return KF_ERR_DEVICE_TIMEOUT;
   if (v & kErrBounds) return KF_ERR_DEVICE_BOUNDS;
+  if (v & kErrLaunchShape) return KF_ERR_CUDA;
   return KF_OK;
 }
 

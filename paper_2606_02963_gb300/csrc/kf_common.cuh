@@ -21,6 +21,7 @@ constexpr uint32_t kErrWaitProducer = 1u;
 constexpr uint32_t kErrWaitMma = 2u;
 constexpr uint32_t kErrWaitEpilogue = 4u;
 constexpr uint32_t kErrBounds = 8u;
+constexpr uint32_t kErrLaunchShape = 16u;  // grid or cluster shape not the variant's
 
 struct DevOp {
   int32_t kind;

@@ -168,6 +168,19 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
   int32_t* off_s = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(misc) + Cfg::kMiscBytes);
   int32_t* ustart_s = off_s + (kMaxGroups + 1);
 
+  // The CTA-pair instructions address the peer CTA of the cluster, and the
+  // unit / couple arithmetic assumes the grid the host sized: refuse any other
+  // launch shape (all threads alike, before any barrier, TMEM or copy).
+  {
+    constexpr uint32_t kCluster = QUAD ? 4u : (CTA2 ? 2u : 1u);
+    constexpr uint32_t kGridMult = COUPLE ? 4u : kCluster;
+    const uint32_t ncl = CTA2 ? cluster_nctarank() : 1u;
+    if (ncl != kCluster || blockDim.x != static_cast<uint32_t>(Cfg::kThr) || gridDim.x % kGridMult != 0 ||
+        gridDim.y != 1 || gridDim.z != 1) {
+      if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
+      return;
+    }
+  }
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   // CTA pairs are the cluster ranks that differ in bit 0; the even rank leads
