@@ -87,6 +87,8 @@ def _load():
             lib.orc_grouped_gemm.argtypes = [P, ctypes.c_int, I64, P, P, ctypes.c_int, I64, I64, P, I32,
                                              I64, I64, P, ctypes.c_int, P, I64]
             lib.orc_grouped_gemm.restype = ctypes.c_int
+            lib.orc_add_rmsnorm.argtypes = [P, P, ctypes.c_int, P, ctypes.c_int, D, I64, I64, P, P]
+            lib.orc_add_rmsnorm.restype = ctypes.c_int
             lib.orc_round_bf16.argtypes = [D]
             lib.orc_round_bf16.restype = D
             _lib = lib
@@ -236,6 +238,24 @@ def grouped_gemm(A, B, offsets, N: int, chain: Sequence[Tuple[str, Dict]], row_i
                          b.shape[1] * K, _ptr(off), G, N, K, ctypes.cast(ops, ctypes.c_void_p),
                          len(chain), _ptr(out), N)
     return out
+
+
+def add_rmsnorm(Y, R, gamma, eps: float) -> Tuple[np.ndarray, np.ndarray]:
+    """Block tail after the MoE FFN (Sec. IV-A, Fused Add + RMSNorm with the MoE
+    finalize): R_out = bf16(R + Y); normed = R_out / sqrt(mean(R_out^2) + eps) *
+    gamma per row.  Y float64 [T, H] (the unrounded MoE output), R [T, H] and
+    gamma [H] at their stored dtype.  Returns (R_out, normed), float64."""
+    lib = _load()
+    y = np.ascontiguousarray(np.asarray(Y, dtype=np.float64))
+    r, rt = _np(R)
+    g, gt = _np(gamma)
+    T, H = y.shape
+    r_out = np.zeros((T, H), np.float64)
+    normed = np.zeros((T, H), np.float64)
+    st = lib.orc_add_rmsnorm(_ptr(y), _ptr(r), rt, _ptr(g), gt, float(eps), T, H, _ptr(r_out), _ptr(normed))
+    if st != 0:
+        raise ValueError("orc_add_rmsnorm: bad arguments")
+    return r_out, normed
 
 
 def round_bf16(x: float) -> float:

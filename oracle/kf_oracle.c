@@ -21,6 +21,12 @@
  *     Y_t = sum_j w_tj * W_down[e_tj] (silu(W_gate[e_tj] x_t) * (W_up[e_tj] x_t)),
  *     with the intermediate h rounded to bf16 (the down GEMM consumes bf16 h);
  *     the "MoE finalize" kernel of Table 1 is the routing-weighted sum over j.
+ *   - the block tail after the MoE FFN (Sec. IV-A: "Fused Add + RMSNorm" and
+ *     "MoE finalize" of the gpt-oss decode path; Sec. VI: fusing kernels of one
+ *     block) is the residual add and RMS normalisation of the new residual
+ *     stream: R_out = bf16(R + Y), normed_j = R_out_j / sqrt(mean(R_out^2) + eps)
+ *     * gamma_j -- the norm reads the stored (bf16) residual, as the next layer
+ *     would.
  *
  * Threads (pthreads) split independent rows / tokens; each row is computed by
  * one thread in a fixed order, so results do not depend on the thread count.
@@ -390,6 +396,24 @@ int orc_moe_ffn(const uint16_t *X, const uint16_t *W_gu, const uint16_t *W_down,
 /* A [* x K] (ld lda), B rows of length K (ld ldb).  out is double with ld ldo. */
 /* Single-threaded over rows when scattering (fixed summation order).           */
 /* ------------------------------------------------------------------------- */
+/* Residual add + RMSNorm per row (see the header): R, gamma read at their stored
+ * dtype, Y in double; R_out (double, holding bf16 values) and normed (double). */
+int orc_add_rmsnorm(const double *Y, const void *R, int rt, const void *gamma, int gt, double eps, int64_t T,
+                    int64_t H, double *R_out, double *normed) {
+  if (T < 0 || H < 1 || !(eps >= 0.0)) return 1;
+  for (int64_t t = 0; t < T; ++t) {
+    double ss = 0.0;
+    for (int64_t j = 0; j < H; ++j) {
+      const double h = orc_round_bf16(orc_load(R, rt, t * H + j) + Y[t * H + j]);
+      R_out[t * H + j] = h;
+      ss += h * h;
+    }
+    const double inv = 1.0 / sqrt(ss / (double)H + eps);
+    for (int64_t j = 0; j < H; ++j) normed[t * H + j] = R_out[t * H + j] * inv * orc_load(gamma, gt, j);
+  }
+  return 0;
+}
+
 int orc_grouped_gemm(const void *A, int at, int64_t lda, const int32_t *row_index, const void *B,
                      int bt, int64_t ldb, int64_t b_group_stride, const int32_t *offsets, int32_t G,
                      int64_t N, int64_t K, const orc_op *ops, int n_ops, double *out, int64_t ldo) {

@@ -25,6 +25,10 @@ MUTATIONS = {
     "moe_drop_weight": ("y[c] += wt * acc;", "y[c] += acc;"),
     "bf16_round_bits": ("ldexp(1.0, e - 8)", "ldexp(1.0, e - 9)"),
     "scale_ignored": ("case ORC_SCALE: return v * op->scalar;", "case ORC_SCALE: return v;"),
+    "rmsnorm_no_eps": ("sqrt(ss / (double)H + eps)", "sqrt(ss / (double)H)"),
+    "rmsnorm_sum_not_mean": ("sqrt(ss / (double)H + eps)", "sqrt(ss + eps)"),
+    "rmsnorm_unrounded_residual": ("const double h = orc_round_bf16(orc_load(R, rt, t * H + j) + Y[t * H + j]);",
+                                   "const double h = orc_load(R, rt, t * H + j) + Y[t * H + j];"),
     "residual_dropped": ("case ORC_RESIDUAL_ADD: return v + orc_load", "case ORC_RESIDUAL_ADD: return v + 0 * orc_load"),
 }
 

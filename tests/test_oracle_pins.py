@@ -347,3 +347,48 @@ def test_row_scale_multiplies_each_row():
     sc = torch.tensor([1.0, -2.0, 0.5, 0.0, 3.0])
     Y = oracle.fused_gemm(X, W, [("row_scale", {"p0": sc})])
     assert np.array_equal(Y, (f64(X) @ f64(W).T) * sc.double().numpy()[:, None])
+
+
+# ------------------------------------------- residual add + RMSNorm (block tail)
+def test_add_rmsnorm_matches_torch_rms_norm():
+    # R + Y chosen exactly representable in fp32, so torch's fp32 -> bf16 rounding
+    # gives the exact bf16 residual independently of the oracle's own rounding
+    g = torch.Generator().manual_seed(21)
+    T, H = 6, 40
+    R = bf16(torch.randn(T, H, generator=g))
+    Y = (torch.randint(-512, 513, (T, H), generator=g).double() / 256.0).numpy()
+    gamma = bf16(torch.rand(H, generator=g) + 0.5)
+    eps = 1e-5
+    r_out, normed = oracle.add_rmsnorm(Y, R, gamma, eps)
+    r_ref = (R.double() + torch.from_numpy(Y)).float().to(torch.bfloat16).double()
+    assert np.array_equal(r_out, r_ref.numpy())
+    ref = F.rms_norm(r_ref, (H,), weight=gamma.double(), eps=eps)
+    assert np.allclose(normed, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_add_rmsnorm_constant_row_and_moments():
+    T, H = 3, 16
+    R = bf16(torch.zeros(T, H))
+    Y = np.array([[1.5] * H, [-3.0] * H, [0.25] * H])
+    gamma = bf16(torch.ones(H))
+    eps = 0.01
+    r_out, normed = oracle.add_rmsnorm(Y, R, gamma, eps)
+    for t, c in enumerate((1.5, -3.0, 0.25)):
+        assert np.all(r_out[t] == c)
+        assert np.allclose(normed[t], c / math.sqrt(c * c + eps), rtol=1e-14)
+    # unit gamma: mean of normed^2 = ms / (ms + eps) exactly
+    g = torch.Generator().manual_seed(22)
+    Yr = torch.randn(4, 64, generator=g).double().numpy()
+    r_out, normed = oracle.add_rmsnorm(Yr, bf16(torch.zeros(4, 64)), bf16(torch.ones(64)), eps)
+    ms = (r_out ** 2).mean(axis=1)
+    assert np.allclose((normed ** 2).mean(axis=1), ms / (ms + eps), rtol=1e-12)
+
+
+def test_add_rmsnorm_scale_invariant_without_eps():
+    g = torch.Generator().manual_seed(23)
+    Yr = (torch.randint(-64, 65, (3, 32), generator=g).double() / 16.0).numpy()
+    gamma = bf16(torch.rand(32, generator=g) + 0.5)
+    R0 = bf16(torch.zeros(3, 32))
+    _, n1 = oracle.add_rmsnorm(Yr, R0, gamma, 0.0)
+    _, n2 = oracle.add_rmsnorm(Yr * 8.0, R0, gamma, 0.0)  # power of two: rounding commutes
+    assert np.allclose(n1, n2, rtol=1e-14, atol=1e-14)
