@@ -364,6 +364,31 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
                             "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
                             "experts_touched": touched, "eager_ms": round(ms_e, 5),
                             "speedup_vs_eager": round(ms_e / ms, 3), "launches_per_step": 6}
+    # MoE block tail at decode: residual add + RMSNorm fused into the MoE finalize,
+    # against the same MoE FFN followed by torch's add and rms_norm
+    T = 64
+    g = torch.Generator("cpu").manual_seed(0)
+    X = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
+    logits = torch.randn(T, E, generator=g).to(dev)
+    R = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
+    gamma = (torch.rand(H, generator=g) + 0.5).to(torch.bfloat16).to(dev)
+    ws = torch.empty(kf.moe_ffn_workspace_bytes(T, H, I, E, k), dtype=torch.uint8, device=dev)
+    y_out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
+    r_out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
+    fused = lambda: kf.moe_ffn_add_rmsnorm(X, logits, m["W_gu"], m["W_down"], k, R, gamma, 1e-5, out=y_out,
+                                           r_out=r_out, workspace=ws)
+    def unfused():
+        y = kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, workspace=ws)
+        h = R + y
+        return F.rms_norm(h, (H,), weight=gamma, eps=1e-5), h
+    ms = time_steps(fused, steps, args.warmup, flush, stream)
+    ms_u = time_steps(unfused, steps, args.warmup, flush, stream)
+    touched = int(torch.unique(torch.topk(logits, k, dim=1).indices).numel())
+    byts = touched * (2 * I * H + H * I) * 2 + T * H * 2 * 4 + 4 * T * E
+    res["moe_T64_add_rmsnorm"] = {"ms": round(ms, 5), "gbs": round(byts / ms / 1e6, 1), "bound": "hbm",
+                                  "roofline_frac": round(byts / (peaks["hbm"] * 1e9) * 1e3 / ms, 4),
+                                  "unfused_ms": round(ms_u, 5), "speedup_vs_unfused": round(ms_u / ms, 3),
+                                  "launches_per_step": 6}
     return res
 
 

@@ -196,6 +196,29 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
 size_t kf_moe_ffn_workspace_ex(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags);
 
 /*
+ * kf_moe_ffn_add_rmsnorm -- the MoE block tail fused into the MoE finalize
+ *                          (Sec. IV-A: the gpt-oss decode kernels "Fused Add +
+ *                          RMSNorm" and "MoE finalize"; Sec. VI: optimising the
+ *                          kernels of one block together)
+ *
+ *   The routed expert FFN of kf_moe_ffn_ex (same arguments and flags), whose
+ *   finalize, instead of writing the FFN output, adds it to the residual stream
+ *   and normalises the result:
+ *     R_out[t,:] = bf16(R[t,:] + MoE(X)[t,:])                (new residual stream)
+ *     Y[t,j]     = bf16(R_out[t,j] / sqrt(mean_j R_out[t,j]^2 + eps) * gamma[j])
+ *   The norm reads the stored bf16 residual, as the next layer would.  R, R_out,
+ *   Y bf16 [T x H] (row stride H), gamma bf16 [H], all 16-byte aligned
+ *   (KF_ERR_MISALIGNED otherwise); R may be R_out (in place).  H <= 8192
+ *   (KF_ERR_UNSUPPORTED above), eps >= 0 (KF_ERR_INVALID_ARG otherwise).
+ *   workspace: kf_moe_ffn_workspace_ex(T, H, I, E, k, flags) bytes, owned by the
+ *   caller like every buffer here; calls sharing it must not overlap on the GPU.
+ */
+kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void* W_gu, const void* W_down,
+                                 const void* R, const void* gamma, float eps, void* R_out, void* Y, int64_t T,
+                                 int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace,
+                                 size_t workspace_bytes, int32_t* topk_ids_out, float* topk_w_out, void* stream);
+
+/*
  * kf_fused_gemm_lse_noalloc -- kf_fused_gemm for row log-sum-exp chains, without
  * a workspace argument.  The paper has no counterpart: this entry point exists for
  * callers that cannot allocate device memory -- e.g. code hosted by another

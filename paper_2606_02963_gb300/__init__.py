@@ -35,7 +35,7 @@ ABI_SYMBOLS = (
     "kf_fused_gemm", "kf_fused_gemm_workspace", "kf_moe_route", "kf_grouped_gemm",
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
-    "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex",
+    "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex", "kf_moe_ffn_add_rmsnorm",
 )
 
 
@@ -81,6 +81,9 @@ def lib() -> ctypes.CDLL:
     L.kf_moe_ffn_workspace.restype = SZ
     L.kf_moe_ffn_ex.argtypes = [P, P, P, P, P, I64, I64, I64, I32, I32, ctypes.c_uint32, P, SZ, P, P, P]
     L.kf_moe_ffn_ex.restype = I32
+    L.kf_moe_ffn_add_rmsnorm.argtypes = [P, P, P, P, P, P, ctypes.c_float, P, P, I64, I64, I64, I32, I32,
+                                         ctypes.c_uint32, P, SZ, P, P, P]
+    L.kf_moe_ffn_add_rmsnorm.restype = I32
     L.kf_moe_ffn_workspace_ex.argtypes = [I64, I64, I64, I32, I32, ctypes.c_uint32]
     L.kf_moe_ffn_workspace_ex.restype = SZ
     L.kf_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
@@ -270,6 +273,33 @@ def moe_ffn(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tensor, W_down: t
                          I, E, k, flags, _ptr(ws), ws_bytes, _ptr(ids), _ptr(w), _stream(stream))
     _check(st, "kf_moe_ffn_ex")
     return (out, ids, w) if return_routing else out
+
+
+def moe_ffn_add_rmsnorm(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tensor, W_down: torch.Tensor, k: int,
+                        R: torch.Tensor, gamma: torch.Tensor, eps: float, out: Optional[torch.Tensor] = None,
+                        r_out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                        deterministic: bool = False, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """MoE block tail fused into the finalize (kf_moe_ffn_add_rmsnorm): returns
+    (Y, R_out) with R_out = bf16(R + MoE(X)) and Y = bf16(rmsnorm(R_out) * gamma).
+    ``r_out`` may be ``R`` (in-place residual update)."""
+    T, H = X.shape
+    E, I2, _ = W_gu.shape
+    I = I2 // 2
+    for t, nm in ((X, "X"), (logits, "logits"), (W_gu, "W_gu"), (W_down, "W_down"), (R, "R"), (gamma, "gamma")):
+        if not t.is_contiguous():
+            raise ValueError(f"{nm} must be contiguous")
+    if out is None:
+        out = torch.empty(T, H, dtype=torch.bfloat16, device=X.device)
+    if r_out is None:
+        r_out = torch.empty(T, H, dtype=torch.bfloat16, device=X.device)
+    L = lib()
+    flags = KF_MOE_DETERMINISTIC if deterministic else 0
+    ws, ws_bytes = _workspace(L.kf_moe_ffn_workspace_ex(T, H, I, E, k, flags), X.device, workspace)
+    st = L.kf_moe_ffn_add_rmsnorm(X.data_ptr(), logits.data_ptr(), W_gu.data_ptr(), W_down.data_ptr(), R.data_ptr(),
+                                  gamma.data_ptr(), float(eps), r_out.data_ptr(), out.data_ptr(), T, H, I, E, k, flags,
+                                  _ptr(ws), ws_bytes, None, None, _stream(stream))
+    _check(st, "kf_moe_ffn_add_rmsnorm")
+    return out, r_out
 
 
 def get_device_error(stream=None) -> Tuple[int, int]:

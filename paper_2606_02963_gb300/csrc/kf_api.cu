@@ -724,9 +724,20 @@ kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const
                        stream);
 }
 
-kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
-                        int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace, size_t ws_bytes,
-                        int32_t* topk_ids_out, float* topk_w_out, void* stream) {
+}  // extern "C"
+
+namespace {
+// Residual add + RMSNorm that replaces the MoE finalize's plain bf16 output.
+struct BlockTail {
+  const void* R;
+  const void* gamma;
+  float eps;
+  void* R_out;
+};
+
+kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
+                       int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace, size_t ws_bytes,
+                       int32_t* topk_ids_out, float* topk_w_out, void* stream, const BlockTail* tail) {
   if (flags & ~KF_MOE_DETERMINISTIC) return KF_ERR_INVALID_ARG;
   const bool det = (flags & KF_MOE_DETERMINISTIC) != 0;
   if (T < 0 || H < 1 || I < 1 || E < 1 || E > 256 || k < 1 || k > E) return KF_ERR_INVALID_ARG;
@@ -787,7 +798,11 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yp, KF_F32, H};
     st = grouped_core(g, pl, nullptr, s, di, true);
     if (st != KF_OK) return st;
-    st = cuda_status(moe_finalize_launch(yp, pos, T, k, H, Y, s, true));
+    if (tail)
+      st = cuda_status(moe_add_rmsnorm_launch(nullptr, yp, pos, k, T, H, tail->R, tail->gamma, tail->eps, tail->R_out, Y,
+                                              s, true));
+    else
+      st = cuda_status(moe_finalize_launch(yp, pos, T, k, H, Y, s, true));
     if (st != KF_OK) return st;
   } else {
     // down: Yacc[token] += w * (h W_down[e]^T), then bf16
@@ -804,7 +819,11 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yacc, KF_F32, H};
     st = grouped_core(g, pl, nullptr, s, di, true);
     if (st != KF_OK) return st;
-    st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s, true));
+    if (tail)
+      st = cuda_status(moe_add_rmsnorm_launch(yacc, nullptr, nullptr, k, T, H, tail->R, tail->gamma, tail->eps,
+                                              tail->R_out, Y, s, true));
+    else
+      st = cuda_status(cvt_f32_bf16_launch(yacc, Y, T * H, s, true));
     if (st != KF_OK) return st;
   }
   if (topk_ids_out &&
@@ -814,6 +833,29 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
       cudaMemcpyAsync(topk_w_out, w, static_cast<size_t>(P) * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
     return KF_ERR_CUDA;
   return KF_OK;
+}
+}  // namespace
+
+extern "C" {
+
+kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
+                        int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace, size_t ws_bytes,
+                        int32_t* topk_ids_out, float* topk_w_out, void* stream) {
+  return moe_ffn_impl(X, logits, W_gu, W_down, Y, T, H, I, E, k, flags, workspace, ws_bytes, topk_ids_out, topk_w_out,
+                      stream, nullptr);
+}
+
+kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void* W_gu, const void* W_down,
+                                 const void* R, const void* gamma, float eps, void* R_out, void* Y, int64_t T,
+                                 int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace,
+                                 size_t ws_bytes, int32_t* topk_ids_out, float* topk_w_out, void* stream) {
+  if (!(eps >= 0.0f) || eps > 1e30f) return KF_ERR_INVALID_ARG;
+  if (T > 0 && (!R || !gamma || !R_out)) return KF_ERR_INVALID_ARG;
+  if (H > kAddRmsNormMaxH) return KF_ERR_UNSUPPORTED;
+  if (T > 0 && (!aligned16(R) || !aligned16(gamma) || !aligned16(R_out))) return KF_ERR_MISALIGNED;
+  const BlockTail tail{R, gamma, eps, R_out};
+  return moe_ffn_impl(X, logits, W_gu, W_down, Y, T, H, I, E, k, flags, workspace, ws_bytes, topk_ids_out, topk_w_out,
+                      stream, &tail);
 }
 
 }  // extern "C"

@@ -320,6 +320,88 @@ cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_
                   pair_pos, T, k, h4, reinterpret_cast<uint2*>(Y));
 }
 
+// ------------------------------------------- MoE block tail: add + RMSNorm
+// One block per token t (Sec. IV-A: Fused Add + RMSNorm and MoE finalize of the
+// gpt-oss decode path, fused): y = the token's MoE output (the fp32 accumulator,
+// or in slot order the sum of its k per-row outputs), R_out = bf16(R + y) (the
+// new residual stream), Y = bf16(R_out * rsqrt(mean(R_out^2) + eps) * gamma).
+// Each thread keeps its (up to kArnMaxV) 4-column groups of R_out in registers
+// between the sum of squares and the normalisation.  R may alias R_out.
+constexpr int kArnThreads = 256;
+constexpr int kArnMaxV = 8;  // H <= 4 * 256 * 8 = 8192
+__global__ void __launch_bounds__(kArnThreads)
+    moe_add_rmsnorm_kernel(const float4* __restrict__ yacc, const float4* __restrict__ yp,
+                           const int32_t* __restrict__ pair_pos, int32_t k, int64_t h4, const uint2* R,
+                           const uint2* __restrict__ gamma, float eps, uint2* R_out, uint2* __restrict__ Y) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
+  const int64_t t = blockIdx.x;
+  float4 hv[kArnMaxV];
+  float ss = 0.0f;
+#pragma unroll
+  for (int v = 0; v < kArnMaxV; ++v) {
+    const int64_t c = threadIdx.x + static_cast<int64_t>(v) * kArnThreads;
+    if (c < h4) {
+      float4 y;
+      if (yacc) {
+        y = yacc[t * h4 + c];
+      } else {
+        y = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int32_t j = 0; j < k; ++j) {
+          const float4 q = yp[static_cast<int64_t>(pair_pos[t * k + j]) * h4 + c];
+          y.x += q.x;
+          y.y += q.y;
+          y.z += q.z;
+          y.w += q.w;
+        }
+      }
+      const uint2 r = R[t * h4 + c];
+      uint2 o;
+      o.x = pack_bf16x2(bf16lo(r.x) + y.x, bf16hi(r.x) + y.y);
+      o.y = pack_bf16x2(bf16lo(r.y) + y.z, bf16hi(r.y) + y.w);
+      R_out[t * h4 + c] = o;
+      const float4 h = make_float4(bf16lo(o.x), bf16hi(o.x), bf16lo(o.y), bf16hi(o.y));  // the stored residual
+      hv[v] = h;
+      ss += h.x * h.x + h.y * h.y + h.z * h.z + h.w * h.w;
+    }
+  }
+  __shared__ float part[kArnThreads / 32];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < kArnThreads / 32 ? part[threadIdx.x] : 0.0f;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (threadIdx.x == 0) part[0] = v;
+  }
+  __syncthreads();
+  const float inv = rsqrtf(part[0] / static_cast<float>(4 * h4) + eps);
+#pragma unroll
+  for (int v = 0; v < kArnMaxV; ++v) {
+    const int64_t c = threadIdx.x + static_cast<int64_t>(v) * kArnThreads;
+    if (c < h4) {
+      const uint2 g = gamma[c];
+      uint2 o;
+      o.x = pack_bf16x2(hv[v].x * inv * bf16lo(g.x), hv[v].y * inv * bf16hi(g.x));
+      o.y = pack_bf16x2(hv[v].z * inv * bf16lo(g.y), hv[v].w * inv * bf16hi(g.y));
+      Y[t * h4 + c] = o;
+    }
+  }
+}
+
+cudaError_t moe_add_rmsnorm_launch(const float* yacc, const float* yp, const int32_t* pair_pos, int32_t k, int64_t T,
+                                   int64_t H, const void* R, const void* gamma, float eps, void* R_out, void* Y,
+                                   cudaStream_t s, bool pdl) {
+  if (T == 0) return cudaSuccess;
+  if (H % 4 != 0 || H / 4 > static_cast<int64_t>(kArnThreads) * kArnMaxV) return cudaErrorInvalidValue;
+  return launch_k(moe_add_rmsnorm_kernel, dim3(static_cast<unsigned>(T)), dim3(kArnThreads), 0, s, pdl,
+                  reinterpret_cast<const float4*>(yacc), reinterpret_cast<const float4*>(yp), pair_pos, k, H / 4,
+                  reinterpret_cast<const uint2*>(R), reinterpret_cast<const uint2*>(gamma), eps,
+                  reinterpret_cast<uint2*>(R_out), reinterpret_cast<uint2*>(Y));
+}
+
 // ----------------------------------------------------------------- row gather
 // out[r, :] = A[idx[r], :] (16-byte vectors; K % 8 == 0 bf16).  An index out of
 // range writes a zero row and sets the bounds bit of the error word.

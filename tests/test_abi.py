@@ -170,3 +170,15 @@ def test_product_path_does_not_touch_the_oracle():
                 assert "oracle" not in src.replace("oracle-free", ""), fn
     out = subprocess.run(["ldd", kf.LIB_PATH], capture_output=True, text=True).stdout
     assert "oracle" not in out
+
+
+def test_moe_add_rmsnorm_argument_errors_before_any_launch():
+    L = kf.lib()
+    fake = 1 << 20  # aligned, never dereferenced: the checks come first
+    def call(H=2880, eps=1e-5, R=fake):
+        return L.kf_moe_ffn_add_rmsnorm(fake, fake, fake, fake, R, fake, eps, fake, fake, 4, H, 2880, 32, 4, 0,
+                                        fake, 1 << 30, None, None, None)
+    assert call(H=16384) == kf.KF_ERR_UNSUPPORTED
+    assert call(eps=-1.0) == kf.KF_ERR_INVALID_ARG
+    assert call(R=None) == kf.KF_ERR_INVALID_ARG
+    assert call(R=fake + 4) == kf.KF_ERR_MISALIGNED

@@ -155,3 +155,51 @@ def test_grouped_row_scale_store():
                         out_dtype=torch.float32)
     ref = oracle.grouped_gemm(A, B, off.numpy(), N, [("row_scale", {"p0": sc})])
     check_f32(C, ref, "row scale")
+
+
+# ------------------------------------------------- MoE block tail: add + RMSNorm
+def _block_inputs(T, H, seed):
+    g = torch.Generator().manual_seed(seed)
+    R = torch.randn(T, H, generator=g).to(torch.bfloat16)
+    gamma = (torch.rand(H, generator=g) + 0.5).to(torch.bfloat16)
+    return R, gamma
+
+
+@pytest.mark.parametrize("T,H,I,E,k,det", [(37, 256, 128, 8, 2, False), (37, 256, 128, 8, 2, True),
+                                           (64, 2880, 2880, 32, 4, False), (300, 2880, 2880, 32, 4, True)])
+def test_moe_add_rmsnorm(T, H, I, E, k, det):
+    m = kf_workloads.moe_generate(T, seed=T + 91, H=H, I=I, E=E, k=k)
+    d = {kk: v.to(DEV) for kk, v in m.items()}
+    R, gamma = _block_inputs(T, H, seed=T)
+    eps = 1e-5
+    Y, R_out = kf.moe_ffn_add_rmsnorm(d["X"], d["logits"], d["W_gu"], d["W_down"], k, R.to(DEV), gamma.to(DEV), eps,
+                                      deterministic=det)
+    torch.cuda.synchronize()
+    r = oracle.moe_route(m["logits"], k)
+    toks = list(range(T)) if T <= 64 else sorted(set([0, T - 1] + list(np.random.default_rng(3).choice(T, 14, replace=False))))
+    y = oracle.moe_ffn(m["X"], m["W_gu"], m["W_down"], r["topk_ids"], r["topk_w"], tokens=toks)
+    r_ref, n_ref = oracle.add_rmsnorm(y, R[toks], gamma, eps)
+    check_bf16(R_out[toks], r_ref, f"residual T={T} det={det}")
+    check_bf16(Y[toks], n_ref, f"normed T={T} det={det}")
+    _no_device_error()
+
+
+def test_moe_add_rmsnorm_in_place_and_consistent_with_moe_ffn():
+    T, H, I, E, k = 64, 512, 256, 16, 4
+    m = kf_workloads.moe_generate(T, seed=5, H=H, I=I, E=E, k=k)
+    d = {kk: v.to(DEV) for kk, v in m.items()}
+    R, gamma = _block_inputs(T, H, seed=6)
+    Rd = R.to(DEV)
+    Y1, R1 = kf.moe_ffn_add_rmsnorm(d["X"], d["logits"], d["W_gu"], d["W_down"], k, Rd, gamma.to(DEV), 1e-6,
+                                    deterministic=True)
+    Rin = Rd.clone()
+    Y2, R2 = kf.moe_ffn_add_rmsnorm(d["X"], d["logits"], d["W_gu"], d["W_down"], k, Rin, gamma.to(DEV), 1e-6,
+                                    r_out=Rin, deterministic=True)
+    torch.cuda.synchronize()
+    assert R2.data_ptr() == Rin.data_ptr()
+    assert torch.equal(Y1, Y2) and torch.equal(R1, R2)
+    # the residual equals R + the plain MoE output up to the bf16 rounding of that output
+    y = kf.moe_ffn(d["X"], d["logits"], d["W_gu"], d["W_down"], k, deterministic=True)
+    diff = (R1.float() - (Rd.float() + y.float())).abs()
+    assert diff.max().item() <= 2e-2 * (Rd.float() + y.float()).abs().max().item()
+    _no_device_error()
