@@ -73,11 +73,13 @@ def chain_spec(wl: Workload) -> List[Tuple[str, Dict[str, object]]]:
 def _round(t: torch.Tensor, dtype: str) -> torch.Tensor:
     if dtype == "bf16":
         return t.to(torch.bfloat16)
+    if dtype == "f16":
+        return t.to(torch.float16)
     return t.to(torch.float32)
 
 
 def generate(name: str, seed: int = 0, M: Optional[int] = None, N: Optional[int] = None,
-             K: Optional[int] = None, dist: str = "default") -> Dict[str, torch.Tensor]:
+             K: Optional[int] = None, dist: str = "default", dtype: Optional[str] = None) -> Dict[str, torch.Tensor]:
     """Draw the inputs of workload ``name`` (optionally at another M/N/K).
 
     ``dist`` selects the distribution sweep used for parity only:
@@ -86,6 +88,8 @@ def generate(name: str, seed: int = 0, M: Optional[int] = None, N: Optional[int]
       "uniform"  U(-1,1) operands,
       "offset"   the default recipe plus a large constant (+8) on the bias / first
                  operand column, which stresses max-subtraction and cancellation.
+    ``dtype`` ("bf16", "f16" or "f32") overrides the workload's dtype: the same
+    fp32 draws, rounded (RNE) to that dtype instead.
     Returns CPU tensors in the workload dtype (fp32 for fp32 workloads).
     """
     wl = WORKLOADS[name]
@@ -93,7 +97,7 @@ def generate(name: str, seed: int = 0, M: Optional[int] = None, N: Optional[int]
     N = wl.N if N is None else N
     K = wl.K if K is None else K
     g = torch.Generator("cpu").manual_seed(seed)
-    dt = wl.dtype
+    dt = wl.dtype if dtype is None else dtype
     out: Dict[str, torch.Tensor] = {}
 
     def normal(*shape, std=1.0):

@@ -42,7 +42,7 @@ _LIB_PATH = os.path.join(_BUILD, "libkf_oracle.so")
 _lock = threading.Lock()
 _lib = None
 
-ORC_F32, ORC_BF16 = 0, 1
+ORC_F32, ORC_BF16, ORC_F16 = 0, 1, 2
 KINDS = {
     "bias": 0, "scale": 1, "relu": 2, "gelu_tanh": 3, "silu": 4, "sigmoid": 5,
     "residual_add": 6, "row_logsumexp": 7, "groupnorm": 8, "swiglu": 9,
@@ -102,6 +102,8 @@ def _np(t) -> Tuple[np.ndarray, int]:
         t = t.detach().cpu().contiguous()
         if t.dtype == torch.bfloat16:
             return t.view(torch.int16).numpy().view(np.uint16), ORC_BF16
+        if t.dtype == torch.float16:
+            return t.view(torch.int16).numpy().view(np.uint16), ORC_F16
         if t.dtype == torch.float32:
             return t.numpy(), ORC_F32
         if t.dtype == torch.int32:
@@ -114,6 +116,8 @@ def _np(t) -> Tuple[np.ndarray, int]:
         return a, ORC_F32
     if a.dtype == np.uint16:
         return a, ORC_BF16
+    if a.dtype == np.float16:
+        return a.view(np.uint16), ORC_F16
     if a.dtype == np.int32:
         return a, -1
     raise TypeError(f"oracle: unsupported array dtype {a.dtype}")

@@ -39,7 +39,7 @@
 #include <unistd.h>
 
 /* dtype codes of this oracle's own interface */
-enum { ORC_F32 = 0, ORC_BF16 = 1 };
+enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_F16 = 2 };
 
 /* tail-op codes of this oracle's own interface */
 enum {
@@ -75,6 +75,20 @@ typedef struct {
 /* Widen one stored element to double.  bf16 is the top half of an IEEE
  * binary32 with the low 16 mantissa bits zero, so the widening is exact. */
 static double orc_load(const void *p, int dt, int64_t i) {
+  if (dt == ORC_F16) {
+    /* IEEE binary16: 1 sign bit, 5 exponent bits (bias 15), 10 fraction bits;
+     * exponent 0 holds the subnormals m 2^-24, exponent 31 inf / nan */
+    const uint16_t b = ((const uint16_t *)p)[i];
+    const int sign = b >> 15, ex = (b >> 10) & 31, fr = b & 1023;
+    double v;
+    if (ex == 0)
+      v = ldexp((double)fr, -24);
+    else if (ex == 31)
+      v = fr ? NAN : INFINITY;
+    else
+      v = ldexp((double)(1024 + fr), ex - 25);
+    return sign ? -v : v;
+  }
   if (dt == ORC_BF16) {
     uint32_t bits = (uint32_t)((const uint16_t *)p)[i] << 16;
     float f;

@@ -29,6 +29,8 @@ MUTATIONS = {
     "rmsnorm_sum_not_mean": ("sqrt(ss / (double)H + eps)", "sqrt(ss + eps)"),
     "rmsnorm_unrounded_residual": ("const double h = orc_round_bf16(orc_load(R, rt, t * H + j) + Y[t * H + j]);",
                                    "const double h = orc_load(R, rt, t * H + j) + Y[t * H + j];"),
+    "f16_exponent_bias": ("v = ldexp((double)(1024 + fr), ex - 25);", "v = ldexp((double)(1024 + fr), ex - 24);"),
+    "f16_subnormal_scale": ("v = ldexp((double)fr, -24);", "v = ldexp((double)fr, -25);"),
     "residual_dropped": ("case ORC_RESIDUAL_ADD: return v + orc_load", "case ORC_RESIDUAL_ADD: return v + 0 * orc_load"),
 }
 

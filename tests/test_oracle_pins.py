@@ -392,3 +392,15 @@ def test_add_rmsnorm_scale_invariant_without_eps():
     _, n1 = oracle.add_rmsnorm(Yr, R0, gamma, 0.0)
     _, n2 = oracle.add_rmsnorm(Yr * 8.0, R0, gamma, 0.0)  # power of two: rounding commutes
     assert np.allclose(n1, n2, rtol=1e-14, atol=1e-14)
+
+
+def test_f16_operands_read_exactly():
+    # every finite binary16 value, read through a K = 1 GEMM against 1.0,
+    # equals numpy's own float16 -> float64 conversion
+    bits = np.arange(0, 1 << 16, dtype=np.uint32).astype(np.uint16)
+    f = bits.view(np.float16)
+    v = f[np.isfinite(f)]
+    X = torch.ones(1, 1, dtype=torch.float16)
+    W = torch.from_numpy(v.copy()).reshape(-1, 1)
+    Y = oracle.fused_gemm(X, W, [])
+    assert np.array_equal(Y[0], v.astype(np.float64))
