@@ -52,7 +52,7 @@ typedef enum kf_status {
   KF_ERR_DEVICE_BOUNDS = 7   /* device-resident indices/offsets out of range   */
 } kf_status;
 
-typedef enum kf_dtype { KF_F32 = 0, KF_BF16 = 1, KF_I32 = 2 } kf_dtype;
+typedef enum kf_dtype { KF_F32 = 0, KF_BF16 = 1, KF_I32 = 2, KF_F16 = 3 } kf_dtype;
 
 /* Tail ops, applied in list order to the fp32 accumulator (Sec. IV-B: the
  * post-GEMM sequence of operations, fused into one kernel). */
@@ -108,8 +108,9 @@ typedef struct kf_epilogue {
  *
  *   X [M x K] (row stride ldx), W [N x K] (row stride ldw), Y [M x N] (row
  *   stride ldy), or Y [M] (fp32 or bf16) when the chain holds ROW_LOGSUMEXP.
- *   Operand dtypes: both KF_BF16 (tcgen05 tensor-core path, fp32 accumulation
- *   in tensor memory; Y bf16 or fp32), or both KF_F32 (exact fp32 FFMA path; Y
+ *   Operand dtypes: both KF_BF16 or both KF_F16 (tcgen05 tensor-core path, fp32
+ *   accumulation in tensor memory; Y bf16, fp16 or fp32; the paper's B580
+ *   kernels ran their matmuls in fp16, Sec. IV-B), or both KF_F32 (exact fp32 FFMA path; Y
  *   fp32; element-wise chains only).
  *   bf16 path: X, W must be 16-byte aligned with ldx, ldw multiples of 8, else
  *   KF_ERR_MISALIGNED.  M == 0 or N == 0 is a no-op; K must be >= 1.

@@ -23,7 +23,7 @@ LIB_PATH = os.path.join(_HERE, "libkf.so")
 
 KF_OK, KF_ERR_INVALID_ARG, KF_ERR_UNSUPPORTED, KF_ERR_MISALIGNED = 0, 1, 2, 3
 KF_ERR_WORKSPACE, KF_ERR_CUDA, KF_ERR_DEVICE_TIMEOUT, KF_ERR_DEVICE_BOUNDS = 4, 5, 6, 7
-KF_F32, KF_BF16, KF_I32 = 0, 1, 2
+KF_F32, KF_BF16, KF_I32, KF_F16 = 0, 1, 2, 3
 OPS = {
     "bias": 0, "scale": 1, "relu": 2, "gelu_tanh": 3, "silu": 4, "sigmoid": 5,
     "residual_add": 6, "row_logsumexp": 7, "groupnorm": 8, "swiglu": 9,
@@ -117,6 +117,8 @@ def _dt(t: torch.Tensor) -> int:
         return KF_F32
     if t.dtype == torch.int32:
         return KF_I32
+    if t.dtype == torch.float16:
+        return KF_F16
     raise TypeError(f"unsupported dtype {t.dtype}")
 
 

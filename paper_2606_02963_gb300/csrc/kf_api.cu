@@ -61,11 +61,12 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// bf16 tensor map, 128-byte swizzle, box = 64 (K) x box_rows (x 1).  Rank 2
-// for A operands ([rows, K]); rank 3 for B operands ([groups, rows, K]), which
-// the kernel always loads with 3-D coordinates (groups = 1 for dense calls).
+// bf16 (or fp16) tensor map, 128-byte swizzle, box = 64 (K) x box_rows (x 1).
+// Rank 2 for A operands ([rows, K]); rank 3 for B operands ([groups, rows, K]),
+// which the kernel always loads with 3-D coordinates (groups = 1 for dense calls).
 kf_status make_map(CUtensorMap* m, const void* base, uint64_t k, uint64_t rows, uint64_t row_stride_bytes,
-                   uint64_t groups, uint64_t group_stride_bytes, uint32_t box_rows, cuuint32_t rank) {
+                   uint64_t groups, uint64_t group_stride_bytes, uint32_t box_rows, cuuint32_t rank,
+                   CUtensorMapDataType dt = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   auto fn = encode_fn();
   if (!fn) return KF_ERR_CUDA;
   std::memset(m, 0, sizeof(*m));
@@ -73,7 +74,7 @@ kf_status make_map(CUtensorMap* m, const void* base, uint64_t k, uint64_t rows, 
   cuuint64_t strides[2] = {row_stride_bytes, group_stride_bytes};
   cuuint32_t box[3] = {static_cast<cuuint32_t>(kBK), box_rows, 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, estr,
+  CUresult r = fn(m, dt, rank, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
@@ -112,8 +113,8 @@ kf_status make_map_blk64(CUtensorMap* m, const void* base, uint64_t cols, uint64
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-int elt_size(int dt) { return dt == KF_BF16 ? 2 : 4; }
-bool float_dtype(int dt) { return dt == KF_F32 || dt == KF_BF16; }
+int elt_size(int dt) { return (dt == KF_BF16 || dt == KF_F16) ? 2 : 4; }
+bool float_dtype(int dt) { return dt == KF_F32 || dt == KF_BF16 || dt == KF_F16; }
 
 bool is_scalar_op(int k) {
   return k == KF_OP_SCALE || k == KF_OP_RELU || k == KF_OP_GELU_TANH || k == KF_OP_SILU || k == KF_OP_SIGMOID ||
@@ -496,7 +497,8 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     // exact fp32 FFMA path: element-wise chains only
     if (pl.mode != kModeStore || yt != KF_F32) return KF_ERR_UNSUPPORTED;
   } else {
-    if (xt != KF_BF16 || wt != KF_BF16) return KF_ERR_UNSUPPORTED;
+    // tensor-core path: A and B both bf16 or both fp16 (one operand format per MMA)
+    if (xt != wt || (xt != KF_BF16 && xt != KF_F16)) return KF_ERR_UNSUPPORTED;
     if (!aligned16(X) || !aligned16(W) || ldx % 8 != 0 || ldw % 8 != 0) return KF_ERR_MISALIGNED;
     if (pl.mode == kModeLse &&
         (!workspace || !aligned16(workspace) || ws_bytes < lse_ws_bytes(M, N)))
@@ -549,9 +551,10 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     tiles_n = (N + bn - 1) / bn;
   }
   CUtensorMap ma, mb;
-  st = make_map(&ma, X, K, M, ldx * 2, 1, 0, kBM, 2);
+  const CUtensorMapDataType op_dt = xt == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  st = make_map(&ma, X, K, M, ldx * 2, 1, 0, kBM, 2, op_dt);
   if (st != KF_OK) return st;
-  st = make_map(&mb, W, K, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, cta2 ? bn / 2 : bn, 3);
+  st = make_map(&mb, W, K, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, cta2 ? bn / 2 : bn, 3, op_dt);
   if (st != KF_OK) return st;
   TcParams p;
   std::memset(&p, 0, sizeof(p));
@@ -575,7 +578,9 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
     if (st != KF_OK) return st;
     p.c_tma = 1;
   }
-  p.fast = yt == KF_BF16 && pl.mode != kModeLse;  // bf16 results: reduced-precision activations suffice
+  // 16-bit results: reduced-precision activations suffice
+  p.fast = (yt == KF_BF16 || yt == KF_F16) && pl.mode != kModeLse;
+  p.ab_f16 = xt == KF_F16;
   const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
   // a compiled chain program, if the chain matches one (bf16 operands staged)
   int sig = kSigGeneric;

@@ -75,6 +75,7 @@ struct TcParams {
   int32_t res_op;       // index in pre[] of a bf16 RESIDUAL_ADD staged by coalesced loads, or -1
   int32_t vec_op;       // index in pre[] of a bf16 BIAS / MUL whose vector is loaded ahead, or -1
   int32_t c_tma;        // output tiles leave through TMA stores (dense, bf16, aligned)
+  int32_t ab_f16;       // A and B are fp16 (else bf16): the MMA's operand format
   // GroupNorm on couples of CTA pairs: per-row statistics exchanged through
   // global memory (workspace) -- [couples][2 slots][2 halves][256 rows] float2,
   // then [couples][2 slots][2 halves][8 row blocks] uint64 flags tagged with
@@ -88,7 +89,15 @@ struct TcParams {
 // ---------------------------------------------------------------- loads/stores
 __device__ __forceinline__ float ld_elem(const void* p, int dt, int64_t i) {
   if (dt == KF_BF16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(p)[i]);
+  if (dt == KF_F16) return __half2float(reinterpret_cast<const __half*>(p)[i]);
   return reinterpret_cast<const float*>(p)[i];
+}
+__device__ __forceinline__ float2 f16x2_to_f2(uint32_t w) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&w));
+}
+__device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
+  __half2 h = __floats2half2_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
 }
 
 // Load 32 consecutive elements starting at element index i0 (first `nvalid`
@@ -106,6 +115,19 @@ __device__ __forceinline__ void ld32(const void* p, int dt, int64_t i0, int nval
         for (int h = 0; h < 4; ++h) {
           o[v * 8 + 2 * h] = __uint_as_float(w[h] << 16);
           o[v * 8 + 2 * h + 1] = __uint_as_float(w[h] & 0xFFFF0000u);
+        }
+      }
+    } else if (dt == KF_F16) {
+      const uint4* q = reinterpret_cast<const uint4*>(reinterpret_cast<const __half*>(p) + i0);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        uint4 u = __ldg(q + v);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const float2 f = f16x2_to_f2(w[h]);
+          o[v * 8 + 2 * h] = f.x;
+          o[v * 8 + 2 * h + 1] = f.y;
         }
       }
     } else {
@@ -134,6 +156,15 @@ __device__ __forceinline__ void ld8(const void* p, int dt, int64_t i0, bool vec_
     for (int h = 0; h < 4; ++h) {
       o[2 * h] = __uint_as_float(w[h] << 16);
       o[2 * h + 1] = __uint_as_float(w[h] & 0xFFFF0000u);
+    }
+  } else if (vec_ok && dt == KF_F16) {
+    uint4 u = __ldg(reinterpret_cast<const uint4*>(reinterpret_cast<const __half*>(p) + i0));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      const float2 f = f16x2_to_f2(w[h]);
+      o[2 * h] = f.x;
+      o[2 * h + 1] = f.y;
     }
   } else if (vec_ok) {
     const float4* q = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(p) + i0);
@@ -164,6 +195,17 @@ __device__ __forceinline__ void st32(void* p, int dt, int64_t i0, int nvalid, bo
         u.w = pack_bf16x2(v[8 * c + 6], v[8 * c + 7]);
         q[c] = u;
       }
+    } else if (dt == KF_F16) {
+      uint4* q = reinterpret_cast<uint4*>(reinterpret_cast<__half*>(p) + i0);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint4 u;
+        u.x = pack_f16x2(v[8 * c + 0], v[8 * c + 1]);
+        u.y = pack_f16x2(v[8 * c + 2], v[8 * c + 3]);
+        u.z = pack_f16x2(v[8 * c + 4], v[8 * c + 5]);
+        u.w = pack_f16x2(v[8 * c + 6], v[8 * c + 7]);
+        q[c] = u;
+      }
     } else {
       float4* q = reinterpret_cast<float4*>(reinterpret_cast<float*>(p) + i0);
 #pragma unroll
@@ -175,6 +217,11 @@ __device__ __forceinline__ void st32(void* p, int dt, int64_t i0, int nvalid, bo
 #pragma unroll
       for (int j = 0; j < 32; ++j)
         if (j < nvalid) q[j] = __float2bfloat16_rn(v[j]);
+    } else if (dt == KF_F16) {
+      __half* q = reinterpret_cast<__half*>(p) + i0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nvalid) q[j] = __float2half_rn(v[j]);
     } else {
       float* q = reinterpret_cast<float*>(p) + i0;
 #pragma unroll

@@ -107,6 +107,8 @@ __global__ void lse_combine_kernel(const __grid_constant__ LseCombineParams p) {
     for (int o = 0; o < p.n_post; ++o) v = apply_scalar_op(p.post[o], v);
     if (p.out_dtype == KF_BF16)
       reinterpret_cast<__nv_bfloat16*>(p.out)[row] = __float2bfloat16_rn(v);
+    else if (p.out_dtype == KF_F16)
+      reinterpret_cast<__half*>(p.out)[row] = __float2half_rn(v);
     else
       reinterpret_cast<float*>(p.out)[row] = v;
   }

@@ -420,6 +420,8 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     if (lane == 0 && leader) {
       int32_t it = 0, tl = 0;
       bool ok = true;
+      // operand format of kind::f16: bf16 (as compiled) or fp16 (A and B alike)
+      const uint32_t idesc = p.ab_f16 ? (Cfg::kIdesc & ~((7u << 7) | (7u << 10))) : Cfg::kIdesc;
       for (int32_t u = unit0; ok && u < total; u += unit_step) {
         for (int s = 0; ok && s < sub_tiles; ++s) {
           const int acc = tl & 1;
@@ -443,9 +445,9 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             for (int kk = 0; kk < kBK / 16; ++kk) {
               const uint64_t ad = desc_sw128_kmajor(a0 + kk * 32), bd = desc_sw128_kmajor(b0 + kk * 32);
               if constexpr (CTA2)
-                tc_mma_bf16_pair(d, ad, bd, Cfg::kIdesc, (kb | kk) != 0 ? 1u : 0u);
+                tc_mma_bf16_pair(d, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
               else
-                tc_mma_bf16(d, ad, bd, Cfg::kIdesc, (kb | kk) != 0 ? 1u : 0u);
+                tc_mma_bf16(d, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
             }
             if constexpr (CTA2)
               tc_commit_pair_mc(&empty[st], pair_mask);  // frees the slot in both CTAs

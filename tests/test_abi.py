@@ -182,3 +182,9 @@ def test_moe_add_rmsnorm_argument_errors_before_any_launch():
     assert call(eps=-1.0) == kf.KF_ERR_INVALID_ARG
     assert call(R=None) == kf.KF_ERR_INVALID_ARG
     assert call(R=fake + 4) == kf.KF_ERR_MISALIGNED
+
+
+def test_mixed_f16_bf16_operands_are_refused(L):
+    # one operand format per tcgen05 MMA: fp16 with bf16 is refused before any launch
+    assert fused(L, xt=kf.KF_F16, wt=kf.KF_BF16) == kf.KF_ERR_UNSUPPORTED
+    assert fused(L, xt=kf.KF_BF16, wt=kf.KF_F16) == kf.KF_ERR_UNSUPPORTED
