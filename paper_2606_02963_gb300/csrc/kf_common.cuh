@@ -87,11 +87,19 @@ struct TcParams {
 };
 
 // ---------------------------------------------------------------- loads/stores
-__device__ __forceinline__ float ld_elem(const void* p, int dt, int64_t i) {
-  if (dt == KF_BF16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(p)[i]);
-  if (dt == KF_F16) return __half2float(reinterpret_cast<const __half*>(p)[i]);
-  return reinterpret_cast<const float*>(p)[i];
+// One element's raw bits (a 32-bit load for fp32, a 16-bit load for bf16 / fp16:
+// predicated, no branch) and their conversion, kept apart so that a run of loads
+// issues back to back before any conversion waits on one.
+__device__ __forceinline__ uint32_t ld_raw(const void* p, int dt, int64_t i) {
+  return dt == KF_F32 ? reinterpret_cast<const uint32_t*>(p)[i]
+                      : static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(p)[i]);
 }
+__device__ __forceinline__ float cvt_raw(uint32_t b, int dt) {
+  if (dt == KF_F32) return __uint_as_float(b);
+  if (dt == KF_BF16) return __uint_as_float(b << 16);
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(b)));
+}
+__device__ __forceinline__ float ld_elem(const void* p, int dt, int64_t i) { return cvt_raw(ld_raw(p, dt, i), dt); }
 __device__ __forceinline__ float2 f16x2_to_f2(uint32_t w) {
   return __half22float2(*reinterpret_cast<const __half2*>(&w));
 }

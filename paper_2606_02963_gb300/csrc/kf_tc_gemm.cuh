@@ -785,24 +785,26 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
         // the vectors of the warp's 4 chunks c0, c0 + step, ... (lane j = column j
         // of each chunk) are loaded into registers first, all at once, and
         // parked in the cache later: one memory round trip instead of twelve
-        float vb[4], vg[4], vt[4];
+        // (raw bits: the conversions wait for the loads only in park_vecs)
+        uint32_t vb[4], vg[4], vt[4];
         auto issue_vecs = [&](int32_t colbase, int c0, int c1, int step) {
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             const int c = c0 + i * step;
             const int32_t col = colbase + c * 32 + lane;
             const bool in = c < c1;
-            vb[i] = (in && pre_bias) ? ld_elem(p.pre[0].p0, p.pre[0].p_dtype, col) : 0.0f;
-            vg[i] = (in && p.norm.p0) ? ld_elem(p.norm.p0, p.norm.p_dtype, col) : 1.0f;
-            vt[i] = (in && p.norm.p1) ? ld_elem(p.norm.p1, p.norm.p_dtype, col) : 0.0f;
+            vb[i] = (in && pre_bias) ? ld_raw(p.pre[0].p0, p.pre[0].p_dtype, col) : 0u;
+            vg[i] = (in && p.norm.p0) ? ld_raw(p.norm.p0, p.norm.p_dtype, col) : 0u;
+            vt[i] = (in && p.norm.p1) ? ld_raw(p.norm.p1, p.norm.p_dtype, col) : 0u;
           }
         };
         auto park_vecs = [&]() {
+          const int bdt = pre_bias ? p.pre[0].p_dtype : KF_F32, ndt = p.norm.p_dtype;
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            gcache[i * 32 + lane] = vb[i];
-            gcache[(4 + i) * 32 + lane] = vg[i];
-            gcache[(8 + i) * 32 + lane] = vt[i];
+            gcache[i * 32 + lane] = pre_bias ? cvt_raw(vb[i], bdt) : 0.0f;
+            gcache[(4 + i) * 32 + lane] = p.norm.p0 ? cvt_raw(vg[i], ndt) : 1.0f;
+            gcache[(8 + i) * 32 + lane] = p.norm.p1 ? cvt_raw(vt[i], ndt) : 0.0f;
           }
           __syncwarp();
         };
