@@ -26,7 +26,16 @@
  *     block) is the residual add and RMS normalisation of the new residual
  *     stream: R_out = bf16(R + Y), normed_j = R_out_j / sqrt(mean(R_out^2) + eps)
  *     * gamma_j -- the norm reads the stored (bf16) residual, as the next layer
- *     would.
+ *     would;
+ *   - the attention input projection with its tail (the Bias + RoPE + KV update
+ *     kernel of the gpt-oss decode path, Sec. IV-A and Table 1, here as the tail
+ *     of the QKV GEMM; the paper gives no formula, this is the standard
+ *     half-split rotary embedding) is
+ *     s = X W^T + b split into nq query, nkv key and nkv value heads of d columns;
+ *     query and key heads are rotated pairwise, (s_i, s_{i+d/2}) ->
+ *     (s_i c - s_{i+d/2} v, s_{i+d/2} c + s_i v) with c = cos[pos][i],
+ *     v = sin[pos][i] from the caller's tables; queries go to q_out[t], keys and
+ *     values to row cache_rows[t] of the key / value caches.
  *
  * Threads (pthreads) split independent rows / tokens; each row is computed by
  * one thread in a fixed order, so results do not depend on the thread count.
@@ -425,6 +434,46 @@ int orc_add_rmsnorm(const double *Y, const void *R, int rt, const void *gamma, i
     const double inv = 1.0 / sqrt(ss / (double)H + eps);
     for (int64_t j = 0; j < H; ++j) normed[t * H + j] = R_out[t * H + j] * inv * orc_load(gamma, gt, j);
   }
+  return 0;
+}
+
+/* Bias + RoPE + KV-cache update of the QKV projection (see the header).  X bf16
+ * [T x H], W bf16 [(nq + 2 nkv) d x H], bias bf16 [(nq + 2 nkv) d] or NULL,
+ * positions / cache_rows int32 [T], cos / sin fp32 [max_pos x d/2]; q_out
+ * double [T x nq d]; k_cache / v_cache double [rows x nkv d] (only the rows
+ * named by cache_rows are written). */
+int orc_qkv_rope_kv(const uint16_t *X, const uint16_t *W, const uint16_t *bias, const int32_t *positions,
+                    const int32_t *cache_rows, const float *cos_t, const float *sin_t, int64_t max_pos, int64_t T,
+                    int64_t H, int32_t nq, int32_t nkv, int32_t d, int64_t rows, double *q_out, double *k_cache,
+                    double *v_cache) {
+  if (T < 0 || H < 1 || nq < 1 || nkv < 1 || d < 2 || d % 2) return 1;
+  const int64_t N = (int64_t)(nq + 2 * nkv) * d, half = d / 2;
+  double *s = (double *)malloc(sizeof(double) * (size_t)N);
+  if (!s) return 2;
+  for (int64_t t = 0; t < T; ++t) {
+    const int32_t pos = positions[t], row = cache_rows[t];
+    if (pos < 0 || pos >= max_pos || row < 0 || row >= rows) { free(s); return 3; }
+    for (int64_t n = 0; n < N; ++n) {
+      double acc = bias ? orc_load(bias, ORC_BF16, n) : 0.0;
+      for (int64_t k = 0; k < H; ++k) acc += orc_load(X, ORC_BF16, t * H + k) * orc_load(W, ORC_BF16, n * H + k);
+      s[n] = acc;
+    }
+    for (int32_t hd = 0; hd < nq + 2 * nkv; ++hd) {
+      double *h = s + (int64_t)hd * d;
+      if (hd < nq + nkv) /* query and key heads: rotate the pairs */
+        for (int64_t i = 0; i < half; ++i) {
+          const double c = (double)cos_t[pos * half + i], v = (double)sin_t[pos * half + i];
+          const double a = h[i], b = h[i + half];
+          h[i] = a * c - b * v;
+          h[i + half] = b * c + a * v;
+        }
+      double *dst = hd < nq ? q_out + t * (int64_t)nq * d + (int64_t)hd * d
+                  : hd < nq + nkv ? k_cache + (int64_t)row * nkv * d + (int64_t)(hd - nq) * d
+                                  : v_cache + (int64_t)row * nkv * d + (int64_t)(hd - nq - nkv) * d;
+      for (int32_t i = 0; i < d; ++i) dst[i] = h[i];
+    }
+  }
+  free(s);
   return 0;
 }
 

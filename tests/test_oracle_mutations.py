@@ -31,6 +31,12 @@ MUTATIONS = {
                                    "const double h = orc_load(R, rt, t * H + j) + Y[t * H + j];"),
     "f16_exponent_bias": ("v = ldexp((double)(1024 + fr), ex - 25);", "v = ldexp((double)(1024 + fr), ex - 24);"),
     "f16_subnormal_scale": ("v = ldexp((double)fr, -24);", "v = ldexp((double)fr, -25);"),
+    "rope_sin_sign": ("h[i] = a * c - b * v;", "h[i] = a * c + b * v;"),
+    "rope_keys_unrotated": ("if (hd < nq + nkv) /* query and key heads", "if (hd < nq) /* query and key heads"),
+    "rope_values_rotated": ("if (hd < nq + nkv) /* query and key heads", "if (hd < nq + 2 * nkv) /* query and key heads"),
+    "rope_token_not_position": ("(double)cos_t[pos * half + i]", "(double)cos_t[t * half + i]"),
+    "rope_adjacent_partner": ("const double a = h[i], b = h[i + half];", "const double a = h[i], b = h[i ^ 1];"),
+    "kv_row_is_token": ("k_cache + (int64_t)row * nkv * d", "k_cache + t * nkv * d"),
     "residual_dropped": ("case ORC_RESIDUAL_ADD: return v + orc_load", "case ORC_RESIDUAL_ADD: return v + 0 * orc_load"),
 }
 

@@ -404,3 +404,104 @@ def test_f16_operands_read_exactly():
     W = torch.from_numpy(v.copy()).reshape(-1, 1)
     Y = oracle.fused_gemm(X, W, [])
     assert np.array_equal(Y[0], v.astype(np.float64))
+
+
+# ---- QKV projection tail: bias, rotary embedding of query / key heads, cache rows
+def _qkv_case(seed, T=5, H=24, nq=3, nkv=2, d=8, max_pos=16, rows=12):
+    g = torch.Generator().manual_seed(seed)
+    N = (nq + 2 * nkv) * d
+    # small integers: every product and sum is exact in fp64
+    X = torch.randint(-4, 5, (T, H), generator=g).to(torch.bfloat16)
+    W = torch.randint(-4, 5, (N, H), generator=g).to(torch.bfloat16)
+    b = torch.randint(-8, 9, (N,), generator=g).to(torch.bfloat16)
+    pos = torch.randperm(max_pos, generator=g)[:T].to(torch.int32)      # positions != token index
+    crow = torch.randperm(rows, generator=g)[:T].to(torch.int32)        # distinct cache rows
+    s = X.double().numpy() @ W.double().numpy().T + b.double().numpy()
+    return X, W, b, pos, crow, s, dict(nq=nq, nkv=nkv, d=d, rows=rows, max_pos=max_pos)
+
+
+def test_qkv_identity_tables_route_plain_projection():
+    X, W, b, pos, crow, s, c = _qkv_case(41)
+    nq, nkv, d, half = c["nq"], c["nkv"], c["d"], c["d"] // 2
+    cos_t = torch.ones(c["max_pos"], half)
+    sin_t = torch.zeros(c["max_pos"], half)
+    k0 = np.arange(c["rows"] * nkv * d, dtype=np.float64).reshape(c["rows"], nkv * d)
+    q, kc, vc = oracle.qkv_rope_kv(X, W, b, pos, crow, cos_t, sin_t, nq, nkv, d, c["rows"], k_cache=k0, v_cache=-k0)
+    assert np.array_equal(q, s[:, :nq * d])
+    assert np.array_equal(kc[crow.numpy()], s[:, nq * d:(nq + nkv) * d])
+    assert np.array_equal(vc[crow.numpy()], s[:, (nq + nkv) * d:])
+    untouched = np.setdiff1d(np.arange(c["rows"]), crow.numpy())
+    assert np.array_equal(kc[untouched], k0[untouched]) and np.array_equal(vc[untouched], -k0[untouched])
+    # no bias: the projection alone
+    q0, _, _ = oracle.qkv_rope_kv(X, W, None, pos, crow, cos_t, sin_t, nq, nkv, d, c["rows"])
+    assert np.array_equal(q0, s[:, :nq * d] - b.double().numpy()[:nq * d])
+
+
+def test_qkv_rotation_is_complex_multiplication():
+    # the pair (s_i, s_{i+d/2}) as the complex number s_i + j s_{i+d/2}, turned by
+    # the angle theta[pos, i]: numpy's complex product, not the oracle's formula
+    X, W, b, pos, crow, s, c = _qkv_case(42, d=16)
+    nq, nkv, d, half = c["nq"], c["nkv"], c["d"], c["d"] // 2
+    g = torch.Generator().manual_seed(43)
+    theta = (torch.rand(c["max_pos"], half, generator=g, dtype=torch.float64) * 12.0 - 6.0)
+    cos_t, sin_t = torch.cos(theta).float(), torch.sin(theta).float()
+    q, kc, vc = oracle.qkv_rope_kv(X, W, b, pos, crow, cos_t, sin_t, nq, nkv, d, c["rows"])
+    rot = cos_t.double().numpy() + 1j * sin_t.double().numpy()  # the stored fp32 pair
+    heads = s.reshape(s.shape[0], nq + 2 * nkv, d)
+    z = heads[:, :nq + nkv, :half] + 1j * heads[:, :nq + nkv, half:]
+    z = z * rot[pos.numpy()][:, None, :]
+    ref = np.concatenate([z.real, z.imag], axis=2)
+    assert np.allclose(q.reshape(-1, nq, d), ref[:, :nq], rtol=1e-12, atol=1e-9)
+    assert np.allclose(kc[crow.numpy()].reshape(-1, nkv, d), ref[:, nq:], rtol=1e-12, atol=1e-9)
+    assert np.array_equal(vc[crow.numpy()], s[:, (nq + nkv) * d:])  # value heads are not rotated
+    # a rotation keeps each pair's length
+    assert np.allclose(np.abs(z), np.abs(heads[:, :nq + nkv, :half] + 1j * heads[:, :nq + nkv, half:]), rtol=1e-6)
+
+
+def test_qkv_quarter_turn_swaps_halves():
+    # cos = 0, sin = 1: (a, b) -> (-b, a) for every pair of a query or key head
+    X, W, b, pos, crow, s, c = _qkv_case(44)
+    nq, nkv, d, half = c["nq"], c["nkv"], c["d"], c["d"] // 2
+    q, kc, _ = oracle.qkv_rope_kv(X, W, b, pos, crow, torch.zeros(c["max_pos"], half),
+                                  torch.ones(c["max_pos"], half), nq, nkv, d, c["rows"])
+    heads = s.reshape(s.shape[0], nq + 2 * nkv, d)
+    ref = np.concatenate([-heads[:, :, half:], heads[:, :, :half]], axis=2)
+    assert np.array_equal(q.reshape(-1, nq, d), ref[:, :nq])
+    assert np.array_equal(kc[crow.numpy()].reshape(-1, nkv, d), ref[:, nq:nq + nkv])
+
+
+def test_qkv_scores_depend_on_relative_position():
+    # with tables cos / sin(p * w_i), a query at position m and a key at position
+    # n score q . k as a function of m - n only (the point of the embedding)
+    T, H, d = 2, 16, 8
+    half = d // 2
+    g = torch.Generator().manual_seed(45)
+    X = torch.randint(-4, 5, (T, H), generator=g).to(torch.bfloat16)
+    W = torch.randint(-4, 5, (3 * d, H), generator=g).to(torch.bfloat16)
+    P = 40
+    w = 10000.0 ** (-np.arange(half) / half)
+    ang = np.arange(P)[:, None] * w[None, :]
+    cos_t = torch.from_numpy(np.cos(ang)).float()
+    sin_t = torch.from_numpy(np.sin(ang)).float()
+
+    def score(m, n):
+        q, kc, _ = oracle.qkv_rope_kv(X, W, None, [m, n], [0, 1], cos_t, sin_t, 1, 1, d, 2)
+        return float(q[0] @ kc[1])
+
+    for m, n, sh in [(3, 1, 7), (10, 20, 5), (0, 0, 31)]:
+        assert math.isclose(score(m, n), score(m + sh, n + sh), rel_tol=1e-5, abs_tol=1e-4)
+    assert not math.isclose(score(3, 1), score(4, 1), rel_tol=1e-3)
+
+
+def test_qkv_rejects_out_of_range_position_or_row():
+    X, W, b, pos, crow, s, c = _qkv_case(46)
+    half = c["d"] // 2
+    cs = torch.ones(c["max_pos"], half), torch.zeros(c["max_pos"], half)
+    bad = pos.clone()
+    bad[2] = c["max_pos"]
+    with pytest.raises(ValueError):
+        oracle.qkv_rope_kv(X, W, b, bad, crow, *cs, c["nq"], c["nkv"], c["d"], c["rows"])
+    badr = crow.clone()
+    badr[0] = -1
+    with pytest.raises(ValueError):
+        oracle.qkv_rope_kv(X, W, b, pos, badr, *cs, c["nq"], c["nkv"], c["d"], c["rows"])
