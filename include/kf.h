@@ -220,6 +220,41 @@ kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void*
                                  size_t workspace_bytes, int32_t* topk_ids_out, float* topk_w_out, void* stream);
 
 /*
+ * kf_qkv_rope_kv -- the attention input projection with its tail fused into the
+ *                   GEMM's epilogue (Sec. IV-A and Table 1: the gpt-oss decode
+ *                   kernel "Bias + RoPE + KV update"; here it runs on the
+ *                   projection's accumulator instead of a second pass)
+ *
+ *   s[t,:] = X[t,:] W^T + bias, N = (nq + 2 nkv) d columns: nq query heads, then
+ *   nkv key heads, then nkv value heads of d columns each.  Query and key heads
+ *   are rotated by the half-split rotary embedding of token t's position p_t:
+ *     (s_i, s_{i+d/2}) -> (s_i c - s_{i+d/2} v, s_{i+d/2} c + s_i v),
+ *     c = cos_t[p_t][i], v = sin_t[p_t][i], i < d/2
+ *   (any frequency scaling lives in the caller's tables).  Queries go to
+ *   q_out[t,:] (nq d columns); keys and values to row cache_rows[t] of k_cache /
+ *   v_cache (nkv d columns each).  Only the named cache rows are written; two
+ *   tokens naming one row leave either token's values there.
+ *   X, W: both bf16 or both fp16 (KF_BF16 / KF_F16 in xw_dtype), X [T x H] row
+ *     stride ldx, W [N x H] row stride ldw (K-major), 16-byte aligned, ldx and
+ *     ldw multiples of 8 (KF_ERR_MISALIGNED otherwise).
+ *   bias: [N] of bias_dtype (KF_BF16, KF_F16 or KF_F32), or NULL.
+ *   positions, cache_rows: int32 [T] on the device.  A position outside
+ *     [0, max_pos) or a cache row outside [0, cache_rows_n) skips that token's
+ *     writes and sets the bounds bit of the device error word
+ *     (kf_get_device_error).
+ *   cos_t, sin_t: fp32 [max_pos x d/2], row stride d/2, 16-byte aligned.
+ *   q_out [T x ldq], k_cache / v_cache [cache_rows_n x ld_cache]: out_dtype
+ *     (KF_BF16, KF_F16 or KF_F32); ldq >= nq d, ld_cache >= nkv d.
+ *   d: a multiple of 64, at most 256 (KF_ERR_UNSUPPORTED otherwise); nq, nkv >= 1.
+ *   T = 0 writes nothing.  All buffers are the caller's; nothing is allocated.
+ */
+kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dtype, int64_t ldx, int64_t ldw, const void* bias,
+                         int32_t bias_dtype, const int32_t* positions, const int32_t* cache_rows, const float* cos_t,
+                         const float* sin_t, int64_t max_pos, int64_t T, int64_t H, int32_t nq, int32_t nkv,
+                         int32_t d, void* q_out, int64_t ldq, void* k_cache, void* v_cache, int64_t ld_cache,
+                         int64_t cache_rows_n, int32_t out_dtype, void* stream);
+
+/*
  * kf_fused_gemm_lse_noalloc -- kf_fused_gemm for row log-sum-exp chains, without
  * a workspace argument.  The paper has no counterpart: this entry point exists for
  * callers that cannot allocate device memory -- e.g. code hosted by another

@@ -20,7 +20,7 @@ from typing import Callable, Dict, List, Optional, Tuple
 
 import torch
 
-__all__ = ["Workload", "WORKLOADS", "generate", "chain_spec", "moe_generate", "MOE_SHAPE"]
+__all__ = ["Workload", "WORKLOADS", "generate", "chain_spec", "moe_generate", "MOE_SHAPE", "qkv_generate", "QKV_SHAPE"]
 
 
 @dataclass(frozen=True)
@@ -168,3 +168,39 @@ def moe_generate(T: int, seed: int = 0, H: int = 2880, I: int = 2880, E: int = 3
         W_gu = (torch.randn(E, 2 * I, H, generator=gd, device=device) * w_std).to(torch.bfloat16)
         W_down = (torch.randn(E, H, I, generator=gd, device=device) * w_std).to(torch.bfloat16)
     return dict(X=X, logits=logits, W_gu=W_gu, W_down=W_down)
+
+
+QKV_SHAPE = dict(H=2880, nq=64, nkv=8, d=64)  # gpt-oss-20b attention input projection
+
+
+def qkv_generate(T: int, seed: int = 0, H: int = 2880, nq: int = 64, nkv: int = 8, d: int = 64,
+                 max_pos: int = 4096, cache_rows: Optional[int] = None, prefill: bool = False,
+                 theta: float = 150000.0, w_std: float = 0.02, dtype: str = "bf16") -> Dict[str, torch.Tensor]:
+    """Inputs of the QKV projection tail: X[T,H] ~ N(0,1); W[(nq+2nkv)d, H] ~
+    N(0, w_std); bias ~ N(0, 0.1); fp32 rotary tables cos / sin(p * theta^(-2i/d))
+    for p < max_pos, i < d/2 (the caller's tables; any frequency scaling would
+    live here).  Decode (default): T sequences, each adding one token at a random
+    position, into distinct random rows of a cache of ``cache_rows`` rows
+    (default max(4096, 2T)).  Prefill: one sequence, positions 0..T-1, cache rows
+    r0..r0+T-1."""
+    g = torch.Generator("cpu").manual_seed(seed)
+    N = (nq + 2 * nkv) * d
+    rows = cache_rows if cache_rows is not None else max(4096, 2 * T)
+    X = _round(torch.randn(T, H, generator=g, dtype=torch.float32), dtype)
+    W = _round(torch.randn(N, H, generator=g, dtype=torch.float32) * w_std, dtype)
+    b = _round(torch.randn(N, generator=g, dtype=torch.float32) * 0.1, dtype)
+    if prefill:
+        if T > max_pos or T > rows:
+            raise ValueError("prefill longer than the tables or the cache")
+        positions = torch.arange(T, dtype=torch.int32)
+        r0 = int(torch.randint(0, rows - T + 1, (1,), generator=g))
+        crow = torch.arange(r0, r0 + T, dtype=torch.int32)
+    else:
+        if T > rows:
+            raise ValueError("more tokens than cache rows")
+        positions = torch.randint(0, max_pos, (T,), generator=g, dtype=torch.int32)
+        crow = torch.randperm(rows, generator=g)[:T].to(torch.int32)
+    inv = theta ** (-torch.arange(0, d // 2, dtype=torch.float64) * 2.0 / d)
+    ang = torch.arange(max_pos, dtype=torch.float64)[:, None] * inv[None, :]
+    return dict(X=X, W=W, b=b, positions=positions, cache_rows=crow, cos=torch.cos(ang).float(),
+                sin=torch.sin(ang).float(), rows=torch.tensor(rows))

@@ -89,7 +89,8 @@ def _load():
             lib.orc_grouped_gemm.restype = ctypes.c_int
             lib.orc_add_rmsnorm.argtypes = [P, P, ctypes.c_int, P, ctypes.c_int, D, I64, I64, P, P]
             lib.orc_add_rmsnorm.restype = ctypes.c_int
-            lib.orc_qkv_rope_kv.argtypes = [P, P, P, P, P, P, P, I64, I64, I64, I32, I32, I32, I64, P, P, P]
+            lib.orc_qkv_rope_kv.argtypes = [P, P, ctypes.c_int, P, ctypes.c_int, P, P, P, P, I64, I64, I64, I32, I32,
+                                            I32, I64, P, P, P]
             lib.orc_qkv_rope_kv.restype = ctypes.c_int
             lib.orc_round_bf16.argtypes = [D]
             lib.orc_round_bf16.restype = D
@@ -267,7 +268,7 @@ def add_rmsnorm(Y, R, gamma, eps: float) -> Tuple[np.ndarray, np.ndarray]:
 def qkv_rope_kv(X, W, bias, positions, cache_rows, cos_t, sin_t, nq: int, nkv: int, d: int, rows: int,
                 k_cache=None, v_cache=None):
     """Bias + RoPE + KV-cache update of the QKV projection (Sec. IV-A) in fp64.
-    X bf16 [T, H]; W bf16 [(nq + 2 nkv) d, H]; bias bf16 or None; positions and
+    X [T, H] and W [(nq + 2 nkv) d, H] of one dtype; bias or None; positions and
     cache_rows int32 [T]; cos_t / sin_t fp32 [max_pos, d/2].  Returns (q_out
     [T, nq d], k_cache [rows, nkv d], v_cache [rows, nkv d]) as float64; the
     caches start from the given arrays (NaN when None) and only the rows named
@@ -275,13 +276,9 @@ def qkv_rope_kv(X, W, bias, positions, cache_rows, cos_t, sin_t, nq: int, nkv: i
     lib = _load()
     x, xt = _np(X)
     w, wt = _np(W)
-    if xt != ORC_BF16 or wt != ORC_BF16:
-        raise TypeError("qkv_rope_kv: X and W must be bf16")
-    b = None
-    if bias is not None:
-        b, bt = _np(bias)
-        if bt != ORC_BF16:
-            raise TypeError("qkv_rope_kv: bias must be bf16")
+    if xt != wt:
+        raise TypeError("qkv_rope_kv: X and W must share one dtype")
+    b, bt = (None, 0) if bias is None else _np(bias)
     T, H = x.shape
     pos = np.ascontiguousarray(np.asarray(positions, dtype=np.int32))
     crow = np.ascontiguousarray(np.asarray(cache_rows, dtype=np.int32))
@@ -291,7 +288,7 @@ def qkv_rope_kv(X, W, bias, positions, cache_rows, cos_t, sin_t, nq: int, nkv: i
     q = np.zeros((T, nq * d), np.float64)
     kc = np.full((rows, nkv * d), np.nan) if k_cache is None else np.array(k_cache, dtype=np.float64, copy=True)
     vc = np.full((rows, nkv * d), np.nan) if v_cache is None else np.array(v_cache, dtype=np.float64, copy=True)
-    st = lib.orc_qkv_rope_kv(_ptr(x), _ptr(w), None if b is None else _ptr(b), _ptr(pos), _ptr(crow), _ptr(c),
+    st = lib.orc_qkv_rope_kv(_ptr(x), _ptr(w), xt, None if b is None else _ptr(b), bt, _ptr(pos), _ptr(crow), _ptr(c),
                              _ptr(sn), max_pos, T, H, nq, nkv, d, rows, _ptr(q), _ptr(kc), _ptr(vc))
     if st != 0:
         raise ValueError(f"orc_qkv_rope_kv: status {st}")

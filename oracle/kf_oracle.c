@@ -437,12 +437,13 @@ int orc_add_rmsnorm(const double *Y, const void *R, int rt, const void *gamma, i
   return 0;
 }
 
-/* Bias + RoPE + KV-cache update of the QKV projection (see the header).  X bf16
- * [T x H], W bf16 [(nq + 2 nkv) d x H], bias bf16 [(nq + 2 nkv) d] or NULL,
+/* Bias + RoPE + KV-cache update of the QKV projection (see the header).  X
+ * [T x H], W [(nq + 2 nkv) d x H], bias [(nq + 2 nkv) d] or NULL,
  * positions / cache_rows int32 [T], cos / sin fp32 [max_pos x d/2]; q_out
  * double [T x nq d]; k_cache / v_cache double [rows x nkv d] (only the rows
- * named by cache_rows are written). */
-int orc_qkv_rope_kv(const uint16_t *X, const uint16_t *W, const uint16_t *bias, const int32_t *positions,
+ * named by cache_rows are written).  xt: element type of X and W, bt: of the
+ * bias (ORC_BF16 / ORC_F16 / ORC_F32 codes). */
+int orc_qkv_rope_kv(const void *X, const void *W, int xt, const void *bias, int bt, const int32_t *positions,
                     const int32_t *cache_rows, const float *cos_t, const float *sin_t, int64_t max_pos, int64_t T,
                     int64_t H, int32_t nq, int32_t nkv, int32_t d, int64_t rows, double *q_out, double *k_cache,
                     double *v_cache) {
@@ -454,8 +455,8 @@ int orc_qkv_rope_kv(const uint16_t *X, const uint16_t *W, const uint16_t *bias, 
     const int32_t pos = positions[t], row = cache_rows[t];
     if (pos < 0 || pos >= max_pos || row < 0 || row >= rows) { free(s); return 3; }
     for (int64_t n = 0; n < N; ++n) {
-      double acc = bias ? orc_load(bias, ORC_BF16, n) : 0.0;
-      for (int64_t k = 0; k < H; ++k) acc += orc_load(X, ORC_BF16, t * H + k) * orc_load(W, ORC_BF16, n * H + k);
+      double acc = bias ? orc_load(bias, bt, n) : 0.0;
+      for (int64_t k = 0; k < H; ++k) acc += orc_load(X, xt, t * H + k) * orc_load(W, xt, n * H + k);
       s[n] = acc;
     }
     for (int32_t hd = 0; hd < nq + 2 * nkv; ++hd) {

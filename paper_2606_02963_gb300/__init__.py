@@ -36,6 +36,7 @@ ABI_SYMBOLS = (
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
     "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex", "kf_moe_ffn_add_rmsnorm",
+    "kf_qkv_rope_kv",
 )
 
 
@@ -84,6 +85,9 @@ def lib() -> ctypes.CDLL:
     L.kf_moe_ffn_add_rmsnorm.argtypes = [P, P, P, P, P, P, ctypes.c_float, P, P, I64, I64, I64, I32, I32,
                                          ctypes.c_uint32, P, SZ, P, P, P]
     L.kf_moe_ffn_add_rmsnorm.restype = I32
+    L.kf_qkv_rope_kv.argtypes = [P, P, I32, I64, I64, P, I32, P, P, P, P, I64, I64, I64, I32, I32, I32, P, I64,
+                                 P, P, I64, I64, I32, P]
+    L.kf_qkv_rope_kv.restype = I32
     L.kf_moe_ffn_workspace_ex.argtypes = [I64, I64, I64, I32, I32, ctypes.c_uint32]
     L.kf_moe_ffn_workspace_ex.restype = SZ
     L.kf_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
@@ -302,6 +306,40 @@ def moe_ffn_add_rmsnorm(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tenso
                                   _ptr(ws), ws_bytes, None, None, _stream(stream))
     _check(st, "kf_moe_ffn_add_rmsnorm")
     return out, r_out
+
+
+def qkv_rope_kv(X: torch.Tensor, W: torch.Tensor, bias: Optional[torch.Tensor], positions: torch.Tensor,
+                cache_rows: torch.Tensor, cos_t: torch.Tensor, sin_t: torch.Tensor, nq: int, nkv: int, d: int,
+                k_cache: torch.Tensor, v_cache: torch.Tensor, q_out: Optional[torch.Tensor] = None,
+                stream=None) -> torch.Tensor:
+    """QKV projection with bias, rotary embedding and key / value cache write
+    (kf_qkv_rope_kv).  Writes rows ``cache_rows`` of ``k_cache`` / ``v_cache``
+    ([rows, nkv d], their dtype is the output dtype) and returns the rotated
+    queries [T, nq d]."""
+    T, H = X.shape
+    if q_out is None:
+        q_out = torch.empty(T, nq * d, dtype=k_cache.dtype, device=X.device)
+    if k_cache.dtype != v_cache.dtype or q_out.dtype != k_cache.dtype:
+        raise TypeError("q_out, k_cache and v_cache must share one dtype")
+    if k_cache.stride() != v_cache.stride() or k_cache.shape[0] != v_cache.shape[0]:
+        raise ValueError("k_cache and v_cache must have one shape and row stride")
+    for t, nm in ((positions, "positions"), (cache_rows, "cache_rows")):
+        if t.dtype != torch.int32 or not t.is_contiguous() or t.numel() != T:
+            raise ValueError(f"{nm} must be contiguous int32 [T]")
+    for t, nm in ((cos_t, "cos_t"), (sin_t, "sin_t")):
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.shape[1] != d // 2:
+            raise ValueError(f"{nm} must be contiguous fp32 [max_pos, d/2]")
+    if bias is not None and not bias.is_contiguous():
+        raise ValueError("bias must be contiguous")
+    if _dt(X) != _dt(W):
+        raise TypeError("X and W must share one dtype")
+    st = lib().kf_qkv_rope_kv(X.data_ptr(), W.data_ptr(), _dt(X), _rows(X, "X"), _rows(W, "W"), _ptr(bias),
+                              _dt(bias) if bias is not None else KF_BF16, positions.data_ptr(), cache_rows.data_ptr(),
+                              cos_t.data_ptr(), sin_t.data_ptr(), cos_t.shape[0], T, H, nq, nkv, d,
+                              q_out.data_ptr(), _rows(q_out, "q_out"), k_cache.data_ptr(), v_cache.data_ptr(),
+                              _rows(k_cache, "k_cache"), k_cache.shape[0], _dt(k_cache), _stream(stream))
+    _check(st, "kf_qkv_rope_kv")
+    return q_out
 
 
 def get_device_error(stream=None) -> Tuple[int, int]:

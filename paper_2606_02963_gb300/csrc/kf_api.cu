@@ -923,3 +923,111 @@ extern "C" kf_status kf_fused_gemm_lse_noalloc(const void* X, int32_t xt, int64_
   if (st != KF_OK) return st;
   return kf_fused_gemm(X, xt, ldx, W, wt, ldw, Y, yt, 1, M, N, K, epi, scratch, kf::kNoAllocScratchBytes, stream);
 }
+
+namespace kf {
+namespace {
+
+// Tile width of the QKV projection: whole heads per tile (a multiple of d),
+// then the fewest tile-widths on the busiest SM (or CTA pair) + a fixed cost
+// per tile, as for the dense store variants.
+int pick_rope_bn(int64_t M, int64_t N, int d, int nsm, bool cta2) {
+  static const int cand[] = {256, 128, 64};
+  int best = 0;
+  int64_t best_cost = INT64_MAX;
+  const int64_t rows = cta2 ? 2 * kBM : kBM;
+  const int64_t workers = cta2 ? nsm / 2 : nsm;
+  const int64_t tm = (M + rows - 1) / rows;
+  for (int bn : cand) {
+    if (bn % d != 0 || !tc_rope_has(bn, cta2)) continue;
+    const int64_t tiles = tm * ((N + bn - 1) / bn);
+    const int64_t cost = ((tiles + workers - 1) / workers) * (bn + 48);
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
+}
+
+}  // namespace
+}  // namespace kf
+
+extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dtype, int64_t ldx, int64_t ldw,
+                                    const void* bias, int32_t bias_dtype, const int32_t* positions,
+                                    const int32_t* cache_rows, const float* cos_t, const float* sin_t,
+                                    int64_t max_pos, int64_t T, int64_t H, int32_t nq, int32_t nkv, int32_t d,
+                                    void* q_out, int64_t ldq, void* k_cache, void* v_cache, int64_t ld_cache,
+                                    int64_t cache_rows_n, int32_t out_dtype, void* stream) {
+  using namespace kf;
+  if (T < 0 || H < 1 || nq < 1 || nkv < 1 || d < 1 || max_pos < 1 || cache_rows_n < 1) return KF_ERR_INVALID_ARG;
+  if (T > INT32_MAX || H > INT32_MAX || max_pos > INT32_MAX || cache_rows_n > INT32_MAX) return KF_ERR_INVALID_ARG;
+  if (d % 64 != 0 || d > 256) return KF_ERR_UNSUPPORTED;
+  const int64_t N = (static_cast<int64_t>(nq) + 2 * static_cast<int64_t>(nkv)) * d;
+  if (N > INT32_MAX) return KF_ERR_INVALID_ARG;
+  if (xw_dtype != KF_BF16 && xw_dtype != KF_F16) return KF_ERR_UNSUPPORTED;
+  if (!float_dtype(out_dtype) || (bias && !float_dtype(bias_dtype))) return KF_ERR_INVALID_ARG;
+  if (ldx < H || ldw < H || ldq < static_cast<int64_t>(nq) * d || ld_cache < static_cast<int64_t>(nkv) * d)
+    return KF_ERR_INVALID_ARG;
+  if (T == 0) return KF_OK;  // nothing to read or write
+  if (!X || !W || !positions || !cache_rows || !cos_t || !sin_t || !q_out || !k_cache || !v_cache)
+    return KF_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(W) || ldx % 8 != 0 || ldw % 8 != 0 || !aligned16(cos_t) || !aligned16(sin_t))
+    return KF_ERR_MISALIGNED;
+  // the bias is the chain before the rotation
+  kf_epilogue_op bop;
+  std::memset(&bop, 0, sizeof(bop));
+  bop.kind = KF_OP_BIAS;
+  bop.p0 = bias;
+  bop.p_dtype = bias_dtype;
+  kf_epilogue epi = {bias ? 1 : 0, &bop};
+  ChainPlan pl;
+  kf_status st = plan_chain(&epi, N, false, &pl);
+  if (st != KF_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DevInfo di;
+  st = device_info(&di);
+  if (st != KF_OK) return st;
+  const bool cta2 = T > kBM && di.nsm >= 2;
+  const int bn = pick_rope_bn(T, N, d, di.nsm, cta2);
+  if (bn == 0) return KF_ERR_UNSUPPORTED;
+  const CUtensorMapDataType op_dt =
+      xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  CUtensorMap ma, mb;
+  st = make_map(&ma, X, H, T, ldx * 2, 1, 0, kBM, 2, op_dt);
+  if (st != KF_OK) return st;
+  st = make_map(&mb, W, H, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, cta2 ? bn / 2 : bn, 3, op_dt);
+  if (st != KF_OK) return st;
+  TcParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.M = static_cast<int32_t>(T);
+  p.N = static_cast<int32_t>(N);
+  p.K = static_cast<int32_t>(H);
+  p.tiles_m = static_cast<int32_t>((T + (cta2 ? 2 * kBM : kBM) - 1) / (cta2 ? 2 * kBM : kBM));
+  p.tiles_n = static_cast<int32_t>((N + bn - 1) / bn);  // whole heads per tile; the last may hold fewer
+  p.num_kb = static_cast<int32_t>((H + kBK - 1) / kBK);
+  p.total_units = p.tiles_m * p.tiles_n;
+  p.C = q_out;
+  p.ldc = ldq;
+  p.c_dtype = out_dtype;
+  p.c_vec_ok = aligned16(q_out) && (ldq * elt_size(out_dtype)) % 16 == 0;
+  fill_params_common(p, pl, di.err);
+  p.res_op = -1;
+  p.vec_op = -1;
+  p.fast = 0;
+  p.ab_f16 = xw_dtype == KF_F16;
+  p.row_dst = cache_rows;
+  p.dst_rows = static_cast<int32_t>(cache_rows_n);
+  p.rope_cos = cos_t;
+  p.rope_sin = sin_t;
+  p.rope_pos = positions;
+  p.rope_max_pos = static_cast<int32_t>(max_pos);
+  p.rope_d = d;
+  p.rope_q_cols = nq * d;
+  p.rope_rot_cols = (nq + nkv) * d;
+  p.k_cache = k_cache;
+  p.v_cache = v_cache;
+  p.ld_cache = ld_cache;
+  p.kv_vec_ok = aligned16(k_cache) && aligned16(v_cache) && (ld_cache * elt_size(out_dtype)) % 16 == 0;
+  const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
+  return cuda_status(tc_rope_launch(bn, cta2, ma, mb, p, grid, s));
+}

@@ -42,6 +42,8 @@ enum TcMode : int {
   kModeGroupNorm = 2,// pre-ops -> GroupNorm -> post-ops -> store
   kModeSwiglu = 3,   // gate/up halves -> silu(g) * u -> post-ops -> store
   kModeScatter = 4,  // chain -> * row scale -> atomic add into C[dst row]
+  kModeRope = 5,     // QKV projection: chain (bias) -> rotary embedding of query / key
+                     // heads -> queries to C[row], keys / values to cache row row_dst[row]
 };
 
 struct TcParams {
@@ -84,6 +86,22 @@ struct TcParams {
   unsigned long long* gx_flag;
   uint32_t gx_epoch;
   int32_t gx_couples;
+  // QKV tail: heads of rope_d columns; columns [0, rope_q_cols) are queries,
+  // [rope_q_cols, rope_rot_cols) keys (both rotated), the rest values.  Row r
+  // turns by the angles of table row rope_pos[r] (cos / sin fp32 [rope_max_pos x
+  // rope_d / 2]); its keys and values go to row row_dst[r] of k_cache / v_cache
+  // (row stride ld_cache, dst_rows rows, element type c_dtype).
+  const float* rope_cos;
+  const float* rope_sin;
+  const int32_t* rope_pos;
+  int32_t rope_max_pos;
+  int32_t rope_d;
+  int32_t rope_q_cols;
+  int32_t rope_rot_cols;
+  void* k_cache;
+  void* v_cache;
+  int64_t ld_cache;
+  int32_t kv_vec_ok;    // caches allow 16-byte stores of 32-column chunks
 };
 
 // ---------------------------------------------------------------- loads/stores

@@ -51,6 +51,10 @@ bool tc_dense_has(int mode, int bn, bool cta2);
 bool tc_dense2_has(int mode, int bn);
 bool tc_dense2_has_prog(int mode, int bn, int sig);  // a compiled chain program for (mode, bn, sig)
 bool tc_grouped_has(int mode, int bn);
+// QKV projection tail (kModeRope): single CTAs or CTA pairs; no output map
+bool tc_rope_has(int bn, bool cta2);
+cudaError_t tc_rope_launch(int bn, bool cta2, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid,
+                           cudaStream_t s);
 // `c` is the output map of the TMA stores, `r` the residual map of the
 // residual-tile variants (unused by the others).
 cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensorMap& a, const CUtensorMap& b,

@@ -100,7 +100,7 @@ struct TcCfg {
   // the asynchronous TMA stores, plus (store mode) one for the residual
   // transposition, which must not reuse a buffer a TMA store may still read
   // (residual tile: 256 B per warp, the bias of its chunks)
-  static constexpr int kWarpStaging = RT ? 256 : ((MODE == kModeStore) ? 3072 : 2048);
+  static constexpr int kWarpStaging = RT ? 256 : (MODE == kModeStore) ? 3072 : (MODE == kModeRope) ? 0 : 2048;
   // residual tile: BN / 32 chunks x 4 row blocks of 32 x 32 bf16 (2 KB, 64-byte
   // swizzle), placed in the A then B regions of two ring slots
   static constexpr int kResTileBytes = 0;
@@ -731,6 +731,75 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
               __threadfence_block();
               mbar_arrive(&empty[rt_s0]);
               mbar_arrive(&empty[rt_s1]);
+            }
+          }
+        }
+        release_acc(tl);
+        ++tl;
+      } else if constexpr (MODE == kModeRope) {
+        // this row's table row and cache row, requested before the wait
+        int32_t pos = 0, crow = 0;
+        if (row_ok) {
+          pos = p.rope_pos[grow];
+          crow = p.row_dst[grow];
+        }
+        if (!wait_acc(tl)) { ok = false; break; }
+        bool wr = row_ok;
+        if (row_ok && (pos < 0 || pos >= p.rope_max_pos || crow < 0 || crow >= p.dst_rows)) {
+          atomicOr(p.err, kErrBounds);
+          wr = false;
+        }
+        const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
+        // rotation pairs: chunk lo of a head's first half with chunk lo + hh of
+        // its second half (hh chunks of 32 columns per half head); the tile
+        // holds whole heads (BN a multiple of rope_d, tiles start on a head)
+        const int hc = p.rope_d >> 5;
+        const int hh = hc >> 1;
+        const int half = p.rope_d >> 1;
+        for (int j = h; j < Cfg::kOutN / 64; j += Cfg::kH) {
+          const int hd_t = j / hh, jj = j - hd_t * hh;
+          const int clo = hd_t * hc + jj;
+          const int32_t col_lo = ui.n0 + clo * 32;
+          if (col_lo >= p.N) break;  // N is whole heads: the partner exists too
+          const int32_t col_hi = col_lo + half;
+          float a[32], b[32];
+          tmem_ld32(tb + clo * 32, a);
+          tmem_ld32(tb + (clo + hh) * 32, b);
+          run_chain<PRE>(fast, p.pre, p.n_pre, a, grow, col_lo, 32, row_ok);
+          run_chain<PRE>(fast, p.pre, p.n_pre, b, grow, col_hi, 32, row_ok);
+          const int32_t hcol = col_lo - (col_lo % p.rope_d);  // first column of the head
+          if (wr && hcol < p.rope_rot_cols) {
+            const float4* cp = reinterpret_cast<const float4*>(p.rope_cos + static_cast<int64_t>(pos) * half + jj * 32);
+            const float4* sp = reinterpret_cast<const float4*>(p.rope_sin + static_cast<int64_t>(pos) * half + jj * 32);
+            float4 c4[8], s4[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              c4[u] = __ldg(cp + u);
+              s4[u] = __ldg(sp + u);
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              const float cc[4] = {c4[u].x, c4[u].y, c4[u].z, c4[u].w};
+              const float ss[4] = {s4[u].x, s4[u].y, s4[u].z, s4[u].w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float x0 = a[4 * u + e], x1 = b[4 * u + e];
+                a[4 * u + e] = fmaf(x0, cc[e], -x1 * ss[e]);
+                b[4 * u + e] = fmaf(x1, cc[e], x0 * ss[e]);
+              }
+            }
+          }
+          if (wr) {
+            if (hcol < p.rope_q_cols) {
+              const int64_t base = static_cast<int64_t>(grow) * p.ldc;
+              st32(p.C, p.c_dtype, base + col_lo, 32, p.c_vec_ok != 0, a);
+              st32(p.C, p.c_dtype, base + col_hi, 32, p.c_vec_ok != 0, b);
+            } else {
+              const bool is_k = hcol < p.rope_rot_cols;
+              void* cache = is_k ? p.k_cache : p.v_cache;
+              const int64_t base = static_cast<int64_t>(crow) * p.ld_cache - (is_k ? p.rope_q_cols : p.rope_rot_cols);
+              st32(cache, p.c_dtype, base + col_lo, 32, p.kv_vec_ok != 0, a);
+              st32(cache, p.c_dtype, base + col_hi, 32, p.kv_vec_ok != 0, b);
             }
           }
         }

@@ -188,3 +188,30 @@ def test_mixed_f16_bf16_operands_are_refused(L):
     # one operand format per tcgen05 MMA: fp16 with bf16 is refused before any launch
     assert fused(L, xt=kf.KF_F16, wt=kf.KF_BF16) == kf.KF_ERR_UNSUPPORTED
     assert fused(L, xt=kf.KF_BF16, wt=kf.KF_F16) == kf.KF_ERR_UNSUPPORTED
+
+
+def test_qkv_rope_kv_argument_errors_before_any_launch(L):
+    fake = 1 << 20  # aligned, never dereferenced: the checks come first
+
+    def call(T=4, H=2880, nq=64, nkv=8, d=64, xw=kf.KF_BF16, out=kf.KF_BF16, ldx=None, ldq=None, ldc=None,
+             X=fake, cos=fake, max_pos=4096, rows=256, bias=None, bdt=kf.KF_BF16, kc=fake):
+        return L.kf_qkv_rope_kv(X, fake, xw, H if ldx is None else ldx, H, bias, bdt, fake, fake, cos, fake,
+                                max_pos, T, H, nq, nkv, d, fake, nq * d if ldq is None else ldq, kc, fake,
+                                nkv * d if ldc is None else ldc, rows, out, None)
+    assert call(d=96) == kf.KF_ERR_UNSUPPORTED          # half a head is not whole 32-column chunks
+    assert call(d=512) == kf.KF_ERR_UNSUPPORTED
+    assert call(xw=kf.KF_F32) == kf.KF_ERR_UNSUPPORTED  # tensor-core operands only
+    assert call(out=kf.KF_I32) == kf.KF_ERR_INVALID_ARG
+    assert call(nkv=0) == kf.KF_ERR_INVALID_ARG
+    assert call(T=-1) == kf.KF_ERR_INVALID_ARG
+    assert call(max_pos=0) == kf.KF_ERR_INVALID_ARG
+    assert call(rows=0) == kf.KF_ERR_INVALID_ARG
+    assert call(ldq=64 * 64 - 8) == kf.KF_ERR_INVALID_ARG
+    assert call(ldc=8 * 64 - 8) == kf.KF_ERR_INVALID_ARG
+    assert call(ldx=2000) == kf.KF_ERR_INVALID_ARG
+    assert call(kc=None) == kf.KF_ERR_INVALID_ARG
+    assert call(X=fake + 2) == kf.KF_ERR_MISALIGNED
+    assert call(ldx=2884) == kf.KF_ERR_MISALIGNED
+    assert call(cos=fake + 4) == kf.KF_ERR_MISALIGNED
+    assert call(bias=fake, bdt=kf.KF_I32) == kf.KF_ERR_INVALID_ARG
+    assert call(T=0, X=None, kc=None) == kf.KF_OK       # empty: nothing read or written

@@ -1,0 +1,135 @@
+"""GPU parity of the QKV projection tail (bias, rotary embedding of query and key
+heads, key / value cache rows; the gpt-oss decode kernel "Bias + RoPE + KV
+update" of Sec. IV-A, here the epilogue of the projection GEMM) against the
+oracle: decode batches (one 128-row tile, narrow tiles), prefill (CTA pairs,
+ragged last row tile), 128-column heads, fp16 operands, fp32 / fp16 outputs,
+no bias, out-of-range positions, untouched cache rows, repeat runs."""
+import numpy as np
+import pytest
+import torch
+
+import kf_workloads
+import oracle
+import paper_2606_02963_gb300 as kf
+from tests._util import check_bf16, check_f32
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+SENT = -7.0  # cache rows no token names keep this value
+
+
+def _run(inp, nq, nkv, d, out_dtype=torch.bfloat16, bias=True, sub=None):
+    """The library's outputs and the oracle's, on the tokens `sub` (all if None)."""
+    rows = int(inp["rows"])
+    kc = torch.full((rows, nkv * d), SENT, dtype=out_dtype, device=DEV)
+    vc = torch.full((rows, nkv * d), SENT, dtype=out_dtype, device=DEV)
+    g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
+    q = kf.qkv_rope_kv(g["X"], g["W"], g["b"] if bias else None, g["positions"], g["cache_rows"], g["cos"],
+                       g["sin"], nq, nkv, d, kc, vc)
+    assert kf.get_device_error()[0] == kf.KF_OK
+    idx = torch.arange(inp["X"].shape[0]) if sub is None else torch.as_tensor(sub)
+    rq, rk, rv = oracle.qkv_rope_kv(inp["X"][idx], inp["W"], inp["b"] if bias else None, inp["positions"][idx],
+                                    inp["cache_rows"][idx], inp["cos"], inp["sin"], nq, nkv, d, rows)
+    return (q, kc, vc), (rq, rk, rv), idx
+
+
+def _check(got, ref, idx, what, out_dtype=torch.bfloat16, all_tokens=True):
+    q, kc, vc = got
+    rq, rk, rv = ref
+    chk = check_f32 if out_dtype == torch.float32 else check_bf16
+    chk(q[idx.to(DEV)], rq, what + " q")
+    named = np.flatnonzero(~np.isnan(rk[:, 0]))
+    chk(kc[torch.as_tensor(named, device=DEV)], rk[named], what + " k")
+    chk(vc[torch.as_tensor(named, device=DEV)], rv[named], what + " v")
+    if all_tokens:
+        other = np.setdiff1d(np.arange(kc.shape[0]), named)
+        if other.size:
+            o = torch.as_tensor(other, device=DEV)
+            assert bool((kc[o] == SENT).all()) and bool((vc[o] == SENT).all()), f"{what}: unnamed rows written"
+
+
+@pytest.mark.parametrize("T", [1, 37, 128])
+def test_decode_gpt_oss_shape(T):
+    s = kf_workloads.QKV_SHAPE
+    inp = kf_workloads.qkv_generate(T, seed=60 + T)
+    got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"])
+    _check(got, ref, idx, f"decode T={T}")
+
+
+@pytest.mark.parametrize("T", [129, 300])
+def test_prefill_ragged_rows_on_cta_pairs(T):
+    s = kf_workloads.QKV_SHAPE
+    inp = kf_workloads.qkv_generate(T, seed=70 + T, H=512, prefill=True, cache_rows=1000)
+    got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"])
+    _check(got, ref, idx, f"prefill T={T}")
+
+
+@pytest.mark.parametrize("T", [50, 200])
+def test_head_dim_128(T):
+    inp = kf_workloads.qkv_generate(T, seed=80 + T, H=256, nq=8, nkv=2, d=128, cache_rows=512)
+    got, ref, idx = _run(inp, 8, 2, 128)
+    _check(got, ref, idx, f"d=128 T={T}")
+
+
+def test_ragged_last_column_tile():
+    # nq + 2 nkv = 7 heads of 64: wide tiles end part-way (whole heads only)
+    T = 300
+    inp = kf_workloads.qkv_generate(T, seed=85, H=192, nq=3, nkv=2, d=64, cache_rows=700)
+    got, ref, idx = _run(inp, 3, 2, 64)
+    _check(got, ref, idx, "7 heads")
+
+
+@pytest.mark.parametrize("out_dtype", [torch.float32, torch.float16])
+def test_fp16_operands_and_wide_outputs(out_dtype):
+    inp = kf_workloads.qkv_generate(64, seed=90, H=640, nq=16, nkv=4, d=64, dtype="f16", cache_rows=300)
+    got, ref, idx = _run(inp, 16, 4, 64, out_dtype=out_dtype)
+    _check(got, ref, idx, f"f16 -> {out_dtype}", out_dtype=out_dtype)
+
+
+def test_no_bias_fp32_output():
+    inp = kf_workloads.qkv_generate(20, seed=91, H=384, nq=4, nkv=1, d=128, cache_rows=64)
+    got, ref, idx = _run(inp, 4, 1, 128, out_dtype=torch.float32, bias=False)
+    _check(got, ref, idx, "no bias", out_dtype=torch.float32)
+
+
+def test_out_of_range_position_skips_only_that_token():
+    T, nq, nkv, d = 40, 4, 2, 64
+    inp = kf_workloads.qkv_generate(T, seed=92, H=256, nq=nq, nkv=nkv, d=d, max_pos=512, cache_rows=128)
+    bad = 17
+    inp["positions"][bad] = 512  # one past the tables
+    rows = int(inp["rows"])
+    kc = torch.full((rows, nkv * d), SENT, dtype=torch.bfloat16, device=DEV)
+    vc = torch.full((rows, nkv * d), SENT, dtype=torch.bfloat16, device=DEV)
+    q = torch.full((T, nq * d), SENT, dtype=torch.bfloat16, device=DEV)
+    g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
+    kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"], nq, nkv, d, kc, vc,
+                   q_out=q)
+    st, raw = kf.get_device_error()
+    assert st == kf.KF_ERR_DEVICE_BOUNDS and raw & 8
+    assert bool((q[bad] == SENT).all())
+    r = int(inp["cache_rows"][bad])
+    assert bool((kc[r] == SENT).all()) and bool((vc[r] == SENT).all())
+    good = torch.tensor([t for t in range(T) if t != bad])
+    rq, rk, rv = oracle.qkv_rope_kv(inp["X"][good], inp["W"], inp["b"], inp["positions"][good],
+                                    inp["cache_rows"][good], inp["cos"], inp["sin"], nq, nkv, d, rows)
+    _check((q, kc, vc), (rq, rk, rv), good, "bad position")
+    assert kf.get_device_error()[0] == kf.KF_OK  # the read cleared the word
+
+
+def test_full_size_prefill_sampled_tokens_and_repeats():
+    # 4096-token prefill at the gpt-oss shape, checked on sampled tokens; the
+    # path's arithmetic order is fixed, so repeated calls agree bit for bit
+    s = kf_workloads.QKV_SHAPE
+    T = 4096
+    inp = kf_workloads.qkv_generate(T, seed=93, prefill=True, cache_rows=8192)
+    sub = [0, 1, 127, 128, 255, 256, 2047, 3001, T - 1]
+    got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"], sub=sub)
+    _check(got, ref, idx, "prefill 4096 sampled", all_tokens=False)
+    g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
+    for _ in range(3):
+        kc = torch.full_like(got[1], SENT)
+        vc = torch.full_like(got[2], SENT)
+        q = kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"],
+                           s["nq"], s["nkv"], s["d"], kc, vc)
+        assert torch.equal(q, got[0]) and torch.equal(kc, got[1]) and torch.equal(vc, got[2])
+    assert kf.get_device_error()[0] == kf.KF_OK

@@ -505,3 +505,15 @@ def test_qkv_rejects_out_of_range_position_or_row():
     badr[0] = -1
     with pytest.raises(ValueError):
         oracle.qkv_rope_kv(X, W, b, pos, badr, *cs, c["nq"], c["nkv"], c["d"], c["rows"])
+
+
+def test_qkv_fp16_operands_read_like_bf16_ones():
+    # small integers are exact in both 16-bit formats: the same projection
+    X, W, b, pos, crow, s, c = _qkv_case(47)
+    half = c["d"] // 2
+    cs = torch.ones(c["max_pos"], half), torch.zeros(c["max_pos"], half)
+    args = (pos, crow, *cs, c["nq"], c["nkv"], c["d"], c["rows"])
+    q16, k16, v16 = oracle.qkv_rope_kv(X.half(), W.half(), b.float(), *args)
+    assert np.array_equal(q16, s[:, :c["nq"] * c["d"]])
+    assert np.array_equal(k16[crow.numpy()], s[:, c["nq"] * c["d"]:(c["nq"] + c["nkv"]) * c["d"]])
+    assert np.array_equal(v16[crow.numpy()], s[:, (c["nq"] + c["nkv"]) * c["d"]:])
