@@ -389,6 +389,49 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
                                   "roofline_frac": round(byts / (peaks["hbm"] * 1e9) * 1e3 / ms, 4),
                                   "unfused_ms": round(ms_u, 5), "speedup_vs_unfused": round(ms_u / ms, 3),
                                   "launches_per_step": 6}
+    # attention input projection with bias + rotary embedding + KV-cache write in
+    # its epilogue (gpt-oss-20b shape), against our GEMM + bias followed by torch's
+    # rotation and cache copies, and cuBLAS's GEMM alone
+    sh = kf_workloads.QKV_SHAPE
+    nq, nkv, dh, Hq = sh["nq"], sh["nkv"], sh["d"], sh["H"]
+    Nq = (nq + 2 * nkv) * dh
+    for T in (1, 64, 4096):
+        inp = kf_workloads.qkv_generate(T, seed=0, prefill=T > 128, cache_rows=max(8192, T))
+        g = {k2: v.to(dev) for k2, v in inp.items() if k2 != "rows"}
+        rows = int(inp["rows"])
+        kc = torch.zeros(rows, nkv * dh, dtype=torch.bfloat16, device=dev)
+        vc = torch.zeros_like(kc)
+        q = torch.empty(T, nq * dh, dtype=torch.bfloat16, device=dev)
+        need = kf.qkv_workspace_bytes(T, nq, nkv, dh)
+        ws = torch.zeros(need, dtype=torch.uint8, device=dev) if need else None
+        fused = lambda: kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"],
+                                       nq, nkv, dh, kc, vc, q_out=q, workspace=ws)
+        y = torch.empty(T, Nq, dtype=torch.bfloat16, device=dev)
+        pos, crow = g["positions"].long(), g["cache_rows"].long()
+
+        def unfused():
+            kf.fused_gemm(g["X"], g["W"], [("bias", {"p0": g["b"]})], out=y)
+            hd = y.view(T, nq + 2 * nkv, dh)
+            c, sn = g["cos"][pos][:, None, :], g["sin"][pos][:, None, :]
+            x = hd[:, :nq + nkv].float()
+            a, b = x[..., :dh // 2], x[..., dh // 2:]
+            r = torch.cat([a * c - b * sn, b * c + a * sn], -1).to(torch.bfloat16)
+            q.copy_(r[:, :nq].reshape(T, -1))
+            kc.index_copy_(0, crow, r[:, nq:].reshape(T, -1))
+            vc.index_copy_(0, crow, hd[:, nq + nkv:].reshape(T, -1))
+        ms = time_steps(fused, steps, args.warmup, flush, stream)
+        ms_u = time_steps(unfused, steps, args.warmup, flush, stream)
+        ms_c = time_steps(lambda: torch.matmul(g["X"], g["W"].t()), steps, args.warmup, flush, stream)
+        byts = Nq * Hq * 2 + T * Hq * 2 + Nq * 2 + T * Nq * 2 + 2 * T * (dh // 2) * 4
+        flops = 2.0 * T * Nq * Hq
+        t_roof = max(flops / (peaks["bf16"] * 1e12), byts / (peaks["hbm"] * 1e9)) * 1e3
+        bound = "hbm" if byts / (peaks["hbm"] * 1e9) > flops / (peaks["bf16"] * 1e12) else "tensor"
+        res[f"qkv_rope_kv_T{T}"] = {"tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
+                                   "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
+                                   "k_split": bool(need), "unfused_ms": round(ms_u, 5),
+                                   "speedup_vs_unfused": round(ms_u / ms, 3), "cublas_gemm_only_ms": round(ms_c, 5),
+                                   "launches_per_step": 1}
+        del g, inp, kc, vc
     return res
 
 
@@ -396,7 +439,17 @@ def profile_workload(name, dev, reps):
     """Run one workload through the public API `reps` times (no timing): the
     command that ncu launch lists and captures of that workload are taken on."""
     import paper_2606_02963_gb300 as kf
-    if name.startswith("moe_T"):
+    if name.startswith("qkv_T"):
+        T = int(name[5:])
+        sh = kf_workloads.QKV_SHAPE
+        inp = kf_workloads.qkv_generate(T, seed=0, prefill=T > 128, cache_rows=max(8192, T))
+        g = {k: v.to(dev) for k, v in inp.items() if k != "rows"}
+        kc = torch.zeros(int(inp["rows"]), sh["nkv"] * sh["d"], dtype=torch.bfloat16, device=dev)
+        vc = torch.zeros_like(kc)
+        for _ in range(reps):
+            kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"], sh["nq"],
+                           sh["nkv"], sh["d"], kc, vc)
+    elif name.startswith("moe_T"):
         T, E, k, H, I = int(name[5:]), 32, 4, 2880, 2880
         g = torch.Generator("cpu").manual_seed(0)
         X = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
@@ -457,7 +510,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=16)
     ap.add_argument("--profile-workload", default=None,
                     help="run one workload's calls --steps times, untimed (the command ncu captures of it use): "
-                         "bf16_gelu_scale_residual, bf16_scale_rowlse, bf16_groupnorm_swish, moe_T64 or moe_T4096")
+                         "bf16_gelu_scale_residual, bf16_scale_rowlse, bf16_groupnorm_swish, moe_T64, moe_T4096 or "
+                         "qkv_T<tokens>")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

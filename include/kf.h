@@ -247,8 +247,8 @@ kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void*
  *     (KF_BF16, KF_F16 or KF_F32); ldq >= nq d, ld_cache >= nkv d.
  *   d: a multiple of 64, at most 256 (KF_ERR_UNSUPPORTED otherwise); nq, nkv >= 1.
  *   workspace (optional): kf_qkv_rope_kv_workspace(T, nq, nkv, d) bytes, 16-byte
- *     aligned, ZERO-FILLED before its first use; non-zero only for decode-sized
- *     calls (T <= 128), which then split the K dimension over all SMs and add
+ *     aligned, ZERO-FILLED before its first use; non-zero only for calls of at
+ *     most 16 tokens, which then split the K dimension over all SMs and add
  *     the partial sums in fp32 (atomically: the summation order, and so the
  *     last bits of the result, may vary from call to call).  Every call leaves
  *     the workspace zero-filled again, unless it reports a device error (then

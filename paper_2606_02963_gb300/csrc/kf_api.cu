@@ -952,6 +952,9 @@ int pick_rope_bn(int64_t M, int64_t N, int d, int nsm, bool cta2) {
 // QKV workspace for K splits: fp32 partial sums [T x N], then a counter per
 // (tile, lane quadrant, warp half) of the widest tile count (64-column tiles)
 constexpr int64_t kRopeMaxSplits = 16;
+// K splits pay off only while the partial sums are few rows: above this the
+// fp32 reductions into the shared rows cost more than the SMs they bring
+constexpr int64_t kRopeSplitMaxT = 16;
 int64_t rope_acc_bytes(int64_t T, int64_t N) { return (T * N * 4 + 255) / 256 * 256; }
 int64_t rope_ws_bytes(int64_t T, int64_t N) { return rope_acc_bytes(T, N) + ((N + 63) / 64) * 4 * 2 * 4; }
 
@@ -985,7 +988,7 @@ int pick_rope_split(int64_t N, int64_t num_kb, int d, int nsm, int* bn_out) {
 }  // namespace kf
 
 extern "C" size_t kf_qkv_rope_kv_workspace(int64_t T, int32_t nq, int32_t nkv, int32_t d) {
-  if (T <= 0 || T > kf::kBM || nq < 1 || nkv < 1 || d < 1) return 0;  // K splits serve decode-sized calls
+  if (T <= 0 || T > kf::kRopeSplitMaxT || nq < 1 || nkv < 1 || d < 1) return 0;  // K splits: few-token calls
   const int64_t N = (static_cast<int64_t>(nq) + 2 * static_cast<int64_t>(nkv)) * d;
   return static_cast<size_t>(kf::rope_ws_bytes(T, N));
 }
@@ -1029,7 +1032,7 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
   const bool cta2 = T > kBM && di.nsm >= 2;
   const int64_t num_kb = (H + kBK - 1) / kBK;
   // decode-sized: K splits over all SMs when the caller gave the workspace
-  const bool split_ok = !cta2 && workspace && aligned16(workspace) &&
+  const bool split_ok = T <= kRopeSplitMaxT && workspace && aligned16(workspace) &&
                         workspace_bytes >= static_cast<size_t>(rope_ws_bytes(T, N));
   int bn = 0, splits = 1;
   if (split_ok)

@@ -216,6 +216,6 @@ def test_qkv_rope_kv_argument_errors_before_any_launch(L):
     assert call(bias=fake, bdt=kf.KF_I32) == kf.KF_ERR_INVALID_ARG
     assert call(T=0, X=None, kc=None) == kf.KF_OK       # empty: nothing read or written
     # K-split workspace only for decode-sized calls
-    assert L.kf_qkv_rope_kv_workspace(128, 64, 8, 64) >= 128 * 5120 * 4
-    assert L.kf_qkv_rope_kv_workspace(129, 64, 8, 64) == 0
+    assert L.kf_qkv_rope_kv_workspace(16, 64, 8, 64) >= 16 * 5120 * 4
+    assert L.kf_qkv_rope_kv_workspace(17, 64, 8, 64) == 0
     assert L.kf_qkv_rope_kv_workspace(0, 64, 8, 64) == 0
