@@ -284,8 +284,11 @@ int pick_dense_bn(int mode, int64_t M, int64_t N, int nsm, bool cta2) {
 // one 128-row tile per group on average) stream each group's weights once and
 // are bound by how evenly the tiles fall on the SMs: take the width with the
 // fewest tile-widths of weights on the busiest SM (+ a small fixed cost per
-// tile).  Otherwise the widest compiled tile that divides N, else the one
-// wasting the fewest columns.
+// tile).  Otherwise the fewest tiles: a tcgen05.mma of K = 16 takes the same
+// time for any N up to 256 on this GPU (measured: ~0.33 us per 64-wide k-block
+// at N = 128, 192 and 256, with or without the operand loads), so a tile's
+// mainloop costs the same whatever its width and the widest tile does the most
+// work per MMA; its epilogue adds a little per column.
 int pick_grouped_outn(int mode, int64_t N, int64_t rows_total, int32_t G, int nsm) {
   static const int cand[] = {256, 192, 128};
   int best = 0;
@@ -304,13 +307,13 @@ int pick_grouped_outn(int mode, int64_t N, int64_t rows_total, int32_t G, int ns
     }
     return best;
   }
-  int64_t best_waste = INT64_MAX;
+  int64_t best_cost = INT64_MAX;
   for (int bn : cand) {
     if (!tc_grouped_has(mode, bn)) continue;
     const int outn = mode == kModeSwiglu ? bn / 2 : bn;
-    const int64_t waste = ((N + outn - 1) / outn) * outn - N;
-    if (waste < best_waste) {
-      best_waste = waste;
+    const int64_t cost = ((N + outn - 1) / outn) * (1024 + outn);
+    if (cost < best_cost) {
+      best_cost = cost;
       best = bn;
     }
   }
