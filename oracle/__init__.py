@@ -82,7 +82,9 @@ def _load():
             lib.orc_fused_gemm.restype = ctypes.c_int
             lib.orc_moe_route.argtypes = [P, I64, I32, I32, P, P, P, P, P, P]
             lib.orc_moe_route.restype = ctypes.c_int
-            lib.orc_moe_ffn.argtypes = [P, P, P, P, P, I64, I64, I32, P, I64, ctypes.c_int, P, ctypes.c_int]
+            D = ctypes.c_double
+            lib.orc_moe_ffn.argtypes = [P, P, P, P, P, I64, I64, I32, P, I64, ctypes.c_int, P, ctypes.c_int,
+                                        P, P, D, D, D]
             lib.orc_moe_ffn.restype = ctypes.c_int
             lib.orc_grouped_gemm.argtypes = [P, ctypes.c_int, I64, P, P, ctypes.c_int, I64, I64, P, I32,
                                              I64, I64, P, ctypes.c_int, P, I64]
@@ -204,9 +206,14 @@ def moe_route(logits, k: int):
 
 
 def moe_ffn(X, W_gu, W_down, topk_ids, topk_w, tokens: Optional[Sequence[int]] = None,
-            round_h: bool = True, nthreads: int = 0) -> np.ndarray:
+            round_h: bool = True, nthreads: int = 0, b_gu=None, b_down=None, alpha: float = 1.0,
+            limit: float = 0.0, linear_offset: float = 0.0) -> np.ndarray:
     """Per-token MoE expert FFN in fp64 (h rounded to bf16 unless round_h=False).
-    Returns float64 [len(tokens), H]."""
+    The expert activation is g' sigmoid(alpha g') (u' + linear_offset) with g, u
+    clamped to (-inf, limit] / [-limit, limit] when limit > 0, after the optional
+    per-expert biases b_gu [E, 2I] (gate then up, bf16); b_down [E, H] (bf16) is
+    added to each expert's output before its routing weight.  The defaults are the
+    plain SwiGLU.  Returns float64 [len(tokens), H]."""
     lib = _load()
     x, _ = _np(X)
     wg, _ = _np(W_gu)
@@ -219,8 +226,18 @@ def moe_ffn(X, W_gu, W_down, topk_ids, topk_w, tokens: Optional[Sequence[int]] =
     toks = np.ascontiguousarray(np.arange(T, dtype=np.int64) if tokens is None
                                 else np.asarray(tokens, dtype=np.int64))
     Y = np.zeros((len(toks), H), np.float64)
+    bg = bd = None
+    if b_gu is not None:
+        bg, t1 = _np(b_gu)
+        if t1 != ORC_BF16:
+            raise TypeError("moe_ffn: b_gu must be bf16")
+    if b_down is not None:
+        bd, t2 = _np(b_down)
+        if t2 != ORC_BF16:
+            raise TypeError("moe_ffn: b_down must be bf16")
     lib.orc_moe_ffn(_ptr(x), _ptr(wg), _ptr(wd), _ptr(ids), _ptr(w), H, I, k, _ptr(toks), len(toks),
-                    1 if round_h else 0, _ptr(Y), int(nthreads))
+                    1 if round_h else 0, _ptr(Y), int(nthreads), None if bg is None else _ptr(bg),
+                    None if bd is None else _ptr(bd), float(alpha), float(limit), float(linear_offset))
     return Y
 
 

@@ -336,15 +336,21 @@ int orc_moe_route(const float *logits, int64_t T, int32_t E, int32_t k, int32_t 
 
 /* ------------------------------------------------------------------------- */
 /* MoE expert FFN, written per token (the plain definition):                   */
-/*   g = W_gu[e, 0:I, :] x_t,  u = W_gu[e, I:2I, :] x_t,                        */
-/*   h = bf16(silu(g) * u)      (or unrounded when round_h == 0),               */
-/*   Y_t = sum_j w_tj * W_down[e_tj] h.                                         */
+/*   g = W_gu[e, 0:I, :] x_t + bg[e],  u = W_gu[e, I:2I, :] x_t + bu[e],        */
+/*   h = bf16(act(g, u))         (or unrounded when round_h == 0),              */
+/*   Y_t = sum_j w_tj * (W_down[e_tj] h + bd[e_tj]).                            */
+/* act(g, u) = g' * sigmoid(alpha g') * (u' + c) with g' = min(g, L) and       */
+/* u' = clamp(u, -L, L) when L > 0 (else g' = g, u' = u): the plain SwiGLU is   */
+/* alpha = 1, L = 0, c = 0 and no biases; the gpt-oss expert activation adds    */
+/* the clamp, a sigmoid slope, the +1 on the linear branch and per-expert       */
+/* biases (b_gu [E x 2I]: gate then up; b_down [E x H]; bf16, or NULL).        */
 /* X [T x H] bf16, W_gu [E x 2I x H] bf16, W_down [E x H x I] bf16.            */
 /* Only tokens listed in `tokens` (n_tok of them) are computed; output row r    */
 /* of Y (double, [n_tok x H]) belongs to token tokens[r].                      */
 /* ------------------------------------------------------------------------- */
 typedef struct {
-  const uint16_t *X, *Wgu, *Wd;
+  const uint16_t *X, *Wgu, *Wd, *bgu, *bd;
+  double alpha, limit, c;
   const int32_t *ids;
   const double *w;
   int64_t H, I;
@@ -381,13 +387,22 @@ static void *orc_moe_worker(void *arg) {
           g += x[c] * orc_load(wg, ORC_BF16, n * H + c);
           u += x[c] * orc_load(wg, ORC_BF16, (I + n) * H + c);
         }
-        double hv = g * orc_sigmoid(g) * u;
+        if (jb->bgu) {
+          g += orc_load(jb->bgu, ORC_BF16, e * 2 * I + n);
+          u += orc_load(jb->bgu, ORC_BF16, e * 2 * I + I + n);
+        }
+        if (jb->limit > 0.0) {
+          g = fmin(g, jb->limit);
+          u = fmax(fmin(u, jb->limit), -jb->limit);
+        }
+        double hv = g * orc_sigmoid(jb->alpha * g) * (u + jb->c);
         h[n] = jb->round_h ? orc_round_bf16(hv) : hv;
       }
       const uint16_t *wd = jb->Wd + e * H * I;
       for (int64_t c = 0; c < H; ++c) {
         double acc = 0.0;
         for (int64_t n = 0; n < I; ++n) acc += h[n] * orc_load(wd, ORC_BF16, c * I + n);
+        if (jb->bd) acc += orc_load(jb->bd, ORC_BF16, e * H + c);
         y[c] += wt * acc;
       }
     }
@@ -399,10 +414,12 @@ static void *orc_moe_worker(void *arg) {
 
 int orc_moe_ffn(const uint16_t *X, const uint16_t *W_gu, const uint16_t *W_down,
                 const int32_t *topk_ids, const double *topk_w, int64_t H, int64_t I, int32_t k,
-                const int64_t *tokens, int64_t n_tok, int round_h, double *Y, int nthreads) {
+                const int64_t *tokens, int64_t n_tok, int round_h, double *Y, int nthreads,
+                const uint16_t *b_gu, const uint16_t *b_down, double alpha, double limit, double c) {
   orc_moe_job jb;
   memset(&jb, 0, sizeof jb);
   jb.X = X; jb.Wgu = W_gu; jb.Wd = W_down; jb.ids = topk_ids; jb.w = topk_w;
+  jb.bgu = b_gu; jb.bd = b_down; jb.alpha = alpha; jb.limit = limit; jb.c = c;
   jb.H = H; jb.I = I; jb.k = k; jb.tokens = tokens; jb.n_tok = n_tok; jb.round_h = round_h;
   jb.Y = Y; jb.next = 0;
   pthread_mutex_init(&jb.mu, NULL);

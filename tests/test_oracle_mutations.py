@@ -37,6 +37,13 @@ MUTATIONS = {
     "rope_token_not_position": ("(double)cos_t[pos * half + i]", "(double)cos_t[t * half + i]"),
     "rope_adjacent_partner": ("const double a = h[i], b = h[i + half];", "const double a = h[i], b = h[i ^ 1];"),
     "kv_row_is_token": ("k_cache + (int64_t)row * nkv * d", "k_cache + t * nkv * d"),
+    "moe_alpha_ignored": ("orc_sigmoid(jb->alpha * g)", "orc_sigmoid(g)"),
+    "moe_gate_clamp_symmetric": ("g = fmin(g, jb->limit);", "g = fmax(fmin(g, jb->limit), -jb->limit);"),
+    "moe_linear_offset_dropped": ("* (u + jb->c);", "* u;"),
+    "moe_down_bias_outside_weight": ("if (jb->bd) acc += orc_load(jb->bd, ORC_BF16, e * H + c);\n        y[c] += wt * acc;",
+                                     "y[c] += wt * acc;\n        if (jb->bd) y[c] += orc_load(jb->bd, ORC_BF16, e * H + c);"),
+    "moe_up_bias_from_gate": ("u += orc_load(jb->bgu, ORC_BF16, e * 2 * I + I + n);",
+                              "u += orc_load(jb->bgu, ORC_BF16, e * 2 * I + n);"),
     "residual_dropped": ("case ORC_RESIDUAL_ADD: return v + orc_load", "case ORC_RESIDUAL_ADD: return v + 0 * orc_load"),
 }
 

@@ -517,3 +517,76 @@ def test_qkv_fp16_operands_read_like_bf16_ones():
     assert np.array_equal(q16, s[:, :c["nq"] * c["d"]])
     assert np.array_equal(k16[crow.numpy()], s[:, c["nq"] * c["d"]:(c["nq"] + c["nkv"]) * c["d"]])
     assert np.array_equal(v16[crow.numpy()], s[:, (c["nq"] + c["nkv"]) * c["d"]:])
+
+
+# ---- gpt-oss expert activation: per-expert biases, clamp, sigmoid slope, +c on the linear branch
+def _gate_case(bg, bu, alpha, limit, c, I=4, H=6, E=3, seed=51):
+    """X = 0, so g and u are the biases exactly; k = 1 (weight 1); W_down maps h[n]
+    to output column n; returns the output row of the token routed to expert 1."""
+    T = 2
+    X = bf16(torch.zeros(T, H))
+    Wgu = bf16(torch.zeros(E, 2 * I, H))
+    Wd = torch.zeros(E, H, I)
+    for n in range(I):
+        Wd[:, n, n] = 1.0
+    Wd = bf16(Wd)
+    b_gu = torch.zeros(E, 2 * I)
+    b_gu[1, :I] = torch.tensor(bg, dtype=torch.float32)
+    b_gu[1, I:] = torch.tensor(bu, dtype=torch.float32)
+    b_gu = bf16(b_gu)
+    logits = torch.tensor([[0.0, 5.0, 0.0], [5.0, 0.0, 0.0]])[:T, :E]
+    r = oracle.moe_route(logits, 1)
+    assert r["topk_ids"][0, 0] == 1 and r["topk_w"][0, 0] == 1.0
+    Y = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"], round_h=False, b_gu=b_gu, alpha=alpha,
+                       limit=limit, linear_offset=c)
+    return Y[0, :I]
+
+
+def test_moe_gate_activation_at_exact_sigmoid_points():
+    # sigmoid(ln 3) = 3/4 and sigmoid(-ln 3) = 1/4 exactly; biases are exact in bf16
+    l3 = math.log(3.0)
+    # slope: g = 1, alpha = ln 3 -> 1 * 3/4 * (u + 1) with u = 2 -> 2.25
+    # gate clamp from above: g = 12 -> 8 with alpha = ln 3 / 8 -> 8 * 3/4 * 3 = 18
+    y = _gate_case([1.0, 12.0, 0.0, -1.0], [2.0, 2.0, 5.0, -1.0], alpha=l3, limit=8.0, c=1.0)
+    assert math.isclose(y[0], 2.25, rel_tol=1e-14)
+    y = _gate_case([12.0, 0.0, 0.0, 0.0], [2.0, 0.0, 0.0, 0.0], alpha=l3 / 8, limit=8.0, c=1.0)
+    assert math.isclose(y[0], 18.0, rel_tol=1e-14)
+    # no clamp below on the gate: g = -12, alpha = ln 3 / 12 -> -12 * 1/4 * (2 + 1) = -9
+    y = _gate_case([-12.0, 0.0, 0.0, 0.0], [2.0, 0.0, 0.0, 0.0], alpha=l3 / 12, limit=8.0, c=1.0)
+    assert math.isclose(y[0], -9.0, rel_tol=1e-14)
+    # the linear branch is clamped on both sides: u = -20 -> -8, u = 20 -> 8
+    y = _gate_case([1.0, 1.0, 0.0, 0.0], [-20.0, 20.0, 0.0, 0.0], alpha=l3, limit=8.0, c=1.0)
+    assert math.isclose(y[0], 0.75 * -7.0, rel_tol=1e-14) and math.isclose(y[1], 0.75 * 9.0, rel_tol=1e-14)
+    # g = 0 or u + c = 0 give exactly zero; without a limit nothing is clamped
+    y = _gate_case([0.0, 1.0, 0.0, 0.0], [7.0, -1.0, 0.0, 0.0], alpha=l3, limit=8.0, c=1.0)
+    assert y[0] == 0.0 and y[1] == 0.0
+    y = _gate_case([12.0, 0.0, 0.0, 0.0], [20.0, 0.0, 0.0, 0.0], alpha=l3 / 12, limit=0.0, c=0.0)
+    assert math.isclose(y[0], 12.0 * 0.75 * 20.0, rel_tol=1e-14)
+
+
+def test_moe_down_bias_is_weighted_per_expert():
+    # X = 0 and W_down = 0: the output is the routing-weighted sum of the chosen
+    # experts' down biases, whatever the activation does
+    T, H, I, E, k = 5, 8, 4, 4, 2
+    g = torch.Generator().manual_seed(52)
+    X = bf16(torch.zeros(T, H))
+    Wgu = bf16(torch.randn(E, 2 * I, H, generator=g))
+    Wd = bf16(torch.zeros(E, H, I))
+    b_gu = bf16(torch.randn(E, 2 * I, generator=g))
+    b_down = bf16(torch.randn(E, H, generator=g))
+    r = oracle.moe_route(torch.randn(T, E, generator=g), k)
+    Y = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"], b_gu=b_gu, b_down=b_down, alpha=1.702, limit=7.0,
+                       linear_offset=1.0)
+    bd = f64(b_down)
+    ref = np.stack([sum(r["topk_w"][t, j] * bd[r["topk_ids"][t, j]] for j in range(k)) for t in range(T)])
+    assert np.allclose(Y, ref, rtol=1e-14, atol=1e-15)
+
+
+def test_moe_gate_defaults_are_the_plain_swiglu():
+    X, Wgu, Wd, logits = _moe_small()
+    r = oracle.moe_route(logits, 2)
+    E, I2, H = Wgu.shape
+    Y0 = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"])
+    Y1 = oracle.moe_ffn(X, Wgu, Wd, r["topk_ids"], r["topk_w"], b_gu=bf16(torch.zeros(E, I2)),
+                        b_down=bf16(torch.zeros(E, H)), alpha=1.0, limit=0.0, linear_offset=0.0)
+    assert np.array_equal(Y0, Y1)
