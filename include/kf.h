@@ -197,6 +197,36 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
 size_t kf_moe_ffn_workspace_ex(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags);
 
 /*
+ * kf_moe_ffn_act -- kf_moe_ffn_ex with the gated-expert activation and biases of
+ *                   the gpt-oss expert MLP (the model of the paper's B200 decode
+ *                   study, Sec. IV-A; the paper itself gives no formula)
+ *
+ *   g = x W_gate[e]^T + bg[e],  u = x W_up[e]^T + bu[e]     (fp32 accumulators)
+ *   g' = min(g, limit), u' = clamp(u, -limit, limit)        (when limit > 0)
+ *   h  = bf16(g' * sigmoid(alpha * g') * (u' + linear_offset))
+ *   Y[t] = sum_j w_tj * (h W_down[e_tj]^T + bd[e_tj])
+ *   {alpha 1, limit 0, linear_offset 0, no biases} is the plain SwiGLU of
+ *   kf_moe_ffn_ex; gpt-oss uses alpha 1.702, limit 7, linear_offset 1 and both
+ *   biases.  Gate and up rows stay the concatenated halves of W_gu[e] (a model
+ *   that interleaves them is permuted once when its weights are loaded).
+ *   b_gu: bf16 [E x 2I] (gate bias then up bias of each expert), b_down: bf16
+ *   [E x H]; either may be NULL; both 16-byte aligned (KF_ERR_MISALIGNED).
+ *   alpha, limit, linear_offset finite and limit >= 0 (KF_ERR_INVALID_ARG).
+ *   Everything else (arguments, flags, workspace, errors) as kf_moe_ffn_ex.
+ */
+typedef struct kf_moe_act {
+  float alpha;
+  float limit;
+  float linear_offset;
+  const void* b_gu;
+  const void* b_down;
+} kf_moe_act;
+kf_status kf_moe_ffn_act(const void* X, const float* logits, const void* W_gu, const void* W_down,
+                         const kf_moe_act* act, void* Y, int64_t T, int64_t H, int64_t I, int32_t E, int32_t k,
+                         uint32_t flags, void* workspace, size_t workspace_bytes, int32_t* topk_ids_out,
+                         float* topk_w_out, void* stream);
+
+/*
  * kf_moe_ffn_add_rmsnorm -- the MoE block tail fused into the MoE finalize
  *                          (Sec. IV-A: the gpt-oss decode kernels "Fused Add +
  *                          RMSNorm" and "MoE finalize"; Sec. VI: optimising the

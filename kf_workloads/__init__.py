@@ -204,3 +204,16 @@ def qkv_generate(T: int, seed: int = 0, H: int = 2880, nq: int = 64, nkv: int = 
     ang = torch.arange(max_pos, dtype=torch.float64)[:, None] * inv[None, :]
     return dict(X=X, W=W, b=b, positions=positions, cache_rows=crow, cos=torch.cos(ang).float(),
                 sin=torch.sin(ang).float(), rows=torch.tensor(rows))
+
+
+# gpt-oss expert activation: sigmoid slope, clamp limit, offset on the linear branch
+GPT_OSS_ACT = dict(alpha=1.702, limit=7.0, linear_offset=1.0)
+
+
+def moe_bias_generate(E: int, H: int, I: int, seed: int = 0, std_gu: float = 0.5,
+                      std_down: float = 0.1) -> Dict[str, torch.Tensor]:
+    """Per-expert biases of the gated expert MLP: b_gu [E, 2I] (gate then up)
+    ~ N(0, std_gu), b_down [E, H] ~ N(0, std_down), bf16."""
+    g = torch.Generator("cpu").manual_seed(seed)
+    return dict(b_gu=(torch.randn(E, 2 * I, generator=g) * std_gu).to(torch.bfloat16),
+                b_down=(torch.randn(E, H, generator=g) * std_down).to(torch.bfloat16))

@@ -36,7 +36,7 @@ ABI_SYMBOLS = (
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
     "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex", "kf_moe_ffn_add_rmsnorm",
-    "kf_qkv_rope_kv", "kf_qkv_rope_kv_workspace",
+    "kf_qkv_rope_kv", "kf_qkv_rope_kv_workspace", "kf_moe_ffn_act",
 )
 
 
@@ -50,6 +50,11 @@ class EpilogueOp(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int32), ("scalar", ctypes.c_float), ("eps", ctypes.c_float),
                 ("groups", ctypes.c_int32), ("p0", ctypes.c_void_p), ("p1", ctypes.c_void_p),
                 ("p_dtype", ctypes.c_int32), ("ld", ctypes.c_int64)]
+
+
+class MoeAct(ctypes.Structure):
+    _fields_ = [("alpha", ctypes.c_float), ("limit", ctypes.c_float), ("linear_offset", ctypes.c_float),
+                ("b_gu", ctypes.c_void_p), ("b_down", ctypes.c_void_p)]
 
 
 class Epilogue(ctypes.Structure):
@@ -82,6 +87,9 @@ def lib() -> ctypes.CDLL:
     L.kf_moe_ffn_workspace.restype = SZ
     L.kf_moe_ffn_ex.argtypes = [P, P, P, P, P, I64, I64, I64, I32, I32, ctypes.c_uint32, P, SZ, P, P, P]
     L.kf_moe_ffn_ex.restype = I32
+    L.kf_moe_ffn_act.argtypes = [P, P, P, P, ctypes.POINTER(MoeAct), P, I64, I64, I64, I32, I32, ctypes.c_uint32, P,
+                                 SZ, P, P, P]
+    L.kf_moe_ffn_act.restype = I32
     L.kf_moe_ffn_add_rmsnorm.argtypes = [P, P, P, P, P, P, ctypes.c_float, P, P, I64, I64, I64, I32, I32,
                                          ctypes.c_uint32, P, SZ, P, P, P]
     L.kf_moe_ffn_add_rmsnorm.restype = I32
@@ -258,10 +266,12 @@ def moe_ffn_workspace_bytes(T: int, H: int, I: int, E: int, k: int, deterministi
 
 def moe_ffn(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tensor, W_down: torch.Tensor, k: int,
             out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
-            return_routing: bool = False, deterministic: bool = False, stream=None):
+            return_routing: bool = False, deterministic: bool = False, act: Optional[Dict] = None, stream=None):
     """Routed MoE expert FFN (kf_moe_ffn_ex): route, gate/up + SwiGLU, down +
     scale + scatter-add (or, deterministic, per-row outputs summed in slot order),
-    bf16 output.  With ``return_routing`` also returns (ids, w)."""
+    bf16 output.  With ``return_routing`` also returns (ids, w).  ``act`` (keys
+    alpha, limit, linear_offset, b_gu [E, 2I], b_down [E, H]; kf_moe_ffn_act)
+    selects the gated-expert activation with per-expert biases."""
     T, H = X.shape
     E, I2, _ = W_gu.shape
     I = I2 // 2
@@ -277,9 +287,21 @@ def moe_ffn(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tensor, W_down: t
     if return_routing:
         ids = torch.empty(T, k, dtype=torch.int32, device=X.device)
         w = torch.empty(T, k, dtype=torch.float32, device=X.device)
-    st = L.kf_moe_ffn_ex(X.data_ptr(), logits.data_ptr(), W_gu.data_ptr(), W_down.data_ptr(), out.data_ptr(), T, H,
-                         I, E, k, flags, _ptr(ws), ws_bytes, _ptr(ids), _ptr(w), _stream(stream))
-    _check(st, "kf_moe_ffn_ex")
+    if act is None:
+        st = L.kf_moe_ffn_ex(X.data_ptr(), logits.data_ptr(), W_gu.data_ptr(), W_down.data_ptr(), out.data_ptr(), T,
+                             H, I, E, k, flags, _ptr(ws), ws_bytes, _ptr(ids), _ptr(w), _stream(stream))
+        _check(st, "kf_moe_ffn_ex")
+    else:
+        for nm in ("b_gu", "b_down"):
+            b = act.get(nm)
+            if b is not None and (b.dtype != torch.bfloat16 or not b.is_contiguous()):
+                raise ValueError(f"{nm} must be contiguous bf16")
+        a = MoeAct(float(act.get("alpha", 1.0)), float(act.get("limit", 0.0)), float(act.get("linear_offset", 0.0)),
+                   _ptr(act.get("b_gu")), _ptr(act.get("b_down")))
+        st = L.kf_moe_ffn_act(X.data_ptr(), logits.data_ptr(), W_gu.data_ptr(), W_down.data_ptr(), ctypes.byref(a),
+                              out.data_ptr(), T, H, I, E, k, flags, _ptr(ws), ws_bytes, _ptr(ids), _ptr(w),
+                              _stream(stream))
+        _check(st, "kf_moe_ffn_act")
     return (out, ids, w) if return_routing else out
 
 

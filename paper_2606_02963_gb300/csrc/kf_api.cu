@@ -3,6 +3,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <chrono>
 #include <cstring>
@@ -381,10 +382,18 @@ size_t grouped_ws_bytes(int64_t rows_total, int64_t K, bool gathered) {
   return gathered ? align_up(static_cast<size_t>(rows_total) * static_cast<size_t>(K) * 2, 256) : 0;
 }
 
+// Per-group bias and the gated SwiGLU of the MoE path (see TcParams).
+struct GroupExtras {
+  const void* gbias = nullptr;  // bf16, group stride gbias_ld
+  int64_t gbias_ld = 0;
+  bool sw_ext = false;
+  float sw_alpha = 1.0f, sw_limit = 0.0f, sw_c = 0.0f;
+};
+
 // `pdl`: the previous kernel in the stream is one of this library's (MoE chain),
 // so the launches here may be programmatic dependents of it.
 kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cudaStream_t s, const DevInfo& di,
-                       bool pdl) {
+                       bool pdl, const GroupExtras* ex = nullptr) {
   const void* A = g.A;
   int64_t lda = g.lda;
   if (g.a_row_index) {
@@ -422,6 +431,14 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   p.dst_rows = static_cast<int32_t>(pl.dst_rows);
   fill_params_common(p, pl, di.err);
   p.fast = g.c_dtype == KF_BF16 && pl.mode != kModeScatter;
+  if (ex) {
+    p.gbias = ex->gbias;
+    p.gbias_ld = ex->gbias_ld;
+    p.sw_ext = ex->sw_ext ? 1 : 0;
+    p.sw_alpha = ex->sw_alpha;
+    p.sw_limit = ex->sw_limit;
+    p.sw_c = ex->sw_c;
+  }
   const int64_t ub = ((g.rows_total + kBM - 1) / kBM + g.G) * p.tiles_n;
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
   CUtensorMap mc;  // grouped outputs are masked per group: plain stores, no TMA map
@@ -745,8 +762,14 @@ struct BlockTail {
 
 kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
                        int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags, void* workspace, size_t ws_bytes,
-                       int32_t* topk_ids_out, float* topk_w_out, void* stream, const BlockTail* tail) {
+                       int32_t* topk_ids_out, float* topk_w_out, void* stream, const BlockTail* tail,
+                       const kf_moe_act* act = nullptr) {
   if (flags & ~KF_MOE_DETERMINISTIC) return KF_ERR_INVALID_ARG;
+  if (act && (!std::isfinite(act->alpha) || !(act->limit >= 0.0f) || !std::isfinite(act->limit) ||
+              !std::isfinite(act->linear_offset)))
+    return KF_ERR_INVALID_ARG;
+  if (act && ((act->b_gu && !aligned16(act->b_gu)) || (act->b_down && !aligned16(act->b_down))))
+    return KF_ERR_MISALIGNED;
   const bool det = (flags & KF_MOE_DETERMINISTIC) != 0;
   if (T < 0 || H < 1 || I < 1 || E < 1 || E > 256 || k < 1 || k > E) return KF_ERR_INVALID_ARG;
   if (T * k > INT32_MAX || H > INT32_MAX || I > INT32_MAX) return KF_ERR_INVALID_ARG;
@@ -789,7 +812,16 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     st = plan_chain(&epi, I, true, &pl);
     if (st != KF_OK) return st;
     GroupedArgs g{X, H, T, stok, W_gu, H, 2 * I * H, off, E, P, I, H, h, KF_BF16, I};
-    st = grouped_core(g, pl, xg, s, di, true);
+    GroupExtras ex;
+    if (act) {
+      ex.gbias = act->b_gu;
+      ex.gbias_ld = 2 * I;
+      ex.sw_ext = true;
+      ex.sw_alpha = act->alpha;
+      ex.sw_limit = act->limit;
+      ex.sw_c = act->linear_offset;
+    }
+    st = grouped_core(g, pl, xg, s, di, true, &ex);
     if (st != KF_OK) return st;
   }
   if (det) {
@@ -804,7 +836,12 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     if (st != KF_OK) return st;
     float* yp = reinterpret_cast<float*>(ws + L.yp);
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yp, KF_F32, H};
-    st = grouped_core(g, pl, nullptr, s, di, true);
+    GroupExtras ex;
+    if (act) {
+      ex.gbias = act->b_down;
+      ex.gbias_ld = H;
+    }
+    st = grouped_core(g, pl, nullptr, s, di, true, &ex);
     if (st != KF_OK) return st;
     if (tail)
       st = cuda_status(moe_add_rmsnorm_launch(nullptr, yp, pos, k, T, H, tail->R, tail->gamma, tail->eps, tail->R_out, Y,
@@ -825,7 +862,12 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     st = plan_chain(&epi, H, true, &pl);
     if (st != KF_OK) return st;
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yacc, KF_F32, H};
-    st = grouped_core(g, pl, nullptr, s, di, true);
+    GroupExtras ex;
+    if (act) {
+      ex.gbias = act->b_down;
+      ex.gbias_ld = H;
+    }
+    st = grouped_core(g, pl, nullptr, s, di, true, &ex);
     if (st != KF_OK) return st;
     if (tail)
       st = cuda_status(moe_add_rmsnorm_launch(yacc, nullptr, nullptr, k, T, H, tail->R, tail->gamma, tail->eps,
@@ -851,6 +893,15 @@ kf_status kf_moe_ffn_ex(const void* X, const float* logits, const void* W_gu, co
                         int32_t* topk_ids_out, float* topk_w_out, void* stream) {
   return moe_ffn_impl(X, logits, W_gu, W_down, Y, T, H, I, E, k, flags, workspace, ws_bytes, topk_ids_out, topk_w_out,
                       stream, nullptr);
+}
+
+kf_status kf_moe_ffn_act(const void* X, const float* logits, const void* W_gu, const void* W_down,
+                         const kf_moe_act* act, void* Y, int64_t T, int64_t H, int64_t I, int32_t E, int32_t k,
+                         uint32_t flags, void* workspace, size_t ws_bytes, int32_t* topk_ids_out, float* topk_w_out,
+                         void* stream) {
+  if (!act) return KF_ERR_INVALID_ARG;
+  return moe_ffn_impl(X, logits, W_gu, W_down, Y, T, H, I, E, k, flags, workspace, ws_bytes, topk_ids_out, topk_w_out,
+                      stream, nullptr, act);
 }
 
 kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void* W_gu, const void* W_down,

@@ -110,6 +110,18 @@ struct TcParams {
   int32_t k_splits;
   float* ks_acc;
   int32_t* ks_cnt;
+  // grouped GEMMs: bf16 bias of the unit's group added to the accumulator
+  // before anything else (column j of group g at gbias[g * gbias_ld + j]; for
+  // SwiGLU the up half's bias follows at + b_rows), or null
+  const void* gbias;
+  int64_t gbias_ld;
+  // SwiGLU with the gated-expert extension (sw_ext != 0): h = g' sigmoid(sw_alpha
+  // g') (u' + sw_c), g' = min(g, sw_limit), u' = clamp(u, -sw_limit, sw_limit)
+  // when sw_limit > 0; otherwise the plain silu(g) * u
+  int32_t sw_ext;
+  float sw_alpha;
+  float sw_limit;
+  float sw_c;
 };
 
 // ---------------------------------------------------------------- loads/stores

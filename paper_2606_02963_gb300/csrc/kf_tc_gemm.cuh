@@ -555,6 +555,14 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           : "memory");
       return r != 0;
     };
+    // grouped GEMMs: add the unit's group bias (bf16) to 32 accumulator columns
+    auto add_gbias = [&](float (&x)[32], int32_t g, int64_t col, int nvalid) {
+      if (!p.gbias) return;
+      float b[32];
+      ld32(p.gbias, KF_BF16, static_cast<int64_t>(g) * p.gbias_ld + col, nvalid, true, b);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) x[j] += b[j];
+    };
     // Chan's pairwise merge of (count, mean, M2) moments
     auto chan = [](float na, float ma, float qa, float nb, float mb, float qb, float& n, float& m, float& qq) {
       n = na + nb;
@@ -687,12 +695,29 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             if (sg.vec_idx >= 0) pack16(bq, sg.vec);
             issue_chunk(c + 2);
             tmem_ld32(tb + c * 32, v);
+            if constexpr (GROUPED) add_gbias(v, ui.g, col0, nvalid);
             run_chain<PRE>(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok, sg);
           } else if constexpr (MODE == kModeSwiglu) {
             float gt[32];
             tmem_ld32(tb + c * 32, gt);
             tmem_ld32(tb + Cfg::kOutN + c * 32, v);
-            if (fast) {
+            if (p.gbias) {
+              add_gbias(gt, ui.g, col0, nvalid);
+              add_gbias(v, ui.g, p.b_rows + col0, nvalid);
+            }
+            if (p.sw_ext) {
+              // gated expert: gate clamped from above, linear branch on both sides
+              const float L = p.sw_limit, al = p.sw_alpha, c1 = p.sw_c;
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                float g1 = gt[j], u1 = v[j];
+                if (L > 0.0f) {
+                  g1 = fminf(g1, L);
+                  u1 = fminf(fmaxf(u1, -L), L);
+                }
+                v[j] = g1 * (fast ? f_sigmoid_fast(al * g1) : f_sigmoid(al * g1)) * (u1 + c1);
+              }
+            } else if (fast) {
               // fp32 hardware tanh: h feeds the down GEMM, which sums 2880 of
               // them, so it keeps more precision than a direct bf16 output needs
 #pragma unroll
@@ -704,6 +729,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             run_chain<POST>(fast, p.post, p.n_post, v, grow, col0, nvalid, row_ok);
           } else {
             tmem_ld32(tb + c * 32, v);
+            if constexpr (GROUPED) add_gbias(v, ui.g, col0, nvalid);
             run_chain<PRE>(fast, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
           }
           if constexpr (RT) {

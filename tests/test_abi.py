@@ -219,3 +219,18 @@ def test_qkv_rope_kv_argument_errors_before_any_launch(L):
     assert L.kf_qkv_rope_kv_workspace(16, 64, 8, 64) >= 16 * 5120 * 4
     assert L.kf_qkv_rope_kv_workspace(17, 64, 8, 64) == 0
     assert L.kf_qkv_rope_kv_workspace(0, 64, 8, 64) == 0
+
+
+def test_moe_ffn_act_argument_errors_before_any_launch(L):
+    fake = 1 << 20
+
+    def call(alpha=1.702, limit=7.0, off=1.0, b_gu=fake, b_down=fake, act=True):
+        a = kf.MoeAct(alpha, limit, off, b_gu, b_down)
+        return L.kf_moe_ffn_act(fake, fake, fake, fake, ctypes.byref(a) if act else None, fake, 4, 2880, 2880, 32, 4,
+                                0, fake, 1 << 30, None, None, None)
+    assert call(act=False) == kf.KF_ERR_INVALID_ARG
+    assert call(limit=-1.0) == kf.KF_ERR_INVALID_ARG
+    assert call(alpha=float("nan")) == kf.KF_ERR_INVALID_ARG
+    assert call(off=float("inf")) == kf.KF_ERR_INVALID_ARG
+    assert call(b_gu=fake + 2) == kf.KF_ERR_MISALIGNED
+    assert call(b_down=fake + 8) == kf.KF_ERR_MISALIGNED

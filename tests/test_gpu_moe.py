@@ -203,3 +203,55 @@ def test_moe_add_rmsnorm_in_place_and_consistent_with_moe_ffn():
     diff = (R1.float() - (Rd.float() + y.float())).abs()
     assert diff.max().item() <= 2e-2 * (Rd.float() + y.float()).abs().max().item()
     _no_device_error()
+
+
+def _act(b, dev=None, **over):
+    a = dict(kf_workloads.GPT_OSS_ACT)
+    a.update(over)
+    if b is not None:
+        a["b_gu"], a["b_down"] = (b["b_gu"].to(dev), b["b_down"].to(dev)) if dev else (b["b_gu"], b["b_down"])
+    return a
+
+
+@pytest.mark.parametrize("det", [False, True])
+@pytest.mark.parametrize("T,H,I,E,k,w_std", [(24, 64, 96, 8, 2, 0.3), (100, 256, 320, 16, 4, 0.15),
+                                             (7, 2880, 2880, 32, 4, 0.02)])
+def test_moe_gated_expert_activation_with_biases(T, H, I, E, k, w_std, det):
+    # weights large enough that many gate / linear values pass the clamp limit
+    m = kf_workloads.moe_generate(T, seed=T + 3, H=H, I=I, E=E, k=k, w_std=w_std)
+    b = kf_workloads.moe_bias_generate(E, H, I, seed=T)
+    out = kf.moe_ffn(m["X"].to(DEV), m["logits"].to(DEV), m["W_gu"].to(DEV), m["W_down"].to(DEV), k,
+                     deterministic=det, act=_act(b, DEV))
+    r = oracle.moe_route(m["logits"], k)
+    ref = oracle.moe_ffn(m["X"], m["W_gu"], m["W_down"], r["topk_ids"], r["topk_w"], **_act(b))
+    check_bf16(out, ref, f"gated moe T={T} det={det}")
+    _no_device_error()
+    if w_std >= 0.15:  # the clamp is live: without it the result differs
+        no_clamp = oracle.moe_ffn(m["X"], m["W_gu"], m["W_down"], r["topk_ids"], r["topk_w"], **_act(b, limit=0.0))
+        assert np.abs(no_clamp - ref).max() > 0.1
+
+
+@pytest.mark.parametrize("T,n_check", [(64, 64), (4096, 16)])
+def test_moe_gated_full_size(T, n_check):
+    m = kf_workloads.moe_generate(T, seed=1)
+    b = kf_workloads.moe_bias_generate(32, 2880, 2880, seed=2)
+    d = {k2: v.to(DEV) for k2, v in m.items()}
+    out = kf.moe_ffn(d["X"], d["logits"], d["W_gu"], d["W_down"], 4, act=_act(b, DEV))
+    torch.cuda.synchronize()
+    r = oracle.moe_route(m["logits"], 4)
+    toks = sorted(set([0, T - 1] + list(np.random.default_rng(3).choice(T, n_check, replace=False))))
+    ref = oracle.moe_ffn(m["X"], m["W_gu"], m["W_down"], r["topk_ids"], r["topk_w"], tokens=toks, **_act(b))
+    check_bf16(out[toks], ref, f"gated moe T={T}")
+    _no_device_error()
+
+
+def test_moe_act_plain_parameters_equal_plain_swiglu_bitwise():
+    # alpha 1, no clamp, offset 0, no biases: the same arithmetic as kf_moe_ffn_ex
+    m = kf_workloads.moe_generate(300, seed=9, H=512, I=384, E=16, k=4, w_std=0.05)
+    d = {k2: v.to(DEV) for k2, v in m.items()}
+    y0 = kf.moe_ffn(d["X"], d["logits"], d["W_gu"], d["W_down"], 4, deterministic=True)
+    y1 = kf.moe_ffn(d["X"], d["logits"], d["W_gu"], d["W_down"], 4, deterministic=True,
+                    act=dict(alpha=1.0, limit=0.0, linear_offset=0.0))
+    torch.cuda.synchronize()
+    assert torch.equal(y0, y1)
+    _no_device_error()
