@@ -389,6 +389,22 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
                                   "roofline_frac": round(byts / (peaks["hbm"] * 1e9) * 1e3 / ms, 4),
                                   "unfused_ms": round(ms_u, 5), "speedup_vs_unfused": round(ms_u / ms, 3),
                                   "launches_per_step": 6}
+    # the gpt-oss expert activation (per-expert biases, clamped gated SwiGLU) at
+    # decode, against the plain SwiGLU path on the same inputs
+    b = kf_workloads.moe_bias_generate(E, H, I, seed=0)
+    act = dict(kf_workloads.GPT_OSS_ACT, b_gu=b["b_gu"].to(dev), b_down=b["b_down"].to(dev))
+    g = torch.Generator("cpu").manual_seed(0)
+    X = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
+    logits = torch.randn(T, E, generator=g).to(dev)
+    gated = lambda: kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, out=y_out, workspace=ws, act=act)
+    plain = lambda: kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, out=y_out, workspace=ws)
+    ms = time_steps(gated, steps, args.warmup, flush, stream)
+    ms_p = time_steps(plain, steps, args.warmup, flush, stream)
+    touched = int(torch.unique(torch.topk(logits, k, dim=1).indices).numel())
+    byts = touched * ((2 * I * H + H * I) * 2 + (2 * I + H) * 2) + 2 * T * H * 2 + 4 * T * E
+    res["moe_T64_gptoss_act"] = {"ms": round(ms, 5), "gbs": round(byts / ms / 1e6, 1), "bound": "hbm",
+                                 "roofline_frac": round(byts / (peaks["hbm"] * 1e9) * 1e3 / ms, 4),
+                                 "plain_swiglu_ms": round(ms_p, 5), "launches_per_step": 6}
     # attention input projection with bias + rotary embedding + KV-cache write in
     # its epilogue (gpt-oss-20b shape), against our GEMM + bias followed by torch's
     # rotation and cache copies, and cuBLAS's GEMM alone
