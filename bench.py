@@ -146,14 +146,29 @@ def whole_job_tflops(flops_per_rank_step, ms_per_step, world):
     return world * flops_per_rank_step / (ms_per_step * 1e-3) / 1e12
 
 
+SETTLE_S = 0.3
+
+
 def time_steps(fn, steps, warmup, flush, stream, host_slack=True):
-    """Mean device time (ms) of fn() over `steps` calls; L2 flushed before each.
+    """Mean device time (ms) of fn() over `steps` calls; L2 flushed before each,
+    after `warmup` untimed calls and at least SETTLE_S seconds of untimed calls.
     With host_slack, a ~100 us device-side sleep follows the flush so that the
     host has enqueued the step before its start event fires (host-side argument
     marshalling is then outside the device-timed window)."""
     for _ in range(warmup):
         flush.zero_()
         fn()
+    torch.cuda.synchronize()
+    # then at least SETTLE_S of back-to-back steps (untimed), so that clocks and
+    # caches are in their steady state whatever ran before on this GPU
+    t_end = time.perf_counter() + SETTLE_S
+    n = 0
+    while time.perf_counter() < t_end and n < 2000:
+        flush.zero_()
+        fn()
+        n += 1
+        if n % 16 == 0:
+            torch.cuda.synchronize()
     torch.cuda.synchronize()
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     for a, b in evs:
