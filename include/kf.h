@@ -110,8 +110,13 @@ typedef struct kf_epilogue {
  *   stride ldy), or Y [M] (fp32 or bf16) when the chain holds ROW_LOGSUMEXP.
  *   Operand dtypes: both KF_BF16 or both KF_F16 (tcgen05 tensor-core path, fp32
  *   accumulation in tensor memory; Y bf16, fp16 or fp32; the paper's B580
- *   kernels ran their matmuls in fp16, Sec. IV-B), or both KF_F32 (exact fp32 FFMA path; Y
- *   fp32; element-wise chains only).
+ *   kernels ran their matmuls in fp16, Sec. IV-B), or both KF_F32 (element-wise
+ *   chains only): problems below 2^30 FLOP (2 M N K) take the exact fp32 FFMA
+ *   path (Y fp32); larger ones run on the tensor cores as three tf32 products
+ *   (3xTF32: each operand split into a tf32 high part and an fp32 remainder,
+ *   X W^T = Xh Wh^T + Xh Wl^T + Xl Wh^T accumulated in fp32; Y fp32, bf16 or
+ *   fp16; needs X, W 16-byte aligned and ldx, ldw multiples of 4, else the
+ *   FFMA path runs) -- kf_fused_gemm_ex chooses explicitly.
  *   bf16 path: X, W must be 16-byte aligned with ldx, ldw multiples of 8, else
  *   KF_ERR_MISALIGNED.  M == 0 or N == 0 is a no-op; K must be >= 1.
  *   workspace: kf_fused_gemm_workspace() bytes.  Required for a row
@@ -127,6 +132,18 @@ kf_status kf_fused_gemm(const void* X, int32_t x_dtype, int64_t ldx, const void*
                         int64_t ldw, void* Y, int32_t y_dtype, int64_t ldy, int64_t M, int64_t N, int64_t K,
                         const kf_epilogue* epi, void* workspace, size_t workspace_bytes, void* stream);
 size_t kf_fused_gemm_workspace(int64_t M, int64_t N, int64_t K, const kf_epilogue* epi);
+
+/* kf_fused_gemm with flags for fp32 operands: KF_GEMM_F32_FFMA keeps the exact
+ * FFMA path at any size; KF_GEMM_F32_TF32X3 takes the 3xTF32 tensor-core path
+ * at any size (KF_ERR_MISALIGNED if X, W or ldx, ldw do not allow its 16-byte
+ * TMA boxes).  Both at once, or an unknown bit: KF_ERR_INVALID_ARG.  flags = 0
+ * is kf_fused_gemm.  No effect on bf16 / fp16 operands. */
+#define KF_GEMM_F32_FFMA 1u
+#define KF_GEMM_F32_TF32X3 2u
+kf_status kf_fused_gemm_ex(const void* X, int32_t x_dtype, int64_t ldx, const void* W, int32_t w_dtype,
+                           int64_t ldw, void* Y, int32_t y_dtype, int64_t ldy, int64_t M, int64_t N, int64_t K,
+                           const kf_epilogue* epi, void* workspace, size_t workspace_bytes, uint32_t flags,
+                           void* stream);
 
 /*
  * kf_moe_route -- top-k routing of T tokens over E experts  (Sec. IV-A, decode path)

@@ -36,8 +36,9 @@ ABI_SYMBOLS = (
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
     "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex", "kf_moe_ffn_add_rmsnorm",
-    "kf_qkv_rope_kv", "kf_qkv_rope_kv_workspace", "kf_moe_ffn_act",
+    "kf_qkv_rope_kv", "kf_qkv_rope_kv_workspace", "kf_moe_ffn_act", "kf_fused_gemm_ex",
 )
+KF_GEMM_F32_FFMA, KF_GEMM_F32_TF32X3 = 1, 2
 
 
 class KfError(RuntimeError):
@@ -75,6 +76,8 @@ def lib() -> ctypes.CDLL:
     P, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
     EP = ctypes.POINTER(Epilogue)
     L.kf_fused_gemm.argtypes = [P, I32, I64, P, I32, I64, P, I32, I64, I64, I64, I64, EP, P, SZ, P]
+    L.kf_fused_gemm_ex.argtypes = [P, I32, I64, P, I32, I64, P, I32, I64, I64, I64, I64, EP, P, SZ, ctypes.c_uint32, P]
+    L.kf_fused_gemm_ex.restype = I32
     L.kf_fused_gemm_workspace.argtypes = [I64, I64, I64, EP]
     L.kf_fused_gemm_workspace.restype = SZ
     L.kf_moe_route.argtypes = [P, I64, I32, I32, P, P, P, P, P, P]
@@ -193,9 +196,10 @@ def _workspace(nbytes: int, device, workspace: Optional[torch.Tensor]) -> Tuple[
 
 def fused_gemm(X: torch.Tensor, W: torch.Tensor, chain: Sequence[Tuple[str, Dict]] = (),
                out: Optional[torch.Tensor] = None, out_dtype: Optional[torch.dtype] = None,
-               workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    """Y = chain(X W^T) on the GPU (kf_fused_gemm).  Y is [M, N], or [M] after a
-    row log-sum-exp (fp32 unless ``out_dtype`` says otherwise)."""
+               workspace: Optional[torch.Tensor] = None, f32_mode: Optional[str] = None, stream=None) -> torch.Tensor:
+    """Y = chain(X W^T) on the GPU (kf_fused_gemm_ex).  Y is [M, N], or [M] after a
+    row log-sum-exp (fp32 unless ``out_dtype`` says otherwise).  fp32 operands:
+    ``f32_mode`` "ffma" or "tf32x3" forces a path (default: by problem size)."""
     M, K = X.shape
     N = W.shape[0]
     lse = any(k == "row_logsumexp" for k, _ in chain)
@@ -208,10 +212,11 @@ def fused_gemm(X: torch.Tensor, W: torch.Tensor, chain: Sequence[Tuple[str, Dict
     ws_need = L.kf_fused_gemm_workspace(M, N, K, ctypes.byref(epi))
     ws, ws_bytes = _workspace(ws_need, X.device, workspace)
     ldy = out.stride(0) if out.dim() == 2 else 1
-    st = L.kf_fused_gemm(X.data_ptr(), _dt(X), _rows(X, "X"), W.data_ptr(), _dt(W), _rows(W, "W"),
-                         out.data_ptr(), _dt(out), ldy, M, N, K, ctypes.byref(epi), _ptr(ws), ws_bytes,
-                         _stream(stream))
-    _check(st, "kf_fused_gemm")
+    flags = {None: 0, "ffma": KF_GEMM_F32_FFMA, "tf32x3": KF_GEMM_F32_TF32X3}[f32_mode]
+    st = L.kf_fused_gemm_ex(X.data_ptr(), _dt(X), _rows(X, "X"), W.data_ptr(), _dt(W), _rows(W, "W"),
+                            out.data_ptr(), _dt(out), ldy, M, N, K, ctypes.byref(epi), _ptr(ws), ws_bytes, flags,
+                            _stream(stream))
+    _check(st, "kf_fused_gemm_ex")
     return out
 
 

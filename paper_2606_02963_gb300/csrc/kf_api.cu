@@ -81,6 +81,23 @@ kf_status make_map(CUtensorMap* m, const void* base, uint64_t k, uint64_t rows, 
   return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
 }
 
+// fp32 operand map for the 3xTF32 path: [rows, K], box 32 (K, 128 bytes) x
+// box_rows, 128-byte swizzle.
+kf_status make_map_f32(CUtensorMap* m, const void* base, uint64_t k, uint64_t rows, uint64_t row_stride_bytes,
+                       uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return KF_ERR_CUDA;
+  std::memset(m, 0, sizeof(*m));
+  cuuint64_t dims[2] = {k, rows};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {32, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? KF_OK : KF_ERR_CUDA;
+}
+
 // Output tensor map for the epilogue's TMA stores: bf16 [rows x cols] (row
 // stride in bytes), box 16 columns x 32 rows, 32-byte swizzle (the layout of the
 // epilogue's tile buffers).
@@ -502,6 +519,14 @@ size_t kf_fused_gemm_workspace(int64_t M, int64_t N, int64_t K, const kf_epilogu
 kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt, int64_t ldw, void* Y,
                         int32_t yt, int64_t ldy, int64_t M, int64_t N, int64_t K, const kf_epilogue* epi,
                         void* workspace, size_t ws_bytes, void* stream) {
+  return kf_fused_gemm_ex(X, xt, ldx, W, wt, ldw, Y, yt, ldy, M, N, K, epi, workspace, ws_bytes, 0u, stream);
+}
+
+kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt, int64_t ldw, void* Y,
+                           int32_t yt, int64_t ldy, int64_t M, int64_t N, int64_t K, const kf_epilogue* epi,
+                           void* workspace, size_t ws_bytes, uint32_t flags, void* stream) {
+  if (flags & ~(KF_GEMM_F32_FFMA | KF_GEMM_F32_TF32X3)) return KF_ERR_INVALID_ARG;
+  if ((flags & KF_GEMM_F32_FFMA) && (flags & KF_GEMM_F32_TF32X3)) return KF_ERR_INVALID_ARG;
   if (M < 0 || N < 0 || K < 1) return KF_ERR_INVALID_ARG;
   if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return KF_ERR_INVALID_ARG;
   if (M == 0 || N == 0) return KF_OK;  // empty problem: nothing to read or write
@@ -513,9 +538,20 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   if (st != KF_OK) return st;
   if (pl.mode != kModeLse && ldy < N) return KF_ERR_INVALID_ARG;
   const bool f32_path = xt == KF_F32 && wt == KF_F32;
+  // fp32 operands: FFMA for small problems, three tf32 tensor-core products for
+  // large ones (>= 2^30 FLOP), or as the flags say
+  bool tf32x3 = false;
   if (f32_path) {
-    // exact fp32 FFMA path: element-wise chains only
-    if (pl.mode != kModeStore || yt != KF_F32) return KF_ERR_UNSUPPORTED;
+    if (pl.mode != kModeStore) return KF_ERR_UNSUPPORTED;  // element-wise chains only
+    const bool big = 2.0 * static_cast<double>(M) * static_cast<double>(N) * static_cast<double>(K) >= 1073741824.0;
+    tf32x3 = (flags & KF_GEMM_F32_TF32X3) || (big && !(flags & KF_GEMM_F32_FFMA));
+    if (tf32x3) {
+      if (!aligned16(X) || !aligned16(W) || ldx % 4 != 0 || ldw % 4 != 0) {
+        if (flags & KF_GEMM_F32_TF32X3) return KF_ERR_MISALIGNED;
+        tf32x3 = false;  // automatic choice: the FFMA path takes any layout
+      }
+    }
+    if (!tf32x3 && yt != KF_F32) return KF_ERR_UNSUPPORTED;
   } else {
     // tensor-core path: A and B both bf16 or both fp16 (one operand format per MMA)
     if (xt != wt || (xt != KF_BF16 && xt != KF_F16)) return KF_ERR_UNSUPPORTED;
@@ -529,6 +565,37 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   st = device_info(&di);
   if (st != KF_OK) return st;
 
+  if (tf32x3) {
+    // tile width: 256 columns (each MMA does twice the work of a 128-wide one
+    // for the same issue cost) when that still gives every SM a tile
+    const int64_t tm = (M + 127) / 128;
+    const int bn = (tm * ((N + 255) / 256) >= di.nsm && tf32x3_has(256)) ? 256 : 128;
+    CUtensorMap ma, mb;
+    st = make_map_f32(&ma, X, K, M, ldx * 4, 128);
+    if (st != KF_OK) return st;
+    st = make_map_f32(&mb, W, K, N, ldw * 4, bn);
+    if (st != KF_OK) return st;
+    Tf32Params tp;
+    std::memset(&tp, 0, sizeof(tp));
+    tp.M = static_cast<int32_t>(M);
+    tp.N = static_cast<int32_t>(N);
+    tp.K = static_cast<int32_t>(K);
+    tp.tiles_m = static_cast<int32_t>(tm);
+    tp.tiles_n = static_cast<int32_t>((N + bn - 1) / bn);
+    tp.num_kb = static_cast<int32_t>((K + 31) / 32);
+    tp.n_ops = pl.n_pre;
+    for (int i = 0; i < pl.n_pre; ++i) tp.ops[i] = pl.pre[i];
+    tp.Y = Y;
+    tp.ldy = ldy;
+    tp.y_dtype = yt;
+    tp.y_vec_ok = aligned16(Y) && (ldy * elt_size(yt)) % 16 == 0;
+    tp.err = di.err;
+    tp.wait_ns = g_wait_ns.load();
+    tp.drain_ns = std::max<uint64_t>(tp.wait_ns, 1000000000ull);
+    const int64_t tiles = static_cast<int64_t>(tp.tiles_m) * tp.tiles_n;
+    const int grid = static_cast<int>(std::min<int64_t>(tiles, di.nsm));
+    return cuda_status(tf32x3_launch(bn, ma, mb, tp, grid, s));
+  }
   if (f32_path) {
     SimtParams sp;
     std::memset(&sp, 0, sizeof(sp));

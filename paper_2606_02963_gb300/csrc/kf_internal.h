@@ -51,6 +51,23 @@ bool tc_dense_has(int mode, int bn, bool cta2);
 bool tc_dense2_has(int mode, int bn);
 bool tc_dense2_has_prog(int mode, int bn, int sig);  // a compiled chain program for (mode, bn, sig)
 bool tc_grouped_has(int mode, int bn);
+// fp32 GEMM + element-wise chain as three tf32 tensor-core products (3xTF32)
+struct Tf32Params {
+  int32_t M, N, K;
+  int32_t tiles_m, tiles_n, num_kb;
+  int32_t n_ops;
+  DevOp ops[kMaxOps];
+  void* Y;
+  int64_t ldy;
+  int32_t y_dtype;
+  int32_t y_vec_ok;
+  uint32_t* err;
+  uint64_t wait_ns;
+  uint64_t drain_ns;
+};
+bool tf32x3_has(int bn);
+cudaError_t tf32x3_launch(int bn, const CUtensorMap& a, const CUtensorMap& b, const Tf32Params& p, int grid,
+                          cudaStream_t s);
 // QKV projection tail (kModeRope): single CTAs or CTA pairs; no output map
 bool tc_rope_has(int bn, bool cta2);
 cudaError_t tc_rope_launch(int bn, bool cta2, const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid,

@@ -234,3 +234,17 @@ def test_moe_ffn_act_argument_errors_before_any_launch(L):
     assert call(off=float("inf")) == kf.KF_ERR_INVALID_ARG
     assert call(b_gu=fake + 2) == kf.KF_ERR_MISALIGNED
     assert call(b_down=fake + 8) == kf.KF_ERR_MISALIGNED
+
+
+def test_fused_gemm_ex_flags_checked_before_any_launch(L):
+    fake = 1 << 20
+    op = kf.EpilogueOp()
+    epi = kf.Epilogue(0, ctypes.cast(ctypes.pointer(op), ctypes.POINTER(kf.EpilogueOp)))
+
+    def call(flags, ldx=64, X=fake):
+        return L.kf_fused_gemm_ex(X, kf.KF_F32, ldx, fake, kf.KF_F32, 64, fake, kf.KF_F32, 64, 64, 64, 64,
+                                  ctypes.byref(epi), None, 0, flags, None)
+    assert call(kf.KF_GEMM_F32_FFMA | kf.KF_GEMM_F32_TF32X3) == kf.KF_ERR_INVALID_ARG
+    assert call(4) == kf.KF_ERR_INVALID_ARG
+    assert call(kf.KF_GEMM_F32_TF32X3, ldx=66) == kf.KF_ERR_MISALIGNED
+    assert call(kf.KF_GEMM_F32_TF32X3, X=fake + 4) == kf.KF_ERR_MISALIGNED
