@@ -1,7 +1,7 @@
 // kf_tc_tf32.cu -- fp32 GEMM + element-wise tail on the tensor cores as three
 // tf32 products (3xTF32).  Each fp32 operand x is split into a tf32 high part
-// h = rna_tf32(x) and the remainder l = x - h (exact in fp32; the tensor core
-// reads its top 19 bits); X W^T is then Xh Wh^T + Xh Wl^T + Xl Wh^T in fp32,
+// h = rna_tf32(x) and the remainder l = rna_tf32(x - h) (x - h is exact in
+// fp32); X W^T is then Xh Wh^T + Xh Wl^T + Xl Wh^T in fp32,
 // dropping only Xl Wl^T (relative size ~2^-22), so the result stays within fp32
 // accuracy while the products run on tcgen05 (kind::tf32) instead of FFMA.
 //
@@ -217,7 +217,8 @@ __global__ void __launch_bounds__(kTfThreads, 1)
           const float4 x = ha[i];
           float4 h, l;
           h.x = rna_tf32(x.x); h.y = rna_tf32(x.y); h.z = rna_tf32(x.z); h.w = rna_tf32(x.w);
-          l.x = x.x - h.x; l.y = x.y - h.y; l.z = x.z - h.z; l.w = x.w - h.w;
+          l.x = rna_tf32(x.x - h.x); l.y = rna_tf32(x.y - h.y);
+          l.z = rna_tf32(x.z - h.z); l.w = rna_tf32(x.w - h.w);
           ha[i] = h;
           la[i] = l;
         }
@@ -227,7 +228,8 @@ __global__ void __launch_bounds__(kTfThreads, 1)
           const float4 x = hb[i];
           float4 h, l;
           h.x = rna_tf32(x.x); h.y = rna_tf32(x.y); h.z = rna_tf32(x.z); h.w = rna_tf32(x.w);
-          l.x = x.x - h.x; l.y = x.y - h.y; l.z = x.z - h.z; l.w = x.w - h.w;
+          l.x = rna_tf32(x.x - h.x); l.y = rna_tf32(x.y - h.y);
+          l.z = rna_tf32(x.z - h.z); l.w = rna_tf32(x.w - h.w);
           hb[i] = h;
           lb[i] = l;
         }
