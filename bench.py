@@ -420,6 +420,28 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
     res["moe_T64_gptoss_act"] = {"ms": round(ms, 5), "gbs": round(byts / ms / 1e6, 1), "bound": "hbm",
                                  "roofline_frac": round(byts / (peaks["hbm"] * 1e9) * 1e3 / ms, 4),
                                  "plain_swiglu_ms": round(ms_p, 5), "launches_per_step": 6}
+    # fp32 operands on the tensor cores (3xTF32) against cuBLAS's fp32 GEMM and
+    # our exact FFMA path; roofline: the tf32 rate (half the bf16 peak) over 3
+    Mf = Nf = Kf = 4096
+    g = torch.Generator("cpu").manual_seed(0)
+    Xf = torch.randn(Mf, Kf, generator=g).to(dev)
+    Wf = (torch.randn(Nf, Kf, generator=g) / Kf ** 0.5).to(dev)
+    bf = torch.randn(Nf, generator=g).to(dev)
+    yf = torch.empty(Mf, Nf, device=dev)
+    chf = [("bias", {"p0": bf}), ("relu", {})]
+    ms = time_steps(lambda: kf.fused_gemm(Xf, Wf, chf, out=yf, f32_mode="tf32x3"), steps, args.warmup, flush, stream)
+    ms_ffma = time_steps(lambda: kf.fused_gemm(Xf, Wf, chf, out=yf, f32_mode="ffma"), 3, 1, flush, stream)
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    ms_c = time_steps(lambda: torch.matmul(Xf, Wf.t()), steps, args.warmup, flush, stream)
+    torch.backends.cuda.matmul.allow_tf32 = prev
+    flops = 2.0 * Mf * Nf * Kf
+    peak3 = peaks["bf16"] / 2 / 3
+    res["fp32_bias_relu_4096_3xtf32"] = {"tflops": round(flops / ms / 1e9, 2), "ms": round(ms, 5), "bound": "tensor",
+                                         "roofline_frac": round(flops / ms / 1e9 / peak3, 4),
+                                         "roofline_peak_tflops": round(peak3, 1), "ffma_path_ms": round(ms_ffma, 5),
+                                         "cublas_fp32_gemm_only_ms": round(ms_c, 5), "launches_per_step": 1}
+    del Xf, Wf, yf
     # attention input projection with bias + rotary embedding + KV-cache write in
     # its epilogue (gpt-oss-20b shape), against our GEMM + bias followed by torch's
     # rotation and cache copies, and cuBLAS's GEMM alone
