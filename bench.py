@@ -455,10 +455,8 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
         kc = torch.zeros(rows, nkv * dh, dtype=torch.bfloat16, device=dev)
         vc = torch.zeros_like(kc)
         q = torch.empty(T, nq * dh, dtype=torch.bfloat16, device=dev)
-        need = kf.qkv_workspace_bytes(T, nq, nkv, dh)
-        ws = torch.zeros(need, dtype=torch.uint8, device=dev) if need else None
         fused = lambda: kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"],
-                                       nq, nkv, dh, kc, vc, q_out=q, workspace=ws)
+                                       nq, nkv, dh, kc, vc, q_out=q)
         y = torch.empty(T, Nq, dtype=torch.bfloat16, device=dev)
         pos, crow = g["positions"].long(), g["cache_rows"].long()
 
@@ -481,7 +479,7 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
         bound = "hbm" if byts / (peaks["hbm"] * 1e9) > flops / (peaks["bf16"] * 1e12) else "tensor"
         res[f"qkv_rope_kv_T{T}"] = {"tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
                                    "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
-                                   "k_split": bool(need), "unfused_ms": round(ms_u, 5),
+                                   "cluster_split": T <= 32, "unfused_ms": round(ms_u, 5),
                                    "speedup_vs_unfused": round(ms_u / ms, 3), "cublas_gemm_only_ms": round(ms_c, 5),
                                    "launches_per_step": 1}
         del g, inp, kc, vc

@@ -293,23 +293,16 @@ kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void*
  *   q_out [T x ldq], k_cache / v_cache [cache_rows_n x ld_cache]: out_dtype
  *     (KF_BF16, KF_F16 or KF_F32); ldq >= nq d, ld_cache >= nkv d.
  *   d: a multiple of 64, at most 256 (KF_ERR_UNSUPPORTED otherwise); nq, nkv >= 1.
- *   workspace (optional): kf_qkv_rope_kv_workspace(T, nq, nkv, d) bytes, 16-byte
- *     aligned, ZERO-FILLED before its first use; non-zero only for calls of at
- *     most 16 tokens, which then split the K dimension over all SMs and add
- *     the partial sums in fp32 (atomically: the summation order, and so the
- *     last bits of the result, may vary from call to call).  Every call leaves
- *     the workspace zero-filled again, unless it reports a device error (then
- *     zero it before the next use).  Calls sharing a workspace must not overlap
- *     on the GPU.  Without it (NULL or too small) each tile runs whole.
+ *   Calls of at most 32 tokens with d dividing 256 run as clusters of CTAs
+ *   that split K over each 256-column tile and add their partial sums in
+ *   shared memory (fixed order: repeated calls are bitwise identical).
  *   T = 0 writes nothing.  All buffers are the caller's; nothing is allocated.
  */
 kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dtype, int64_t ldx, int64_t ldw, const void* bias,
                          int32_t bias_dtype, const int32_t* positions, const int32_t* cache_rows, const float* cos_t,
                          const float* sin_t, int64_t max_pos, int64_t T, int64_t H, int32_t nq, int32_t nkv,
                          int32_t d, void* q_out, int64_t ldq, void* k_cache, void* v_cache, int64_t ld_cache,
-                         int64_t cache_rows_n, int32_t out_dtype, void* workspace, size_t workspace_bytes,
-                         void* stream);
-size_t kf_qkv_rope_kv_workspace(int64_t T, int32_t nq, int32_t nkv, int32_t d);
+                         int64_t cache_rows_n, int32_t out_dtype, void* stream);
 
 /*
  * kf_fused_gemm_lse_noalloc -- kf_fused_gemm for row log-sum-exp chains, without

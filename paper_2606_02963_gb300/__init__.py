@@ -36,7 +36,7 @@ ABI_SYMBOLS = (
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
     "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex", "kf_moe_ffn_add_rmsnorm",
-    "kf_qkv_rope_kv", "kf_qkv_rope_kv_workspace", "kf_moe_ffn_act", "kf_fused_gemm_ex",
+    "kf_qkv_rope_kv", "kf_moe_ffn_act", "kf_fused_gemm_ex",
 )
 KF_GEMM_F32_FFMA, KF_GEMM_F32_TF32X3 = 1, 2
 
@@ -97,10 +97,8 @@ def lib() -> ctypes.CDLL:
                                          ctypes.c_uint32, P, SZ, P, P, P]
     L.kf_moe_ffn_add_rmsnorm.restype = I32
     L.kf_qkv_rope_kv.argtypes = [P, P, I32, I64, I64, P, I32, P, P, P, P, I64, I64, I64, I32, I32, I32, P, I64,
-                                 P, P, I64, I64, I32, P, SZ, P]
+                                 P, P, I64, I64, I32, P]
     L.kf_qkv_rope_kv.restype = I32
-    L.kf_qkv_rope_kv_workspace.argtypes = [I64, I32, I32, I32]
-    L.kf_qkv_rope_kv_workspace.restype = SZ
     L.kf_moe_ffn_workspace_ex.argtypes = [I64, I64, I64, I32, I32, ctypes.c_uint32]
     L.kf_moe_ffn_workspace_ex.restype = SZ
     L.kf_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
@@ -340,14 +338,11 @@ def moe_ffn_add_rmsnorm(X: torch.Tensor, logits: torch.Tensor, W_gu: torch.Tenso
 def qkv_rope_kv(X: torch.Tensor, W: torch.Tensor, bias: Optional[torch.Tensor], positions: torch.Tensor,
                 cache_rows: torch.Tensor, cos_t: torch.Tensor, sin_t: torch.Tensor, nq: int, nkv: int, d: int,
                 k_cache: torch.Tensor, v_cache: torch.Tensor, q_out: Optional[torch.Tensor] = None,
-                workspace: Optional[torch.Tensor] = None, k_split: bool = True, stream=None) -> torch.Tensor:
+                stream=None) -> torch.Tensor:
     """QKV projection with bias, rotary embedding and key / value cache write
     (kf_qkv_rope_kv).  Writes rows ``cache_rows`` of ``k_cache`` / ``v_cache``
     ([rows, nkv d], their dtype is the output dtype) and returns the rotated
-    queries [T, nq d].  Decode-sized calls split K over the SMs in a workspace
-    of ``qkv_workspace_bytes`` bytes that must be zero-filled before its first
-    use and is left zero-filled; without one a zeroed workspace is made here
-    (``k_split=False``: no workspace, every tile runs whole)."""
+    queries [T, nq d]."""
     T, H = X.shape
     if q_out is None:
         q_out = torch.empty(T, nq * d, dtype=k_cache.dtype, device=X.device)
@@ -366,22 +361,13 @@ def qkv_rope_kv(X: torch.Tensor, W: torch.Tensor, bias: Optional[torch.Tensor], 
     if _dt(X) != _dt(W):
         raise TypeError("X and W must share one dtype")
     L = lib()
-    need = L.kf_qkv_rope_kv_workspace(T, nq, nkv, d) if k_split else 0
-    if workspace is None and need:
-        workspace = torch.zeros(need, dtype=torch.uint8, device=X.device)
-    ws, ws_bytes = (None, 0) if need == 0 else _workspace(need, X.device, workspace)
     st = L.kf_qkv_rope_kv(X.data_ptr(), W.data_ptr(), _dt(X), _rows(X, "X"), _rows(W, "W"), _ptr(bias),
                               _dt(bias) if bias is not None else KF_BF16, positions.data_ptr(), cache_rows.data_ptr(),
                               cos_t.data_ptr(), sin_t.data_ptr(), cos_t.shape[0], T, H, nq, nkv, d,
                               q_out.data_ptr(), _rows(q_out, "q_out"), k_cache.data_ptr(), v_cache.data_ptr(),
-                              _rows(k_cache, "k_cache"), k_cache.shape[0], _dt(k_cache), _ptr(ws), ws_bytes,
-                              _stream(stream))
+                              _rows(k_cache, "k_cache"), k_cache.shape[0], _dt(k_cache), _stream(stream))
     _check(st, "kf_qkv_rope_kv")
     return q_out
-
-
-def qkv_workspace_bytes(T: int, nq: int, nkv: int, d: int) -> int:
-    return lib().kf_qkv_rope_kv_workspace(T, nq, nkv, d)
 
 
 def get_device_error(stream=None) -> Tuple[int, int]:

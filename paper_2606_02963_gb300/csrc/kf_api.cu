@@ -1051,6 +1051,11 @@ namespace {
 // Tile width of the QKV projection: whole heads per tile (a multiple of d),
 // then the fewest tile-widths on the busiest SM (or CTA pair) + a fixed cost
 // per tile, as for the dense store variants.
+// Calls of at most this many tokens take the cluster-split decode kernel; above
+// it the per-token reduction costs more than the whole-tile kernel's MMAs
+// (measured at 64 and 128 tokens)
+constexpr int64_t kQkvClusterMaxT = 32;
+
 int pick_rope_bn(int64_t M, int64_t N, int d, int nsm, bool cta2) {
   static const int cand[] = {256, 128, 64};
   int best = 0;
@@ -1070,57 +1075,15 @@ int pick_rope_bn(int64_t M, int64_t N, int d, int nsm, bool cta2) {
   return best;
 }
 
-// QKV workspace for K splits: fp32 partial sums [T x N], then a counter per
-// (tile, lane quadrant, warp half) of the widest tile count (64-column tiles)
-constexpr int64_t kRopeMaxSplits = 16;
-// K splits pay off only while the partial sums are few rows: above this the
-// fp32 reductions into the shared rows cost more than the SMs they bring
-constexpr int64_t kRopeSplitMaxT = 16;
-int64_t rope_acc_bytes(int64_t T, int64_t N) { return (T * N * 4 + 255) / 256 * 256; }
-int64_t rope_ws_bytes(int64_t T, int64_t N) { return rope_acc_bytes(T, N) + ((N + 63) / 64) * 4 * 2 * 4; }
-
-// K splits of a decode-sized QKV projection (one 128-row tile): the split count
-// that minimises the busiest SM's k-blocks (+ a per-unit cost for the ramp and
-// the partial sums), weighted by the bytes a k-block stages (A rows + B rows).
-// Returns the tile width in *bn and the split count.
-int pick_rope_split(int64_t N, int64_t num_kb, int d, int nsm, int* bn_out) {
-  static const int cand[] = {256, 128, 64};
-  int64_t best_cost = INT64_MAX;
-  int best_s = 1, best_bn = 0;
-  for (int bn : cand) {
-    if (bn % d != 0 || !tc_rope_has(bn, false)) continue;
-    const int64_t tiles = (N + bn - 1) / bn;
-    for (int64_t sp = 1; sp <= std::min<int64_t>(kRopeMaxSplits, num_kb); ++sp) {
-      const int64_t waves = (tiles * sp + nsm - 1) / nsm;
-      const int64_t kper = (num_kb + sp - 1) / sp;
-      const int64_t cost = waves * (kper + (sp > 1 ? 2 : 0)) * (bn + kBM);
-      if (cost < best_cost) {
-        best_cost = cost;
-        best_s = static_cast<int>(sp);
-        best_bn = bn;
-      }
-    }
-  }
-  *bn_out = best_bn;
-  return best_s;
-}
-
 }  // namespace
 }  // namespace kf
-
-extern "C" size_t kf_qkv_rope_kv_workspace(int64_t T, int32_t nq, int32_t nkv, int32_t d) {
-  if (T <= 0 || T > kf::kRopeSplitMaxT || nq < 1 || nkv < 1 || d < 1) return 0;  // K splits: few-token calls
-  const int64_t N = (static_cast<int64_t>(nq) + 2 * static_cast<int64_t>(nkv)) * d;
-  return static_cast<size_t>(kf::rope_ws_bytes(T, N));
-}
 
 extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dtype, int64_t ldx, int64_t ldw,
                                     const void* bias, int32_t bias_dtype, const int32_t* positions,
                                     const int32_t* cache_rows, const float* cos_t, const float* sin_t,
                                     int64_t max_pos, int64_t T, int64_t H, int32_t nq, int32_t nkv, int32_t d,
                                     void* q_out, int64_t ldq, void* k_cache, void* v_cache, int64_t ld_cache,
-                                    int64_t cache_rows_n, int32_t out_dtype, void* workspace,
-                                    size_t workspace_bytes, void* stream) {
+                                    int64_t cache_rows_n, int32_t out_dtype, void* stream) {
   using namespace kf;
   if (T < 0 || H < 1 || nq < 1 || nkv < 1 || d < 1 || max_pos < 1 || cache_rows_n < 1) return KF_ERR_INVALID_ARG;
   if (T > INT32_MAX || H > INT32_MAX || max_pos > INT32_MAX || cache_rows_n > INT32_MAX) return KF_ERR_INVALID_ARG;
@@ -1152,14 +1115,56 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
   if (st != KF_OK) return st;
   const bool cta2 = T > kBM && di.nsm >= 2;
   const int64_t num_kb = (H + kBK - 1) / kBK;
-  // decode-sized: K splits over all SMs when the caller gave the workspace
-  const bool split_ok = T <= kRopeSplitMaxT && workspace && aligned16(workspace) &&
-                        workspace_bytes >= static_cast<size_t>(rope_ws_bytes(T, N));
-  int bn = 0, splits = 1;
-  if (split_ok)
-    splits = pick_rope_split(N, num_kb, d, di.nsm, &bn);
-  else
-    bn = pick_rope_bn(T, N, d, di.nsm, cta2);
+  if (T <= kQkvClusterMaxT && 256 % d == 0) {
+    // few tokens: clusters of S CTAs split K over one 256-column tile and
+    // reduce through distributed shared memory; S as large as keeps every
+    // cluster of the call resident at once
+    const int64_t tiles = (N + 255) / 256;
+    int S = 1;
+    for (int cand : {8, 6, 4, 2}) {
+      int nc = 0;
+      if (cand <= num_kb && qkv_decode_clusters(cand, &nc) == cudaSuccess && nc >= tiles) {
+        S = cand;
+        break;
+      }
+    }
+    const CUtensorMapDataType dt = xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    CUtensorMap ma, mb;
+    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, kBM, 2, dt);
+    if (st != KF_OK) return st;
+    st = make_map(&mb, W, H, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, 256, 3, dt);
+    if (st != KF_OK) return st;
+    QkvDecodeParams dp;
+    std::memset(&dp, 0, sizeof(dp));
+    dp.T = static_cast<int32_t>(T);
+    dp.N = static_cast<int32_t>(N);
+    dp.K = static_cast<int32_t>(H);
+    dp.num_kb = static_cast<int32_t>(num_kb);
+    dp.splits = S;
+    dp.ab_f16 = xw_dtype == KF_F16;
+    dp.bias = bias;
+    dp.bias_dtype = bias_dtype;
+    dp.cos_t = cos_t;
+    dp.sin_t = sin_t;
+    dp.positions = positions;
+    dp.cache_rows = cache_rows;
+    dp.max_pos = static_cast<int32_t>(max_pos);
+    dp.rows = static_cast<int32_t>(cache_rows_n);
+    dp.rope_d = d;
+    dp.q_cols = nq * d;
+    dp.rot_cols = (nq + nkv) * d;
+    dp.q_out = q_out;
+    dp.ldq = ldq;
+    dp.k_cache = k_cache;
+    dp.v_cache = v_cache;
+    dp.ld_cache = ld_cache;
+    dp.out_dtype = out_dtype;
+    dp.err = di.err;
+    dp.wait_ns = g_wait_ns.load();
+    dp.drain_ns = std::max<uint64_t>(dp.wait_ns, 1000000000ull);
+    return cuda_status(qkv_decode_launch(ma, mb, dp, static_cast<int>(tiles), s));
+  }
+  const int bn = pick_rope_bn(T, N, d, di.nsm, cta2);
   if (bn == 0) return KF_ERR_UNSUPPORTED;
   const CUtensorMapDataType op_dt =
       xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
@@ -1176,12 +1181,7 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
   p.tiles_m = static_cast<int32_t>((T + (cta2 ? 2 * kBM : kBM) - 1) / (cta2 ? 2 * kBM : kBM));
   p.tiles_n = static_cast<int32_t>((N + bn - 1) / bn);  // whole heads per tile; the last may hold fewer
   p.num_kb = static_cast<int32_t>(num_kb);
-  p.total_units = p.tiles_m * p.tiles_n * splits;
-  p.k_splits = splits;
-  if (splits > 1) {
-    p.ks_acc = static_cast<float*>(workspace);
-    p.ks_cnt = reinterpret_cast<int32_t*>(static_cast<char*>(workspace) + rope_acc_bytes(T, N));
-  }
+  p.total_units = p.tiles_m * p.tiles_n;
   p.C = q_out;
   p.ldc = ldq;
   p.c_dtype = out_dtype;

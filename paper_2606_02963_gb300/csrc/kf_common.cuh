@@ -102,14 +102,6 @@ struct TcParams {
   void* v_cache;
   int64_t ld_cache;
   int32_t kv_vec_ok;    // caches allow 16-byte stores of 32-column chunks
-  // K split (dense single-CTA QKV tail): unit u is tile u / k_splits over the
-  // k-blocks [s * num_kb / k_splits, (s + 1) * num_kb / k_splits), s = u %
-  // k_splits.  Partial sums are added into ks_acc (fp32 [M x N], zero between
-  // calls); the last split of a tile to arrive at ks_cnt[(tile * 4 + quadrant)
-  // * 2 + half] (zero between calls) finishes those rows and zeroes both again.
-  int32_t k_splits;
-  float* ks_acc;
-  int32_t* ks_cnt;
   // grouped GEMMs: bf16 bias of the unit's group added to the accumulator
   // before anything else (column j of group g at gbias[g * gbias_ld + j]; for
   // SwiGLU the up half's bias follows at + b_rows), or null

@@ -66,6 +66,33 @@ struct Tf32Params {
   uint64_t drain_ns;
 };
 bool tf32x3_has(int bn);
+// QKV projection tail for <= 128 tokens: K split over the CTAs of a cluster,
+// partials reduced through distributed shared memory
+struct QkvDecodeParams {
+  int32_t T, N, K, num_kb;
+  int32_t splits;        // CTAs per cluster = K splits of a 256-column tile
+  int32_t ab_f16;
+  const void* bias;      // [N] or null
+  int32_t bias_dtype;
+  const float* cos_t;
+  const float* sin_t;
+  const int32_t* positions;
+  const int32_t* cache_rows;
+  int32_t max_pos, rows;
+  int32_t rope_d, q_cols, rot_cols;
+  void* q_out;
+  int64_t ldq;
+  void* k_cache;
+  void* v_cache;
+  int64_t ld_cache;
+  int32_t out_dtype;
+  uint32_t* err;
+  uint64_t wait_ns;
+  uint64_t drain_ns;
+};
+cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
+                              cudaStream_t s);
+cudaError_t qkv_decode_clusters(int splits, int* out);
 cudaError_t tf32x3_launch(int bn, const CUtensorMap& a, const CUtensorMap& b, const Tf32Params& p, int grid,
                           cudaStream_t s);
 // QKV projection tail (kModeRope): single CTAs or CTA pairs; no output map

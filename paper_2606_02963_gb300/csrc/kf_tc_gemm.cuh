@@ -128,7 +128,6 @@ struct TcCfg {
 
 struct UnitInfo {
   int32_t m0, m_end, n0, g, n_blk;
-  int32_t tile;  // dense: the (row, column) tile of the unit (K splits share it)
 };
 
 // PRE / POST: compiled op programs (Prog<...>) for the chain before / after the
@@ -293,14 +292,8 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     return j < Cfg::kResBlocksA ? smA + sl * kABytes + j * 2048 : smB + sl * Cfg::kBBytes + (j - Cfg::kResBlocksA) * 2048;
   };
 
-  // K split (dense only): the k-blocks of unit u
-  const int32_t ksplit = (!GROUPED && p.k_splits > 1) ? p.k_splits : 1;
-  auto kb_begin = [&](int32_t u) -> int32_t { return ksplit > 1 ? (u % ksplit) * p.num_kb / ksplit : 0; };
-  auto kb_end = [&](int32_t u) -> int32_t { return ksplit > 1 ? (u % ksplit + 1) * p.num_kb / ksplit : p.num_kb; };
-
   auto decode = [&](int32_t u) -> UnitInfo {
     UnitInfo r;
-    r.tile = 0;
     if constexpr (GROUPED) {
       int lo = 0, hi = p.G - 1;  // last g with ustart_s[g] <= u
       while (lo < hi) {
@@ -320,9 +313,8 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
       r.m_end = min(off_s[g + 1], r.m0 + kBM);
       r.n0 = r.n_blk * Cfg::kOutN;
     } else {
-      r.tile = u / ksplit;
-      const int32_t mb = r.tile % p.tiles_m;
-      r.n_blk = r.tile / p.tiles_m;
+      const int32_t mb = u % p.tiles_m;
+      r.n_blk = u / p.tiles_m;
       r.g = 0;
       r.m0 = mb * Cfg::kRowsPerUnit + static_cast<int32_t>(prank) * kBM;  // this CTA's 128 rows
       r.m_end = min(p.M, r.m0 + kBM);
@@ -345,8 +337,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
         const UnitInfo ui = decode(u);
         for (int s = 0; ok && s < sub_tiles; ++s) {
           const int32_t nb0 = ui.n0 + s * BN + static_cast<int32_t>(prank) * Cfg::kBRows;
-          const int32_t kb1 = kb_end(u);
-          for (int32_t kb = kb_begin(u); kb < kb1; ++kb) {
+          for (int32_t kb = 0; kb < p.num_kb; ++kb) {
             const int st = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1;
             if (!mbar_wait(&empty[st], ph ^ 1, abort_flag, p.wait_ns)) {
@@ -441,8 +432,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           }
           tc_fence_after();
           const uint32_t d = tmem + acc * Cfg::kAccStride;
-          const int32_t kb0 = kb_begin(u), kb1 = kb_end(u);
-          for (int32_t kb = kb0; kb < kb1; ++kb) {
+          for (int32_t kb = 0; kb < p.num_kb; ++kb) {
             const int st = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1;
             if (!mbar_wait(&full[st], ph, abort_flag, p.wait_ns)) {
@@ -455,7 +445,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {
               const uint64_t ad = desc_sw128_kmajor(a0 + kk * 32), bd = desc_sw128_kmajor(b0 + kk * 32);
-              const uint32_t accum = (kb != kb0 || kk != 0) ? 1u : 0u;
+              const uint32_t accum = (kb | kk) != 0 ? 1u : 0u;
               if constexpr (CTA2)
                 tc_mma_bf16_pair(d, ad, bd, idesc, accum);
               else
@@ -838,78 +828,16 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             }
           }
         };
-        if (ksplit <= 1) {
-          for (int j = h; j < Cfg::kOutN / 64; j += Cfg::kH) {
-            const int32_t col_lo = pair_col(j);
-            if (col_lo >= p.N) break;  // N is whole heads: the partner exists too
-            const int clo = (col_lo - ui.n0) >> 5;
-            float a[32], b[32];
-            tmem_ld32(tb + clo * 32, a);
-            tmem_ld32(tb + (clo + hh) * 32, b);
-            finish(a, b, col_lo);
-          }
-          release_acc(tl);
-        } else {
-          // K split: add this unit's partial sums into the fp32 rows of the
-          // workspace (vector reductions in L2), then arrive on the counter of
-          // this (tile, quadrant, half); the last split to arrive reads the
-          // complete sums back, zeroes them and finishes the rows
-          float* acc = p.ks_acc;
-          for (int j = h; j < Cfg::kOutN / 64; j += Cfg::kH) {
-            const int32_t col_lo = pair_col(j);
-            if (col_lo >= p.N) break;
-            const int clo = (col_lo - ui.n0) >> 5;
-            float a[32], b[32];
-            tmem_ld32(tb + clo * 32, a);
-            tmem_ld32(tb + (clo + hh) * 32, b);
-            if (row_ok) {
-              float4* pa = reinterpret_cast<float4*>(acc + static_cast<int64_t>(grow) * p.N + col_lo);
-              float4* pb = reinterpret_cast<float4*>(acc + static_cast<int64_t>(grow) * p.N + col_lo + half);
-#pragma unroll
-              for (int u = 0; u < 8; ++u) {
-                atomicAdd(pa + u, make_float4(a[4 * u], a[4 * u + 1], a[4 * u + 2], a[4 * u + 3]));
-                atomicAdd(pb + u, make_float4(b[4 * u], b[4 * u + 1], b[4 * u + 2], b[4 * u + 3]));
-              }
-            }
-          }
-          release_acc(tl);  // the accumulator is free for the next unit before the fix-up
-          if (wrows > 0 && h < Cfg::kOutN / 64) {
-            int32_t* cnt = p.ks_cnt + (static_cast<int64_t>(ui.tile) * 4 + q) * 2 + h;
-            __threadfence();  // this lane's additions are visible before its arrival
-            __syncwarp();
-            int last = 0;
-            if (lane == 0) last = atomicAdd(cnt, 1) == ksplit - 1;
-            last = __shfl_sync(0xffffffffu, last, 0);
-            if (last) {
-              __threadfence();
-              for (int j = h; j < Cfg::kOutN / 64; j += Cfg::kH) {
-                const int32_t col_lo = pair_col(j);
-                if (col_lo >= p.N) break;
-                float a[32], b[32];
-#pragma unroll
-                for (int e = 0; e < 32; ++e) a[e] = b[e] = 0.0f;
-                if (row_ok) {
-                  float4* pa = reinterpret_cast<float4*>(acc + static_cast<int64_t>(grow) * p.N + col_lo);
-                  float4* pb = reinterpret_cast<float4*>(acc + static_cast<int64_t>(grow) * p.N + col_lo + half);
-#pragma unroll
-                  for (int u = 0; u < 8; ++u) {
-                    const float4 x = __ldcg(pa + u), y = __ldcg(pb + u);
-                    a[4 * u] = x.x; a[4 * u + 1] = x.y; a[4 * u + 2] = x.z; a[4 * u + 3] = x.w;
-                    b[4 * u] = y.x; b[4 * u + 1] = y.y; b[4 * u + 2] = y.z; b[4 * u + 3] = y.w;
-                  }
-                  const float4 z = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-#pragma unroll
-                  for (int u = 0; u < 8; ++u) {
-                    __stcg(pa + u, z);
-                    __stcg(pb + u, z);
-                  }
-                }
-                finish(a, b, col_lo);
-              }
-              if (lane == 0) *cnt = 0;  // every split of this launch has arrived
-            }
-          }
+        for (int j = h; j < Cfg::kOutN / 64; j += Cfg::kH) {
+          const int32_t col_lo = pair_col(j);
+          if (col_lo >= p.N) break;  // N is whole heads: the partner exists too
+          const int clo = (col_lo - ui.n0) >> 5;
+          float a[32], b[32];
+          tmem_ld32(tb + clo * 32, a);
+          tmem_ld32(tb + (clo + hh) * 32, b);
+          finish(a, b, col_lo);
         }
+        release_acc(tl);
         ++tl;
       } else if constexpr (MODE == kModeLse) {
         if (!pair_vote(wait_acc(tl))) { ok = false; break; }

@@ -1,0 +1,361 @@
+// kf_tc_qkv_decode.cu -- the QKV projection tail for decode-sized calls (at most
+// 128 tokens): bias + rotary embedding + key / value cache rows, with the K
+// dimension split over the CTAs of a cluster and the partial sums reduced
+// through distributed shared memory (the gpt-oss decode kernel "Bias + RoPE +
+// KV update" of Sec. IV-A, here fused with its GEMM).
+//
+// A decode GEMM reads each weight once; one 256-column tile per CTA over the
+// whole K would keep only N / 256 SMs busy and pay 4 MMAs per 64-wide k-block
+// for all of K.  Here a cluster of S CTAs shares one 256-column tile (four
+// 64-column heads): CTA r multiplies the k-blocks [r K / S, (r + 1) K / S),
+// writes its 128 x 256 fp32 partial from TMEM into its own shared memory (the
+// operand ring, free by then), and after a cluster barrier the epilogue warps
+// of all S CTAs take the tile's (token, head) items in turn: a warp sums the S
+// partials of its item (lane j: columns j and j + d/2 of the head, read from
+// each CTA's shared memory through DSMEM), adds the bias, rotates query and key
+// heads and stores the row to q_out or to the token's cache row.  No global
+// workspace, no atomics, no waits between CTAs other than the two hardware
+// cluster barriers.
+//
+// Warp roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 epilogue.
+#include "kf_internal.h"
+
+namespace kf {
+namespace {
+
+constexpr int kDcThreads = 320;
+constexpr int kDcBM = 128;          // token rows of the MMA (zero-filled past T)
+constexpr int kDcBK = 64;           // K elements per 128-byte row
+constexpr int kDcBN = 256;          // tile columns
+constexpr int kDcPartStride = 257;  // floats per partial row (odd: conflict-free row-per-lane stores)
+
+template <int STAGES>
+struct DcCfg {
+  static constexpr int kABytes = kDcBM * kDcBK * 2;      // 16 KB: 128 token rows (zero-filled past T)
+  static constexpr int kBBytes = kDcBN * kDcBK * 2;    // 32 KB
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr uint32_t kTxBytes = kStageBytes;
+  static constexpr int kPartBytes = kDcBM * kDcPartStride * 4;
+  static constexpr int kRingBytes = STAGES * kStageBytes;
+  static_assert(kPartBytes <= kRingBytes, "the partial fits the ring");
+  static constexpr int kBarBytes = 8 * (2 * STAGES + 2);
+  static constexpr int kSmemBytes = 1024 + kRingBytes + kBarBytes + 64;
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(kDcBM, kDcBN);
+  static_assert(kSmemBytes <= 232448, "shared memory");
+};
+
+__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+
+template <int STAGES>
+__global__ void __launch_bounds__(kDcThreads, 1)
+    kf_qkv_decode_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                         const __grid_constant__ QkvDecodeParams p) {
+  using Cfg = DcCfg<STAGES>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* smB = sm;                                   // B stages first
+  uint8_t* smA = sm + STAGES * Cfg::kBBytes;
+  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: [128 rows][257] fp32
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kRingBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* accf = bars + 2 * STAGES;
+  uint64_t* drain = bars + 2 * STAGES + 1;
+  uint32_t* misc = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 2);
+  uint32_t* tmem_slot = misc;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
+  volatile int* zero_flag = reinterpret_cast<volatile int*>(misc + 2);
+
+  // the split count is the cluster size; refuse any other launch shape before
+  // any barrier, TMEM allocation or copy
+  const uint32_t S = cluster_nctarank();
+  if (S != static_cast<uint32_t>(p.splits) || blockDim.x != kDcThreads || gridDim.x % S != 0 || gridDim.y != 1 ||
+      gridDim.z != 1) {
+    if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
+    return;
+  }
+  const uint32_t r = cluster_ctarank();
+  const int32_t tile = static_cast<int32_t>(blockIdx.x / S);
+  const int32_t n0 = tile * kDcBN;
+  const int32_t kb0 = static_cast<int32_t>(r) * p.num_kb / static_cast<int32_t>(S);
+  const int32_t kb1 = static_cast<int32_t>(r + 1) * p.num_kb / static_cast<int32_t>(S);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accf, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *zero_flag = 0;
+    fence_mbarrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    __syncwarp();
+    tmem_alloc(tmem_slot, kDcBN);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncwarp();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      int32_t it = 0;
+      for (int32_t kb = kb0; kb < kb1; ++kb, ++it) {
+        const int st = it % STAGES;
+        if (!mbar_wait(&empty[st], ((it / STAGES) & 1) ^ 1, abort_flag, p.wait_ns)) {
+          *abort_flag = 1;
+          atomicOr(p.err, kErrWaitProducer);
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&full[st], Cfg::kTxBytes);
+        tma_load_2d(smA + st * Cfg::kABytes, &tmA, &full[st], kb * kDcBK, 0);
+        tma_load_3d(smB + st * Cfg::kBBytes, &tmB, &full[st], kb * kDcBK, n0, 0);
+      }
+      if (!ok)  // copies still in flight land before the ring is reused or the CTA exits
+        for (int32_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
+          mbar_wait(&full[j % STAGES], (j / STAGES) & 1, zero_flag, p.drain_ns);
+    }
+  } else if (warp == 1) {
+    // --------------------------------------------------------------------- MMA
+    if (lane == 0) {
+      const uint32_t idesc = p.ab_f16 ? (Cfg::kIdesc & ~((7u << 7) | (7u << 10))) : Cfg::kIdesc;
+      int32_t it = 0;
+      for (int32_t kb = kb0; kb < kb1; ++kb, ++it) {
+        const int st = it % STAGES;
+        if (!mbar_wait(&full[st], (it / STAGES) & 1, abort_flag, p.wait_ns)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a0 = smem_u32(smA + st * Cfg::kABytes);
+        const uint32_t b0 = smem_u32(smB + st * Cfg::kBBytes);
+#pragma unroll
+        for (int kk = 0; kk < kDcBK / 16; ++kk)
+          tc_mma_bf16(tmem, desc_sw128_kmajor(a0 + kk * 32), desc_sw128_kmajor(b0 + kk * 32), idesc,
+                      (kb != kb0 || kk != 0) ? 1u : 0u);
+        tc_commit(&empty[st]);
+      }
+      if (ok) {
+        tc_commit(accf);
+      } else {
+        *abort_flag = 1;
+        atomicOr(p.err, kErrWaitMma);
+        tc_commit(drain);  // arrives once every MMA issued so far has completed
+        mbar_wait(drain, 0, zero_flag, p.drain_ns);
+      }
+    }
+  } else {
+    // ------------------------------------- epilogue part 1: partial -> own smem
+    const int ew = warp - 2;
+    const int q = warp & 3;                      // TMEM lane quadrant
+    const int hh = ew >> 2;                      // column half: [128 hh, 128 hh + 128)
+    const int32_t row = q * 32 + lane;
+    bool w = mbar_wait(accf, 0, abort_flag, p.wait_ns);
+    w = __all_sync(0xffffffffu, w);
+    if (!w) {
+      *abort_flag = 1;
+      if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+    } else {
+      tc_fence_after();
+      fence_proxy_async_smem();  // the ring's last copies were async-proxy writes
+      const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+      if (q * 32 < p.T) {  // quadrants past the last token have nothing to keep
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(tmem + lane_off + hh * 128 + c * 32, v);
+          if (row < p.T) {
+            float* dst = part + row * kDcPartStride + hh * 128 + c * 32;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) dst[j] = v[j];
+          }
+        }
+      }
+    }
+  }
+  // every CTA's partial is in its shared memory (the ring is idle: all copies
+  // landed and all MMAs completed before the accumulator was signalled)
+  tc_fence_before();
+  __syncwarp();
+  cluster_sync();
+
+  if (warp >= 2 && !*abort_flag) {
+    // --------------------- epilogue part 2: reduce S partials, bias, rotate, store
+    // Items (token, head) of the tile go to the cluster's warps in turn; a warp
+    // takes up to kBatch items at a time and issues all their loads (positions,
+    // cache rows, the S partials, bias, table rows) before any arithmetic or
+    // store, so their latencies overlap.  Lane j holds the pairs j + 32 m of a
+    // head (d / 2 <= 128: m < 4).
+    constexpr int kBatch = 4, kMaxPl = 4;
+    const int ew = warp - 2;
+    const int d = p.rope_d, half = d >> 1, npl = half >> 5;
+    const int heads = kDcBN / d;
+    const int32_t items = p.T * heads;
+    const int32_t stride = static_cast<int32_t>(S) * 8;
+    const uint32_t part_base = smem_u32(part);
+    for (int32_t base = static_cast<int32_t>(r) + static_cast<int32_t>(S) * ew; base < items;
+         base += stride * kBatch) {
+      float a[kBatch][kMaxPl], b[kBatch][kMaxPl];
+      int32_t tt[kBatch], hc[kBatch], pos[kBatch], crow[kBatch];
+      bool live[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int32_t it = base + stride * j;
+        const int32_t t = it / heads, hl = it % heads;
+        tt[j] = t;
+        hc[j] = hl * d;
+        live[j] = it < items && n0 + hl * d < p.N;
+        pos[j] = live[j] ? p.positions[t] : 0;
+        crow[j] = live[j] ? p.cache_rows[t] : 0;
+#pragma unroll
+        for (int m = 0; m < kMaxPl; ++m) {
+          a[j][m] = 0.0f;
+          b[j][m] = 0.0f;
+          if (live[j] && m < npl) {
+            const int i = lane + 32 * m;
+            const uint32_t off = static_cast<uint32_t>((t * kDcPartStride + hl * d + i) * 4);
+            for (uint32_t s2 = 0; s2 < S; ++s2) {
+              const uint32_t bs = mapa_shared(part_base, s2);
+              a[j][m] += ld_cluster_f32(bs + off);
+              b[j][m] += ld_cluster_f32(bs + off + static_cast<uint32_t>(half * 4));
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        if (!live[j]) continue;
+        if (pos[j] < 0 || pos[j] >= p.max_pos || crow[j] < 0 || crow[j] >= p.rows) {
+          if (lane == 0) atomicOr(p.err, kErrBounds);
+          continue;
+        }
+        const int32_t hcol = n0 + hc[j];
+        const bool rotate = hcol < p.rot_cols;
+        void* dst;
+        int64_t dst0;
+        if (hcol < p.q_cols) {
+          dst = p.q_out;
+          dst0 = static_cast<int64_t>(tt[j]) * p.ldq + hcol;
+        } else {
+          dst = rotate ? p.k_cache : p.v_cache;
+          dst0 = static_cast<int64_t>(crow[j]) * p.ld_cache + hcol - (rotate ? p.q_cols : p.rot_cols);
+        }
+#pragma unroll
+        for (int m = 0; m < kMaxPl; ++m) {
+          if (m >= npl) break;
+          const int i = lane + 32 * m;
+          float x0 = a[j][m], x1 = b[j][m];
+          if (p.bias) {
+            x0 += ld_elem(p.bias, p.bias_dtype, hcol + i);
+            x1 += ld_elem(p.bias, p.bias_dtype, hcol + i + half);
+          }
+          if (rotate) {
+            const float c = __ldg(p.cos_t + static_cast<int64_t>(pos[j]) * half + i);
+            const float sn = __ldg(p.sin_t + static_cast<int64_t>(pos[j]) * half + i);
+            const float y0 = fmaf(x0, c, -x1 * sn), y1 = fmaf(x1, c, x0 * sn);
+            x0 = y0;
+            x1 = y1;
+          }
+          if (p.out_dtype == KF_F32) {
+            reinterpret_cast<float*>(dst)[dst0 + i] = x0;
+            reinterpret_cast<float*>(dst)[dst0 + i + half] = x1;
+          } else if (p.out_dtype == KF_BF16) {
+            reinterpret_cast<__nv_bfloat16*>(dst)[dst0 + i] = __float2bfloat16_rn(x0);
+            reinterpret_cast<__nv_bfloat16*>(dst)[dst0 + i + half] = __float2bfloat16_rn(x1);
+          } else {
+            reinterpret_cast<__half*>(dst)[dst0 + i] = __float2half_rn(x0);
+            reinterpret_cast<__half*>(dst)[dst0 + i + half] = __float2half_rn(x1);
+          }
+        }
+      }
+    }
+  }
+  // no CTA leaves while another may still read its shared memory
+  cluster_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kDcBN);
+  }
+}
+
+template <int STAGES>
+cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
+                      cudaStream_t s) {
+  using Cfg = DcCfg<STAGES>;
+  auto kern = kf_qkv_decode_kernel<STAGES>;
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(tiles * p.splits, 1, 1);
+  cfg.blockDim = dim3(kDcThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a, b, p);
+}
+
+}  // namespace
+
+cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
+                              cudaStream_t s) {
+  if (p.splits < 1 || p.splits > 8) return cudaErrorInvalidValue;
+  return launch_dc<4>(a, b, p, tiles, s);
+}
+
+// co-resident clusters of `splits` CTAs for the decode kernel on this device
+cudaError_t qkv_decode_clusters(int splits, int* out) {
+  using Cfg = DcCfg<4>;
+  auto kern = kf_qkv_decode_kernel<4>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(splits, 1, 1);
+  cfg.blockDim = dim3(kDcThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaOccupancyMaxActiveClusters(out, kern, &cfg);
+}
+
+}  // namespace kf

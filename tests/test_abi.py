@@ -197,7 +197,7 @@ def test_qkv_rope_kv_argument_errors_before_any_launch(L):
              X=fake, cos=fake, max_pos=4096, rows=256, bias=None, bdt=kf.KF_BF16, kc=fake):
         return L.kf_qkv_rope_kv(X, fake, xw, H if ldx is None else ldx, H, bias, bdt, fake, fake, cos, fake,
                                 max_pos, T, H, nq, nkv, d, fake, nq * d if ldq is None else ldq, kc, fake,
-                                nkv * d if ldc is None else ldc, rows, out, None, 0, None)
+                                nkv * d if ldc is None else ldc, rows, out, None)
     assert call(d=96) == kf.KF_ERR_UNSUPPORTED          # half a head is not whole 32-column chunks
     assert call(d=512) == kf.KF_ERR_UNSUPPORTED
     assert call(xw=kf.KF_F32) == kf.KF_ERR_UNSUPPORTED  # tensor-core operands only
@@ -215,10 +215,6 @@ def test_qkv_rope_kv_argument_errors_before_any_launch(L):
     assert call(cos=fake + 4) == kf.KF_ERR_MISALIGNED
     assert call(bias=fake, bdt=kf.KF_I32) == kf.KF_ERR_INVALID_ARG
     assert call(T=0, X=None, kc=None) == kf.KF_OK       # empty: nothing read or written
-    # K-split workspace only for decode-sized calls
-    assert L.kf_qkv_rope_kv_workspace(16, 64, 8, 64) >= 16 * 5120 * 4
-    assert L.kf_qkv_rope_kv_workspace(17, 64, 8, 64) == 0
-    assert L.kf_qkv_rope_kv_workspace(0, 64, 8, 64) == 0
 
 
 def test_moe_ffn_act_argument_errors_before_any_launch(L):

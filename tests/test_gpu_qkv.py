@@ -1,9 +1,11 @@
 """GPU parity of the QKV projection tail (bias, rotary embedding of query and key
 heads, key / value cache rows; the gpt-oss decode kernel "Bias + RoPE + KV
-update" of Sec. IV-A, here the epilogue of the projection GEMM) against the
-oracle: decode batches (one 128-row tile, narrow tiles), prefill (CTA pairs,
-ragged last row tile), 128-column heads, fp16 operands, fp32 / fp16 outputs,
-no bias, out-of-range positions, untouched cache rows, repeat runs."""
+update" of Sec. IV-A, here fused with the projection GEMM) against the oracle:
+few-token calls (clusters splitting K, partials reduced in shared memory),
+decode batches up to 128 tokens (one 128-row tile, narrow tiles), prefill (CTA
+pairs, ragged last row tile), 128- and 256-column heads, ragged last column
+tile, fp16 operands, fp32 / fp16 outputs, no bias, out-of-range positions,
+untouched cache rows, repeat runs."""
 import numpy as np
 import pytest
 import torch
@@ -18,23 +20,15 @@ DEV = "cuda"
 SENT = -7.0  # cache rows no token names keep this value
 
 
-def _run(inp, nq, nkv, d, out_dtype=torch.bfloat16, bias=True, sub=None, k_split=True, ws=None):
-    """The library's outputs and the oracle's, on the tokens `sub` (all if None).
-    Decode-sized calls split K unless ``k_split`` is False; the workspace is
-    checked to be zero-filled again afterwards."""
+def _run(inp, nq, nkv, d, out_dtype=torch.bfloat16, bias=True, sub=None):
+    """The library's outputs and the oracle's, on the tokens `sub` (all if None)."""
     rows = int(inp["rows"])
     kc = torch.full((rows, nkv * d), SENT, dtype=out_dtype, device=DEV)
     vc = torch.full((rows, nkv * d), SENT, dtype=out_dtype, device=DEV)
     g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
-    T = inp["X"].shape[0]
-    need = kf.qkv_workspace_bytes(T, nq, nkv, d) if k_split else 0
-    if need and ws is None:
-        ws = torch.zeros(need, dtype=torch.uint8, device=DEV)
     q = kf.qkv_rope_kv(g["X"], g["W"], g["b"] if bias else None, g["positions"], g["cache_rows"], g["cos"],
-                       g["sin"], nq, nkv, d, kc, vc, workspace=ws, k_split=k_split)
+                       g["sin"], nq, nkv, d, kc, vc)
     assert kf.get_device_error()[0] == kf.KF_OK
-    if need:
-        assert int(torch.count_nonzero(ws[:need])) == 0, "workspace not left zero-filled"
     idx = torch.arange(inp["X"].shape[0]) if sub is None else torch.as_tensor(sub)
     rq, rk, rv = oracle.qkv_rope_kv(inp["X"][idx], inp["W"], inp["b"] if bias else None, inp["positions"][idx],
                                     inp["cache_rows"][idx], inp["cos"], inp["sin"], nq, nkv, d, rows)
@@ -56,24 +50,40 @@ def _check(got, ref, idx, what, out_dtype=torch.bfloat16, all_tokens=True):
             assert bool((kc[o] == SENT).all()) and bool((vc[o] == SENT).all()), f"{what}: unnamed rows written"
 
 
-@pytest.mark.parametrize("k_split", [True, False])
-@pytest.mark.parametrize("T", [1, 16, 37, 128])
-def test_decode_gpt_oss_shape(T, k_split):
+@pytest.mark.parametrize("T", [1, 16, 32, 33, 64, 128])
+def test_decode_gpt_oss_shape(T):
+    # <= 32 tokens: clusters splitting K; 33..128: one 128-row tile per CTA
     s = kf_workloads.QKV_SHAPE
     inp = kf_workloads.qkv_generate(T, seed=60 + T)
-    got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"], k_split=k_split)
-    _check(got, ref, idx, f"decode T={T} split={k_split}")
+    got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"])
+    _check(got, ref, idx, f"decode T={T}")
 
 
-def test_decode_calls_reuse_one_workspace():
-    # the workspace is left zero-filled, so back-to-back calls of different
-    # shapes share it without clearing
+@pytest.mark.parametrize("nq,nkv,d", [(8, 2, 128), (2, 1, 256), (3, 2, 64)])
+def test_few_tokens_other_head_sizes_and_ragged_tile(nq, nkv, d):
+    # 128- and 256-column heads (two / four pairs per lane), and 7 heads of 64
+    # (the last 256-column tile holds three heads)
+    inp = kf_workloads.qkv_generate(20, seed=90 + d + nq, H=640, nq=nq, nkv=nkv, d=d, cache_rows=100)
+    got, ref, idx = _run(inp, nq, nkv, d)
+    _check(got, ref, idx, f"few tokens nq={nq} nkv={nkv} d={d}")
+
+
+def test_few_token_path_repeats_bitwise():
+    # the cluster reduction sums the partials in a fixed order
     s = kf_workloads.QKV_SHAPE
-    ws = torch.zeros(kf.qkv_workspace_bytes(16, s["nq"], s["nkv"], s["d"]), dtype=torch.uint8, device=DEV)
-    for i, T in enumerate([16, 3, 1, 9]):
-        inp = kf_workloads.qkv_generate(T, seed=100 + i)
-        got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"], ws=ws)
-        _check(got, ref, idx, f"reuse T={T}")
+    inp = kf_workloads.qkv_generate(7, seed=95)
+    g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
+    outs = []
+    for _ in range(3):
+        kc = torch.zeros(int(inp["rows"]), s["nkv"] * s["d"], dtype=torch.bfloat16, device=DEV)
+        vc = torch.zeros_like(kc)
+        q = kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"], s["nq"],
+                           s["nkv"], s["d"], kc, vc)
+        outs.append((q, kc, vc))
+    torch.cuda.synchronize()
+    for o in outs[1:]:
+        assert all(torch.equal(x, y) for x, y in zip(o, outs[0]))
+    assert kf.get_device_error()[0] == kf.KF_OK
 
 
 @pytest.mark.parametrize("T", [129, 300])
@@ -99,9 +109,10 @@ def test_ragged_last_column_tile():
     _check(got, ref, idx, "7 heads")
 
 
+@pytest.mark.parametrize("T", [8, 64])
 @pytest.mark.parametrize("out_dtype", [torch.float32, torch.float16])
-def test_fp16_operands_and_wide_outputs(out_dtype):
-    inp = kf_workloads.qkv_generate(64, seed=90, H=2880, nq=16, nkv=4, d=64, dtype="f16", cache_rows=300)
+def test_fp16_operands_and_wide_outputs(out_dtype, T):
+    inp = kf_workloads.qkv_generate(T, seed=90, H=2880, nq=16, nkv=4, d=64, dtype="f16", cache_rows=300)
     got, ref, idx = _run(inp, 16, 4, 64, out_dtype=out_dtype)
     _check(got, ref, idx, f"f16 -> {out_dtype}", out_dtype=out_dtype)
 
@@ -122,12 +133,10 @@ def test_out_of_range_position_skips_only_that_token():
     vc = torch.full((rows, nkv * d), SENT, dtype=torch.bfloat16, device=DEV)
     q = torch.full((T, nq * d), SENT, dtype=torch.bfloat16, device=DEV)
     g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
-    ws = torch.zeros(kf.qkv_workspace_bytes(T, nq, nkv, d), dtype=torch.uint8, device=DEV)
     kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"], nq, nkv, d, kc, vc,
-                   q_out=q, workspace=ws)
+                   q_out=q)
     st, raw = kf.get_device_error()
     assert st == kf.KF_ERR_DEVICE_BOUNDS and raw & 8
-    assert int(torch.count_nonzero(ws)) == 0  # a skipped token's partial sums are cleared too
     assert bool((q[bad] == SENT).all())
     r = int(inp["cache_rows"][bad])
     assert bool((kc[r] == SENT).all()) and bool((vc[r] == SENT).all())
