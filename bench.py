@@ -490,7 +490,15 @@ def profile_workload(name, dev, reps):
     """Run one workload through the public API `reps` times (no timing): the
     command that ncu launch lists and captures of that workload are taken on."""
     import paper_2606_02963_gb300 as kf
-    if name.startswith("qkv_T"):
+    if name.startswith("fp32_tf32x3_"):
+        n = int(name[len("fp32_tf32x3_"):])
+        g = torch.Generator("cpu").manual_seed(0)
+        X = torch.randn(n, n, generator=g).to(dev)
+        W = (torch.randn(n, n, generator=g) / n ** 0.5).to(dev)
+        b = torch.randn(n, generator=g).to(dev)
+        for _ in range(reps):
+            kf.fused_gemm(X, W, [("bias", {"p0": b}), ("relu", {})], f32_mode="tf32x3")
+    elif name.startswith("qkv_T"):
         T = int(name[5:])
         sh = kf_workloads.QKV_SHAPE
         inp = kf_workloads.qkv_generate(T, seed=0, prefill=T > 128, cache_rows=max(8192, T))
@@ -561,8 +569,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=16)
     ap.add_argument("--profile-workload", default=None,
                     help="run one workload's calls --steps times, untimed (the command ncu captures of it use): "
-                         "bf16_gelu_scale_residual, bf16_scale_rowlse, bf16_groupnorm_swish, moe_T64, moe_T4096 or "
-                         "qkv_T<tokens>")
+                         "bf16_gelu_scale_residual, bf16_scale_rowlse, bf16_groupnorm_swish, moe_T64, moe_T4096, "
+                         "qkv_T<tokens> or fp32_tf32x3_<n>")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
