@@ -309,8 +309,6 @@ cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecod
   if (!configured[dev]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
@@ -336,26 +334,37 @@ cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const 
   return launch_dc<4>(a, b, p, tiles, s);
 }
 
-// co-resident clusters of `splits` CTAs for the decode kernel on this device
+// co-resident clusters of `splits` CTAs for the decode kernel on the current
+// device (queried once per device and cluster size)
 cudaError_t qkv_decode_clusters(int splits, int* out) {
-  using Cfg = DcCfg<4>;
-  auto kern = kf_qkv_decode_kernel<4>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(splits, 1, 1);
-  cfg.blockDim = dim3(kDcThreads, 1, 1);
-  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaOccupancyMaxActiveClusters(out, kern, &cfg);
+  static int cache[64][9] = {};  // 0: not yet queried
+  if (splits < 1 || splits > 8) return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (cache[dev][splits] == 0) {
+    using Cfg = DcCfg<4>;
+    auto kern = kf_qkv_decode_kernel<4>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(splits, 1, 1);
+    cfg.blockDim = dim3(kDcThreads, 1, 1);
+    cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = splits;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int nc = 0;
+    e = cudaOccupancyMaxActiveClusters(&nc, kern, &cfg);
+    if (e != cudaSuccess) return e;
+    cache[dev][splits] = nc > 0 ? nc : -1;
+  }
+  *out = cache[dev][splits] > 0 ? cache[dev][splits] : 0;
+  return cudaSuccess;
 }
 
 }  // namespace kf
