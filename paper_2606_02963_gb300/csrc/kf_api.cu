@@ -771,8 +771,10 @@ kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows
 //   topk_ids i32 [T k] | topk_w f32 [T k] | offsets i32 [E+1] | sorted_token i32 [T k]
 //   | sorted_w f32 [T k] | Xg bf16 [T k, H] | h bf16 [T k, I] | Yacc f32 [T, H]
 struct MoeLayout {
-  size_t ids, w, off, st, sw, xg, h, yacc, pos, yp, total;
+  size_t ids, w, off, st, sw, cnt, xg, h, yacc, pos, yp, total;
 };
+// pairs from which the routing sort runs on many blocks
+constexpr int64_t kSortMultiBlockPairs = 2048;
 // deterministic mode adds: pair_pos i32 [T k] | Yp f32 [T k, H]
 static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags = 0) {
   MoeLayout L;
@@ -788,6 +790,7 @@ static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t 
   L.off = take(static_cast<size_t>(E + 1) * 4);
   L.st = take(P * 4);
   L.sw = take(P * 4);
+  L.cnt = take(static_cast<size_t>(route_sort_mb_blocks(static_cast<int32_t>(P))) * static_cast<size_t>(E) * 4);
   L.xg = take(P * static_cast<size_t>(H) * 2);
   L.h = take(P * static_cast<size_t>(I) * 2);
   L.yacc = take(static_cast<size_t>(T) * static_cast<size_t>(H) * 4);
@@ -868,7 +871,11 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
   if (!det && cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
   st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, ids, w, s));
   if (st != KF_OK) return st;
-  st = cuda_status(route_sort_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos, s, true));
+  if (P >= kSortMultiBlockPairs)
+    st = cuda_status(route_sort_mb_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos,
+                                          reinterpret_cast<int32_t*>(ws + L.cnt), s, true));
+  else
+    st = cuda_status(route_sort_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos, s, true));
   if (st != KF_OK) return st;
   // gate/up: h = silu(Xg W_gate[e]^T) * (Xg W_up[e]^T), rows gathered by token
   {

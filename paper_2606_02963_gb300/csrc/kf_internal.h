@@ -151,6 +151,12 @@ cudaError_t route_topk_launch(const float* logits, int32_t T, int32_t E, int32_t
 cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
                               int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
                               cudaStream_t s, bool pdl);
+// Multi-block stable sort (same order), for many pairs: `counts` is scratch of
+// route_sort_mb_blocks(T k) x E int32
+cudaError_t route_sort_mb_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
+                                 int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
+                                 int32_t* counts, cudaStream_t s, bool pdl);
+int32_t route_sort_mb_blocks(int32_t P);
 cudaError_t moe_finalize_launch(const float* Yp, const int32_t* pair_pos, int64_t T, int32_t k, int64_t H, void* Y,
                                 cudaStream_t s, bool pdl);
 // MoE block tail: R_out = bf16(R + y), Y = bf16(rmsnorm(R_out) * gamma) per token;

@@ -288,6 +288,110 @@ cudaError_t route_sort_launch(const int32_t* ids, const float* w, int32_t T, int
                   sorted_token, sorted_w, pair_pos);
 }
 
+// Multi-block form of the same stable counting sort, for many pairs (one SM
+// issuing every scattered store of the one-block kernel takes ~24 us at 16 K
+// pairs).  Pairs go in chunks of kSortChunk, one chunk per block:
+//   route_count_kernel    per-block expert histogram -> counts[b][e]
+//   route_scatter_kernel  block b's first slot of expert e = (pairs of experts
+//                         < e) + (pairs of expert e in blocks < b); within the
+//                         block, warps hold 32 consecutive pairs each, ranked by
+//                         __match_any_sync and offset by the earlier warps' counts.
+// The order is the one-block kernel's (increasing pair index within an expert).
+constexpr int kSortChunk = 256;  // pairs per block = threads per block
+
+__global__ void __launch_bounds__(kSortChunk) route_count_kernel(const int32_t* __restrict__ ids, int32_t P,
+                                                                 int32_t E, int32_t* __restrict__ counts) {
+  griddep_wait();  // after the routing kernel (programmatic launch)
+  griddep_launch_dependents();
+  __shared__ int32_t cnt[kMaxExperts];
+  for (int e = threadIdx.x; e < E; e += blockDim.x) cnt[e] = 0;
+  __syncthreads();
+  const int32_t p = blockIdx.x * kSortChunk + threadIdx.x;
+  if (p < P) atomicAdd(&cnt[ids[p]], 1);
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) counts[static_cast<int64_t>(blockIdx.x) * E + e] = cnt[e];
+}
+
+__global__ void __launch_bounds__(kSortChunk) route_scatter_kernel(const int32_t* __restrict__ ids,
+                                                                   const float* __restrict__ w, int32_t P,
+                                                                   int32_t E, int32_t k,
+                                                                   const int32_t* __restrict__ counts,
+                                                                   int32_t* offsets, int32_t* sorted_token,
+                                                                   float* sorted_w, int32_t* pair_pos) {
+  griddep_wait();  // after the count kernel (programmatic launch)
+  griddep_launch_dependents();
+  constexpr int kW = kSortChunk / 32;
+  __shared__ int32_t base[kMaxExperts];   // this block's first slot per expert
+  __shared__ int32_t tot[kMaxExperts];
+  __shared__ int32_t wcnt[kW][kMaxExperts];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int32_t nb = gridDim.x, b = blockIdx.x;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int32_t before = 0, all = 0;
+    for (int32_t bb = 0; bb < nb; ++bb) {
+      const int32_t c = counts[static_cast<int64_t>(bb) * E + e];
+      if (bb < b) before += c;
+      all += c;
+    }
+    base[e] = before;
+    tot[e] = all;
+  }
+  for (int i = threadIdx.x; i < kW * E; i += blockDim.x) wcnt[i / E][i % E] = 0;
+  __syncthreads();
+  if (warp == 0) {
+    // exclusive scan of the expert totals (lane l owns experts l*per .. l*per+per-1)
+    const int per = (E + 31) / 32;
+    int32_t local = 0;
+    for (int i = 0; i < per; ++i) {
+      const int e = lane * per + i;
+      if (e < E) local += tot[e];
+    }
+    int32_t incl = local;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int32_t o = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += o;
+    }
+    int32_t run = incl - local;
+    for (int i = 0; i < per; ++i) {
+      const int e = lane * per + i;
+      if (e < E) {
+        base[e] += run;
+        if (b == 0) offsets[e] = run;
+        run += tot[e];
+      }
+    }
+    if (b == 0 && lane == 31) offsets[E] = run;
+  }
+  // ranks within the warp's 32 pairs, and the warp's count per expert
+  const int32_t p = b * kSortChunk + threadIdx.x;
+  const bool valid = p < P;
+  const int32_t e = valid ? ids[p] : E + lane;  // invalid lanes never match a real expert
+  const uint32_t peers = __match_any_sync(0xffffffffu, e);
+  const int rank = __popc(peers & ((1u << lane) - 1u));
+  if (valid && rank == 0) wcnt[warp][e] = __popc(peers);
+  __syncthreads();
+  if (valid) {
+    int32_t pos = base[e] + rank;
+    for (int ww = 0; ww < warp; ++ww) pos += wcnt[ww][e];
+    sorted_token[pos] = p / k;
+    sorted_w[pos] = w[p];
+    if (pair_pos) pair_pos[p] = pos;
+  }
+}
+
+cudaError_t route_sort_mb_launch(const int32_t* ids, const float* w, int32_t T, int32_t E, int32_t k,
+                                 int32_t* offsets, int32_t* sorted_token, float* sorted_w, int32_t* pair_pos,
+                                 int32_t* counts, cudaStream_t s, bool pdl) {
+  const int32_t P = T * k;
+  const int nb = (P + kSortChunk - 1) / kSortChunk;
+  cudaError_t e = launch_k(route_count_kernel, dim3(nb), dim3(kSortChunk), 0, s, pdl, ids, P, E, counts);
+  if (e != cudaSuccess) return e;
+  return launch_k(route_scatter_kernel, dim3(nb), dim3(kSortChunk), 0, s, true, ids, w, P, E, k,
+                  static_cast<const int32_t*>(counts), offsets, sorted_token, sorted_w, pair_pos);
+}
+int32_t route_sort_mb_blocks(int32_t P) { return (P + kSortChunk - 1) / kSortChunk; }
+
 // ------------------------------------------------ deterministic MoE finalize
 // Y[t, :] = bf16( sum_{j = 0..k-1} Yp[pair_pos[t*k + j], :] ), slot order fixed.
 __global__ void moe_finalize_kernel(const float4* __restrict__ Yp, const int32_t* __restrict__ pair_pos, int64_t T,
