@@ -755,6 +755,10 @@ kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows
   if (!aligned16(A) || !aligned16(B) || lda % 8 != 0 || ldb % 8 != 0 || b_group_stride % 8 != 0)
     return KF_ERR_MISALIGNED;
   if (a_row_index && K % 8 != 0) return KF_ERR_MISALIGNED;
+  if (a_row_index) {
+    if (!workspace || !aligned16(workspace) || ws_bytes < grouped_ws_bytes(rows_total, K, true))
+      return KF_ERR_WORKSPACE;
+  }
   DevInfo di;
   st = device_info(&di);
   if (st != KF_OK) return st;
