@@ -173,10 +173,8 @@ kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int
  *   C is [rows_total x N] (stride ldc), bf16 or fp32; with
  *   ROW_SCALE_SCATTER_ADD C is the fp32 scatter target instead.
  *   A, B bf16; alignment rules as kf_fused_gemm (also b_group_stride % 8 == 0).
- *   A gather reads the rows in place by index (TMA tile::gather4 in the GEMM's
- *   producer warp); kf_grouped_gemm_workspace() is 0 and workspace may be NULL.
- *   Bad device-side offsets/indices set KF_ERR_DEVICE_BOUNDS in the error word
- *   (a row with an index outside [0, a_rows) is computed from row 0).
+ *   workspace: kf_grouped_gemm_workspace() bytes (the gathered rows live there).
+ *   Bad device-side offsets/indices set KF_ERR_DEVICE_BOUNDS in the error word.
  */
 kf_status kf_grouped_gemm(const void* A, int32_t a_dtype, int64_t lda, int64_t a_rows, const int32_t* a_row_index,
                           const void* B, int32_t b_dtype, int64_t ldb, int64_t b_group_stride,

@@ -396,10 +396,7 @@ struct GroupedArgs {
 };
 
 size_t grouped_ws_bytes(int64_t rows_total, int64_t K, bool gathered) {
-  (void)rows_total;
-  (void)K;
-  (void)gathered;
-  return 0;  // gathered rows are read in place by the GEMM
+  return gathered ? align_up(static_cast<size_t>(rows_total) * static_cast<size_t>(K) * 2, 256) : 0;
 }
 
 // Per-group bias and the gated SwiGLU of the MoE path (see TcParams).
@@ -414,17 +411,21 @@ struct GroupExtras {
 // so the launches here may be programmatic dependents of it.
 kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cudaStream_t s, const DevInfo& di,
                        bool pdl, const GroupExtras* ex = nullptr) {
-  (void)ws;
-  // gathered A rows: the GEMM's producer warp reads them straight from A by index
-  // (TMA tile::gather4 with one-row boxes), no gathered copy
-  const bool gather = g.a_row_index != nullptr;
+  const void* A = g.A;
+  int64_t lda = g.lda;
+  if (g.a_row_index) {
+    kf_status st =
+        cuda_status(gather_rows_launch(g.A, g.lda, g.a_rows, g.a_row_index, g.rows_total, g.K, ws, di.err, s, pdl));
+    if (st != KF_OK) return st;
+    A = ws;
+    lda = g.K;
+  }
   const int bn = pick_grouped_outn(pl.mode, g.N, g.rows_total, g.G, di.nsm);
   if (bn == 0) return KF_ERR_UNSUPPORTED;
   const int outn = pl.mode == kModeSwiglu ? bn / 2 : bn;
   const int64_t nb = pl.mode == kModeSwiglu ? 2 * g.N : g.N;
   CUtensorMap ma, mb;
-  kf_status st = gather ? make_map(&ma, g.A, g.K, g.a_rows, g.lda * 2, 1, 0, 1, 2)
-                        : make_map(&ma, g.A, g.K, g.rows_total, g.lda * 2, 1, 0, kBM, 2);
+  kf_status st = make_map(&ma, A, g.K, g.rows_total, lda * 2, 1, 0, kBM, 2);
   if (st != KF_OK) return st;
   st = make_map(&mb, g.B, g.K, nb, g.ldb * 2, g.G, g.b_group_stride * 2, mode_box(pl.mode, bn), 3);
   if (st != KF_OK) return st;
@@ -442,8 +443,6 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   p.ldc = g.ldc;
   p.c_dtype = g.c_dtype;
   p.c_vec_ok = aligned16(g.C) && (g.ldc * elt_size(g.c_dtype)) % 16 == 0;
-  p.a_rows = g.a_row_index;
-  p.a_src_rows = static_cast<int32_t>(g.a_rows);
   p.row_scale = pl.row_scale;
   p.row_dst = pl.row_dst;
   p.dst_rows = static_cast<int32_t>(pl.dst_rows);
@@ -461,7 +460,8 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
   CUtensorMap mc;  // grouped outputs are masked per group: plain stores, no TMA map
   std::memset(&mc, 0, sizeof(mc));
-  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, mc, p, grid, s, pdl));
+  // after the gather (when there is one) the GEMM follows a library kernel
+  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, mc, p, grid, s, pdl || g.a_row_index != nullptr));
 }
 
 }  // namespace
@@ -771,7 +771,7 @@ kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows
 //   topk_ids i32 [T k] | topk_w f32 [T k] | offsets i32 [E+1] | sorted_token i32 [T k]
 //   | sorted_w f32 [T k] | Xg bf16 [T k, H] | h bf16 [T k, I] | Yacc f32 [T, H]
 struct MoeLayout {
-  size_t ids, w, off, st, sw, cnt, h, yacc, pos, yp, total;
+  size_t ids, w, off, st, sw, cnt, xg, h, yacc, pos, yp, total;
 };
 // pairs from which the routing sort runs on many blocks
 constexpr int64_t kSortMultiBlockPairs = 2048;
@@ -791,6 +791,7 @@ static MoeLayout moe_layout(int64_t T, int64_t H, int64_t I, int32_t E, int32_t 
   L.st = take(P * 4);
   L.sw = take(P * 4);
   L.cnt = take(static_cast<size_t>(route_sort_mb_blocks(static_cast<int32_t>(P))) * static_cast<size_t>(E) * 4);
+  L.xg = take(P * static_cast<size_t>(H) * 2);
   L.h = take(P * static_cast<size_t>(I) * 2);
   L.yacc = take(static_cast<size_t>(T) * static_cast<size_t>(H) * 4);
   L.pos = L.yp = 0;
@@ -859,6 +860,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
   auto* off = reinterpret_cast<int32_t*>(ws + L.off);
   auto* stok = reinterpret_cast<int32_t*>(ws + L.st);
   auto* sw = reinterpret_cast<float*>(ws + L.sw);
+  void* xg = ws + L.xg;
   void* h = ws + L.h;
   auto* yacc = reinterpret_cast<float*>(ws + L.yacc);
   const int64_t P = T * k;
@@ -893,7 +895,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
       ex.sw_limit = act->limit;
       ex.sw_c = act->linear_offset;
     }
-    st = grouped_core(g, pl, nullptr, s, di, true, &ex);
+    st = grouped_core(g, pl, xg, s, di, true, &ex);
     if (st != KF_OK) return st;
   }
   if (det) {

@@ -102,11 +102,6 @@ struct TcParams {
   void* v_cache;
   int64_t ld_cache;
   int32_t kv_vec_ok;    // caches allow 16-byte stores of 32-column chunks
-  // grouped GEMMs with gathered A rows: row r of the A operand is row a_rows[r]
-  // of the A tensor (tmA then has one-row boxes: the producer warp gathers four
-  // rows per lane with tile::gather4), or null
-  const int32_t* a_rows;
-  int32_t a_src_rows;   // rows of the A tensor (an index outside sets the bounds bit)
   // grouped GEMMs: bf16 bias of the unit's group added to the accumulator
   // before anything else (column j of group g at gbias[g * gbias_ld + j]; for
   // SwiGLU the up half's bias follows at + b_rows), or null

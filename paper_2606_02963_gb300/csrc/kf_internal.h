@@ -166,6 +166,8 @@ constexpr int64_t kAddRmsNormMaxH = 8192;
 cudaError_t moe_add_rmsnorm_launch(const float* yacc, const float* yp, const int32_t* pair_pos, int32_t k, int64_t T,
                                    int64_t H, const void* R, const void* gamma, float eps, void* R_out, void* Y,
                                    cudaStream_t s, bool pdl);
+cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
+                               int64_t K, void* out, uint32_t* err, cudaStream_t s, bool pdl);
 cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s, bool pdl);
 
 }  // namespace kf

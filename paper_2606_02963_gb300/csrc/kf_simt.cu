@@ -508,6 +508,37 @@ cudaError_t moe_add_rmsnorm_launch(const float* yacc, const float* yp, const int
                   reinterpret_cast<uint2*>(R_out), reinterpret_cast<uint2*>(Y));
 }
 
+// ----------------------------------------------------------------- row gather
+// out[r, :] = A[idx[r], :] (16-byte vectors; K % 8 == 0 bf16).  An index out of
+// range writes a zero row and sets the bounds bit of the error word.
+__global__ void gather_rows_kernel(const uint4* __restrict__ A, int64_t lda_v, int64_t a_rows,
+                                   const int32_t* __restrict__ idx, int64_t rows, int64_t kv,
+                                   uint4* __restrict__ out, uint32_t* err) {
+  griddep_wait();  // after the library kernel this one follows (programmatic launch)
+  griddep_launch_dependents();
+  const int64_t total = rows * kv;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / kv, c = i % kv;
+    const int32_t src = idx[r];
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (src >= 0 && src < a_rows)
+      v = __ldg(A + src * lda_v + c);
+    else if (c == 0)
+      atomicOr(err, kErrBounds);
+    out[i] = v;
+  }
+}
+
+cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
+                               int64_t K, void* out, uint32_t* err, cudaStream_t s, bool pdl) {
+  if (rows == 0) return cudaSuccess;
+  const int64_t kv = K / 8, total = rows * kv;
+  int blocks = static_cast<int>(std::min<int64_t>((total + 255) / 256, 148 * 16));
+  return launch_k(gather_rows_kernel, dim3(blocks), dim3(256), 0, s, pdl, reinterpret_cast<const uint4*>(A), lda / 8,
+                  a_rows, idx, rows, kv, reinterpret_cast<uint4*>(out), err);
+}
+
 // ------------------------------------------------------------ fp32 -> bf16
 __global__ void cvt_f32_bf16_kernel(const float4* __restrict__ in, uint2* __restrict__ out, int64_t n4) {
   griddep_wait();  // after the library kernel this one follows (programmatic launch)

@@ -330,58 +330,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (GROUPED && !CTA2 && p.a_rows) {
-      // Gathered A rows: the whole warp produces; lane l gathers rows 4l..4l+3
-      // of each 128-row A box (rows past the operand's end repeat its last row;
-      // their results belong to no group and are never stored), lane 0 arms the
-      // barrier and loads B.
-      int32_t it = 0;
-      bool ok = true;
-      for (int32_t u = unit0; ok && u < total; u += unit_step) {
-        const UnitInfo ui = decode(u);
-        int32_t src[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          src[i] = p.a_rows[min(ui.m0 + 4 * lane + i, p.M - 1)];
-          if (src[i] < 0 || src[i] >= p.a_src_rows) {
-            atomicOr(p.err, kErrBounds);
-            src[i] = 0;
-          }
-        }
-        for (int32_t kb = 0; kb < p.num_kb; ++kb) {
-          const int st = it % STAGES;
-          const uint32_t ph = (it / STAGES) & 1;
-          bool w = true;
-          if (lane == 0) w = mbar_wait(&empty[st], ph ^ 1, abort_flag, p.wait_ns);
-          w = __shfl_sync(0xffffffffu, w, 0);
-          if (!w) {
-            if (lane == 0) {
-              *abort_flag = 1;
-              atomicOr(p.err, kErrWaitProducer);
-            }
-            ok = false;
-            break;
-          }
-          if (lane == 0) mbar_arrive_expect_tx(&full[st], Cfg::kTxBytes);
-          __syncwarp();
-          uint8_t* a = smA + st * kABytes;
-          uint8_t* b = smB + st * Cfg::kBBytes;
-          tma_gather4(a + lane * 4 * 128, &tmA, &full[st], kb * kBK, src[0], src[1], src[2], src[3]);
-          if (lane == 0) {
-            if constexpr (MODE == kModeSwiglu) {
-              tma_load_3d(b, &tmB, &full[st], kb * kBK, ui.n0, ui.g);
-              tma_load_3d(b + Cfg::kOutN * 128, &tmB, &full[st], kb * kBK, p.b_rows + ui.n0, ui.g);
-            } else {
-              tma_load_3d(b, &tmB, &full[st], kb * kBK, ui.n0, ui.g);
-            }
-          }
-          ++it;
-        }
-      }
-      if (!ok && lane == 0)  // copies still in flight land before the CTA exits
-        for (int32_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
-          mbar_wait(&full[j % STAGES], (j / STAGES) & 1, zero_flag, p.drain_ns);
-    } else if (lane == 0) {
+    if (lane == 0) {
       int32_t it = 0, rt_units = 0;
       bool ok = true;
       for (int32_t u = unit0; ok && u < total; u += unit_step) {

@@ -49,22 +49,6 @@ def _groups(sizes, K, nb, seed, w_std=0.05):
     return rows, off, B, g
 
 
-def test_grouped_gather_index_out_of_range_is_reported():
-    # the gathered rows are read in place by index; an index outside A sets the
-    # bounds bit (that row is computed from row 0) and faults nothing
-    N, K, T = 96, 128, 40
-    rows, off, B, g = _groups([30, 34], K, 2 * N, seed=5)
-    A = torch.randn(T, K, generator=g).to(torch.bfloat16)
-    idx = torch.randint(0, T, (rows,), generator=g, dtype=torch.int32)
-    idx[17] = T + 5
-    h = kf.grouped_gemm(A.to(DEV), B.to(DEV), off.to(DEV), N, [("swiglu", {})], row_index=idx.to(DEV))
-    st, raw = kf.get_device_error()
-    assert st == kf.KF_ERR_DEVICE_BOUNDS and raw & 8
-    good = [r for r in range(rows) if r != 17]
-    ref = oracle.grouped_gemm(A, B, off.numpy(), N, [("swiglu", {})], row_index=idx.clamp(max=T - 1).numpy())
-    check_bf16(h[good], ref[good], "gather with one bad index")
-
-
 @pytest.mark.parametrize("sizes", [[0, 1, 7, 129, 0, 300], [8] * 32, [0, 0, 5], [256]])
 def test_grouped_swiglu_with_gather(sizes):
     N, K = 288, 200
