@@ -1137,7 +1137,7 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
     }
     const CUtensorMapDataType dt = xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     CUtensorMap ma, mb;
-    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, kBM, 2, dt);
+    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, 32, 2, dt);  // 32-row A boxes (T <= 32)
     if (st != KF_OK) return st;
     st = make_map(&mb, W, H, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, 256, 3, dt);
     if (st != KF_OK) return st;

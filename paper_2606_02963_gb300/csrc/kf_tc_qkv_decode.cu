@@ -24,20 +24,26 @@ namespace kf {
 namespace {
 
 constexpr int kDcThreads = 320;
-constexpr int kDcBM = 128;          // token rows of the MMA (zero-filled past T)
+constexpr int kDcBM = 128;          // rows of the MMA (only the first T are tokens)
+constexpr int kDcARows = 32;        // token rows staged per k-block (T <= 32)
 constexpr int kDcBK = 64;           // K elements per 128-byte row
 constexpr int kDcBN = 256;          // tile columns
 constexpr int kDcPartStride = 257;  // floats per partial row (odd: conflict-free row-per-lane stores)
 
 template <int STAGES>
 struct DcCfg {
-  static constexpr int kABytes = kDcBM * kDcBK * 2;      // 16 KB: 128 token rows (zero-filled past T)
+  // A: 32 token rows per k-block (4 KB).  The MMA reads 128 rows from there; the
+  // 96 past the box are the next stages' bytes and feed only accumulator rows
+  // past T, which are never stored (A stages come first, so the reads stay in
+  // the ring).
+  static constexpr int kABytes = kDcARows * kDcBK * 2;
   static constexpr int kBBytes = kDcBN * kDcBK * 2;    // 32 KB
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr uint32_t kTxBytes = kStageBytes;
-  static constexpr int kPartBytes = kDcBM * kDcPartStride * 4;
+  static constexpr int kPartBytes = kDcARows * kDcPartStride * 4;
   static constexpr int kRingBytes = STAGES * kStageBytes;
   static_assert(kPartBytes <= kRingBytes, "the partial fits the ring");
+  static_assert(STAGES * kABytes + kBBytes >= kDcBM * kDcBK * 2, "the MMA's 128-row reads stay in the ring");
   static constexpr int kBarBytes = 8 * (2 * STAGES + 2);
   static constexpr int kSmemBytes = 1024 + kRingBytes + kBarBytes + 64;
   static constexpr uint32_t kIdesc = idesc_bf16_f32(kDcBM, kDcBN);
@@ -57,9 +63,9 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   using Cfg = DcCfg<STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* smB = sm;                                   // B stages first
-  uint8_t* smA = sm + STAGES * Cfg::kBBytes;
-  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: [128 rows][257] fp32
+  uint8_t* smA = sm;                                   // A stages first (see DcCfg)
+  uint8_t* smB = sm + STAGES * Cfg::kABytes;
+  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: [32 rows][257] fp32
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kRingBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
@@ -74,7 +80,7 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   // any barrier, TMEM allocation or copy
   const uint32_t S = cluster_nctarank();
   if (S != static_cast<uint32_t>(p.splits) || blockDim.x != kDcThreads || gridDim.x % S != 0 || gridDim.y != 1 ||
-      gridDim.z != 1) {
+      gridDim.z != 1 || p.T > kDcARows) {
     if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
     return;
   }
@@ -331,7 +337,7 @@ cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecod
 cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
                               cudaStream_t s) {
   if (p.splits < 1 || p.splits > 8) return cudaErrorInvalidValue;
-  return launch_dc<4>(a, b, p, tiles, s);
+  return launch_dc<6>(a, b, p, tiles, s);
 }
 
 // co-resident clusters of `splits` CTAs for the decode kernel on the current
@@ -343,8 +349,8 @@ cudaError_t qkv_decode_clusters(int splits, int* out) {
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (cache[dev][splits] == 0) {
-    using Cfg = DcCfg<4>;
-    auto kern = kf_qkv_decode_kernel<4>;
+    using Cfg = DcCfg<6>;
+    auto kern = kf_qkv_decode_kernel<6>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
