@@ -1,5 +1,5 @@
 // kf_tc_qkv_decode.cu -- the QKV projection tail for decode-sized calls (at most
-// 128 tokens): bias + rotary embedding + key / value cache rows, with the K
+// 32 tokens): bias + rotary embedding + key / value cache rows, with the K
 // dimension split over the CTAs of a cluster and the partial sums reduced
 // through distributed shared memory (the gpt-oss decode kernel "Bias + RoPE +
 // KV update" of Sec. IV-A, here fused with its GEMM).
@@ -8,8 +8,8 @@
 // whole K would keep only N / 256 SMs busy and pay 4 MMAs per 64-wide k-block
 // for all of K.  Here a cluster of S CTAs shares one 256-column tile (four
 // 64-column heads): CTA r multiplies the k-blocks [r K / S, (r + 1) K / S),
-// writes its 128 x 256 fp32 partial from TMEM into its own shared memory (the
-// operand ring, free by then), and after a cluster barrier the epilogue warps
+// writes the T token rows of its 128 x 256 fp32 partial from TMEM into its own
+// shared memory (the operand ring, free by then), and after a cluster barrier the epilogue warps
 // of all S CTAs take the tile's (token, head) items in turn: a warp sums the S
 // partials of its item (lane j: columns j and j + d/2 of the head, read from
 // each CTA's shared memory through DSMEM), adds the bias, rotates query and key
