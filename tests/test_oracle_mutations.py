@@ -1,6 +1,7 @@
 """Plant one mistake at a time in a copy of the oracle (on the CPU) and check that
-the pins in test_oracle_pins.py catch it.  This shows the pins constrain every
-part of the oracle the parity tests rely on."""
+the pins in test_oracle_pins.py catch it, and, on their own, the hand-worked
+examples of test_golden.py.  This shows both constrain every part of the oracle
+the parity tests rely on."""
 import os
 import subprocess
 import sys
@@ -56,8 +57,10 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     mpath = tmp_path / "kf_oracle.c"
     mpath.write_text(src.replace(old, new))
     env = dict(os.environ, KF_ORACLE_SRC=str(mpath), KF_ORACLE_BUILD=str(tmp_path / "_build"))
-    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-rf", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py"),
+                        os.path.join(ROOT, "tests", "test_golden.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
-    assert "failed" in r.stdout, r.stdout[-2000:]
+    assert r.returncode != 0, f"nothing caught mutation {name}:\n{r.stdout[-2000:]}"
+    for f in ("test_oracle_pins.py", "test_golden.py"):
+        assert f"FAILED tests/{f}" in r.stdout, f"{f} did not catch mutation {name}:\n{r.stdout[-2000:]}"
