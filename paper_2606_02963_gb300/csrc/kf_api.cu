@@ -1060,8 +1060,9 @@ namespace {
 // per tile, as for the dense store variants.
 // Calls of at most this many tokens take the cluster-split decode kernel; above
 // it the per-token reduction costs more than the whole-tile kernel's MMAs
-// (measured at 64 and 128 tokens)
-constexpr int64_t kQkvClusterMaxT = 32;
+// (gpt-oss-20b shape: 48 tokens 20.5 against 22.5 us, 64 tokens 24.6 against 22.5)
+constexpr int64_t kQkvClusterMaxT = 48;
+static_assert(kQkvClusterMaxT <= kQkvDecodeMaxRows, "the decode kernel's token box");
 
 int pick_rope_bn(int64_t M, int64_t N, int d, int nsm, bool cta2) {
   static const int cand[] = {256, 128, 64};
@@ -1130,14 +1131,14 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
     int S = 1;
     for (int cand : {8, 6, 4, 2}) {
       int nc = 0;
-      if (cand <= num_kb && qkv_decode_clusters(cand, &nc) == cudaSuccess && nc >= tiles) {
+      if (cand <= num_kb && qkv_decode_clusters(T, cand, &nc) == cudaSuccess && nc >= tiles) {
         S = cand;
         break;
       }
     }
     const CUtensorMapDataType dt = xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     CUtensorMap ma, mb;
-    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, 32, 2, dt);  // 32-row A boxes (T <= 32)
+    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, qkv_decode_box_rows(T), 2, dt);  // token boxes of 32 or 64 rows
     if (st != KF_OK) return st;
     st = make_map(&mb, W, H, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, 256, 3, dt);
     if (st != KF_OK) return st;

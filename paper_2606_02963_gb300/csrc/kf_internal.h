@@ -90,9 +90,12 @@ struct QkvDecodeParams {
   uint64_t wait_ns;
   uint64_t drain_ns;
 };
+// few-token QKV tail: at most this many tokens; A boxes of qkv_decode_box_rows(T) rows
+constexpr int kQkvDecodeMaxRows = 64;
 cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
                               cudaStream_t s);
-cudaError_t qkv_decode_clusters(int splits, int* out);
+int qkv_decode_box_rows(int64_t T);
+cudaError_t qkv_decode_clusters(int64_t T, int splits, int* out);
 cudaError_t tf32x3_launch(int bn, const CUtensorMap& a, const CUtensorMap& b, const Tf32Params& p, int grid,
                           cudaStream_t s);
 // QKV projection tail (kModeRope): single CTAs or CTA pairs; no output map

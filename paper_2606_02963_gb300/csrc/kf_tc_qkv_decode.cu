@@ -1,5 +1,5 @@
 // kf_tc_qkv_decode.cu -- the QKV projection tail for decode-sized calls (at most
-// 32 tokens): bias + rotary embedding + key / value cache rows, with the K
+// 64 tokens): bias + rotary embedding + key / value cache rows, with the K
 // dimension split over the CTAs of a cluster and the partial sums reduced
 // through distributed shared memory (the gpt-oss decode kernel "Bias + RoPE +
 // KV update" of Sec. IV-A, here fused with its GEMM).
@@ -15,7 +15,13 @@
 // each CTA's shared memory through DSMEM), adds the bias, rotates query and key
 // heads and stores the row to q_out or to the token's cache row.  No global
 // workspace, no atomics, no waits between CTAs other than the two hardware
-// cluster barriers.
+// cluster barriers.  While the MMAs run, the epilogue warps already load what
+// their first items need besides the sums (positions, cache rows, bias, the
+// table rows of the positions), so that after the barrier only the partial sums
+// are read.
+//
+// Token rows are staged in boxes of ROWS = 32 (six-stage ring) or 64 rows
+// (five stages): the box is what limits the tokens of a call.
 //
 // Warp roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 epilogue.
 #include "kf_internal.h"
@@ -25,22 +31,22 @@ namespace {
 
 constexpr int kDcThreads = 320;
 constexpr int kDcBM = 128;          // rows of the MMA (only the first T are tokens)
-constexpr int kDcARows = 32;        // token rows staged per k-block (T <= 32)
 constexpr int kDcBK = 64;           // K elements per 128-byte row
 constexpr int kDcBN = 256;          // tile columns
 constexpr int kDcPartStride = 257;  // floats per partial row (odd: conflict-free row-per-lane stores)
 
-template <int STAGES>
+template <int ROWS, int STAGES>
 struct DcCfg {
-  // A: 32 token rows per k-block (4 KB).  The MMA reads 128 rows from there; the
-  // 96 past the box are the next stages' bytes and feed only accumulator rows
-  // past T, which are never stored (A stages come first, so the reads stay in
-  // the ring).
-  static constexpr int kABytes = kDcARows * kDcBK * 2;
+  // A: ROWS token rows per k-block (4 or 8 KB).  The MMA reads 128 rows from
+  // there; the ones past the box are the next stages' bytes and feed only
+  // accumulator rows past T, which are never stored (A stages come first, so
+  // the reads stay in the ring).
+  static_assert(ROWS == 32 || ROWS == 64, "token box");
+  static constexpr int kABytes = ROWS * kDcBK * 2;
   static constexpr int kBBytes = kDcBN * kDcBK * 2;    // 32 KB
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr uint32_t kTxBytes = kStageBytes;
-  static constexpr int kPartBytes = kDcARows * kDcPartStride * 4;
+  static constexpr int kPartBytes = ROWS * kDcPartStride * 4;
   static constexpr int kRingBytes = STAGES * kStageBytes;
   static_assert(kPartBytes <= kRingBytes, "the partial fits the ring");
   static_assert(STAGES * kABytes + kBBytes >= kDcBM * kDcBK * 2, "the MMA's 128-row reads stay in the ring");
@@ -56,16 +62,59 @@ __device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
   return v;
 }
 
-template <int STAGES>
+// Operands of one (token, head) item that do not depend on the sums: lane j
+// holds pairs j + 32 m of the head (d / 2 <= 128: m < 4).
+constexpr int kBatch = 4, kMaxPl = 4;
+struct DcItem {
+  int32_t t, hcol, pos, crow;
+  bool live, ok, rotate;
+  float b0[kMaxPl], b1[kMaxPl], c[kMaxPl], s[kMaxPl];
+};
+
+// Items it = base + stride j (j < kBatch) of a tile: token it / heads, head
+// it % heads.  All loads are issued before any is used.  A position or cache row
+// out of range clears `ok` (the item is then reported and skipped, and no table
+// row is read for it).
+__device__ __forceinline__ void dc_load_items(const QkvDecodeParams& p, int32_t n0, int32_t base, int32_t stride,
+                                              int32_t items, int heads, int lane, DcItem (&it)[kBatch]) {
+  const int d = p.rope_d, half = d >> 1, npl = half >> 5;
+#pragma unroll
+  for (int j = 0; j < kBatch; ++j) {
+    const int32_t idx = base + stride * j;
+    const int32_t hl = idx % heads;
+    it[j].t = idx / heads;
+    it[j].hcol = n0 + hl * d;
+    it[j].live = idx < items && it[j].hcol < p.N;
+    it[j].pos = it[j].live ? p.positions[it[j].t] : 0;
+    it[j].crow = it[j].live ? p.cache_rows[it[j].t] : 0;
+  }
+#pragma unroll
+  for (int j = 0; j < kBatch; ++j) {
+    it[j].ok = it[j].live && it[j].pos >= 0 && it[j].pos < p.max_pos && it[j].crow >= 0 && it[j].crow < p.rows;
+    it[j].rotate = it[j].hcol < p.rot_cols;
+#pragma unroll
+    for (int m = 0; m < kMaxPl; ++m) {
+      const int i = lane + 32 * m;
+      const bool use = it[j].ok && m < npl;
+      it[j].b0[m] = use && p.bias ? ld_elem(p.bias, p.bias_dtype, it[j].hcol + i) : 0.0f;
+      it[j].b1[m] = use && p.bias ? ld_elem(p.bias, p.bias_dtype, it[j].hcol + i + half) : 0.0f;
+      const bool tab = use && it[j].rotate;
+      it[j].c[m] = tab ? __ldg(p.cos_t + static_cast<int64_t>(it[j].pos) * half + i) : 1.0f;
+      it[j].s[m] = tab ? __ldg(p.sin_t + static_cast<int64_t>(it[j].pos) * half + i) : 0.0f;
+    }
+  }
+}
+
+template <int ROWS, int STAGES>
 __global__ void __launch_bounds__(kDcThreads, 1)
     kf_qkv_decode_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                          const __grid_constant__ QkvDecodeParams p) {
-  using Cfg = DcCfg<STAGES>;
+  using Cfg = DcCfg<ROWS, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* smA = sm;                                   // A stages first (see DcCfg)
   uint8_t* smB = sm + STAGES * Cfg::kABytes;
-  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: [32 rows][257] fp32
+  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: [ROWS][257] fp32
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kRingBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
@@ -80,7 +129,7 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   // any barrier, TMEM allocation or copy
   const uint32_t S = cluster_nctarank();
   if (S != static_cast<uint32_t>(p.splits) || blockDim.x != kDcThreads || gridDim.x % S != 0 || gridDim.y != 1 ||
-      gridDim.z != 1 || p.T > kDcARows) {
+      gridDim.z != 1 || p.T > ROWS) {
     if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
     return;
   }
@@ -91,6 +140,13 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   const int32_t kb1 = static_cast<int32_t>(r + 1) * p.num_kb / static_cast<int32_t>(S);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  // (token, head) items of the tile go to the cluster's epilogue warps in turn;
+  // a warp takes up to kBatch items at a time
+  const int heads = kDcBN / p.rope_d;
+  const int32_t items = p.T * heads;
+  const int32_t stride = static_cast<int32_t>(S) * 8;
+  const int32_t first = static_cast<int32_t>(r) + static_cast<int32_t>(S) * (warp - 2);
+  DcItem batch[kBatch];  // the epilogue warp's current items
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -175,6 +231,8 @@ __global__ void __launch_bounds__(kDcThreads, 1)
     const int q = warp & 3;                      // TMEM lane quadrant
     const int hh = ew >> 2;                      // column half: [128 hh, 128 hh + 128)
     const int32_t row = q * 32 + lane;
+    // the first batch's operands load while the MMAs run
+    if (first < items) dc_load_items(p, n0, first, stride, items, heads, lane, batch);
     bool w = mbar_wait(accf, 0, abort_flag, p.wait_ns);
     w = __all_sync(0xffffffffu, w);
     if (!w) {
@@ -205,39 +263,23 @@ __global__ void __launch_bounds__(kDcThreads, 1)
 
   if (warp >= 2 && !*abort_flag) {
     // --------------------- epilogue part 2: reduce S partials, bias, rotate, store
-    // Items (token, head) of the tile go to the cluster's warps in turn; a warp
-    // takes up to kBatch items at a time and issues all their loads (positions,
-    // cache rows, the S partials, bias, table rows) before any arithmetic or
-    // store, so their latencies overlap.  Lane j holds the pairs j + 32 m of a
-    // head (d / 2 <= 128: m < 4).
-    constexpr int kBatch = 4, kMaxPl = 4;
-    const int ew = warp - 2;
+    // A warp issues the DSMEM loads of all its batch's partial sums before any
+    // arithmetic or store, so their latencies overlap; the other operands of
+    // the first batch are in registers already.
     const int d = p.rope_d, half = d >> 1, npl = half >> 5;
-    const int heads = kDcBN / d;
-    const int32_t items = p.T * heads;
-    const int32_t stride = static_cast<int32_t>(S) * 8;
     const uint32_t part_base = smem_u32(part);
-    for (int32_t base = static_cast<int32_t>(r) + static_cast<int32_t>(S) * ew; base < items;
-         base += stride * kBatch) {
+    for (int32_t base = first; base < items; base += stride * kBatch) {
+      if (base != first) dc_load_items(p, n0, base, stride, items, heads, lane, batch);
       float a[kBatch][kMaxPl], b[kBatch][kMaxPl];
-      int32_t tt[kBatch], hc[kBatch], pos[kBatch], crow[kBatch];
-      bool live[kBatch];
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) {
-        const int32_t it = base + stride * j;
-        const int32_t t = it / heads, hl = it % heads;
-        tt[j] = t;
-        hc[j] = hl * d;
-        live[j] = it < items && n0 + hl * d < p.N;
-        pos[j] = live[j] ? p.positions[t] : 0;
-        crow[j] = live[j] ? p.cache_rows[t] : 0;
 #pragma unroll
         for (int m = 0; m < kMaxPl; ++m) {
           a[j][m] = 0.0f;
           b[j][m] = 0.0f;
-          if (live[j] && m < npl) {
+          if (batch[j].ok && m < npl) {
             const int i = lane + 32 * m;
-            const uint32_t off = static_cast<uint32_t>((t * kDcPartStride + hl * d + i) * 4);
+            const uint32_t off = static_cast<uint32_t>((batch[j].t * kDcPartStride + (batch[j].hcol - n0) + i) * 4);
             for (uint32_t s2 = 0; s2 < S; ++s2) {
               const uint32_t bs = mapa_shared(part_base, s2);
               a[j][m] += ld_cluster_f32(bs + off);
@@ -248,34 +290,28 @@ __global__ void __launch_bounds__(kDcThreads, 1)
       }
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) {
-        if (!live[j]) continue;
-        if (pos[j] < 0 || pos[j] >= p.max_pos || crow[j] < 0 || crow[j] >= p.rows) {
+        if (!batch[j].live) continue;
+        if (!batch[j].ok) {
           if (lane == 0) atomicOr(p.err, kErrBounds);
           continue;
         }
-        const int32_t hcol = n0 + hc[j];
-        const bool rotate = hcol < p.rot_cols;
+        const int32_t hcol = batch[j].hcol;
         void* dst;
         int64_t dst0;
         if (hcol < p.q_cols) {
           dst = p.q_out;
-          dst0 = static_cast<int64_t>(tt[j]) * p.ldq + hcol;
+          dst0 = static_cast<int64_t>(batch[j].t) * p.ldq + hcol;
         } else {
-          dst = rotate ? p.k_cache : p.v_cache;
-          dst0 = static_cast<int64_t>(crow[j]) * p.ld_cache + hcol - (rotate ? p.q_cols : p.rot_cols);
+          dst = batch[j].rotate ? p.k_cache : p.v_cache;
+          dst0 = static_cast<int64_t>(batch[j].crow) * p.ld_cache + hcol - (batch[j].rotate ? p.q_cols : p.rot_cols);
         }
 #pragma unroll
         for (int m = 0; m < kMaxPl; ++m) {
           if (m >= npl) break;
           const int i = lane + 32 * m;
-          float x0 = a[j][m], x1 = b[j][m];
-          if (p.bias) {
-            x0 += ld_elem(p.bias, p.bias_dtype, hcol + i);
-            x1 += ld_elem(p.bias, p.bias_dtype, hcol + i + half);
-          }
-          if (rotate) {
-            const float c = __ldg(p.cos_t + static_cast<int64_t>(pos[j]) * half + i);
-            const float sn = __ldg(p.sin_t + static_cast<int64_t>(pos[j]) * half + i);
+          float x0 = a[j][m] + batch[j].b0[m], x1 = b[j][m] + batch[j].b1[m];
+          if (batch[j].rotate) {
+            const float c = batch[j].c[m], sn = batch[j].s[m];
             const float y0 = fmaf(x0, c, -x1 * sn), y1 = fmaf(x1, c, x0 * sn);
             x0 = y0;
             x1 = y1;
@@ -303,11 +339,11 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   }
 }
 
-template <int STAGES>
+template <int ROWS, int STAGES>
 cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
                       cudaStream_t s) {
-  using Cfg = DcCfg<STAGES>;
-  auto kern = kf_qkv_decode_kernel<STAGES>;
+  using Cfg = DcCfg<ROWS, STAGES>;
+  auto kern = kf_qkv_decode_kernel<ROWS, STAGES>;
   static bool configured[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -332,44 +368,54 @@ cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecod
   return cudaLaunchKernelEx(&cfg, kern, a, b, p);
 }
 
-}  // namespace
-
-cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
-                              cudaStream_t s) {
-  if (p.splits < 1 || p.splits > 8) return cudaErrorInvalidValue;
-  return launch_dc<6>(a, b, p, tiles, s);
+// co-resident clusters of `splits` CTAs of one variant on the current device
+template <int ROWS, int STAGES>
+cudaError_t clusters_dc(int splits, int* out) {
+  using Cfg = DcCfg<ROWS, STAGES>;
+  auto kern = kf_qkv_decode_kernel<ROWS, STAGES>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(splits, 1, 1);
+  cfg.blockDim = dim3(kDcThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaOccupancyMaxActiveClusters(out, kern, &cfg);
 }
 
-// co-resident clusters of `splits` CTAs for the decode kernel on the current
-// device (queried once per device and cluster size)
-cudaError_t qkv_decode_clusters(int splits, int* out) {
-  static int cache[64][9] = {};  // 0: not yet queried
-  if (splits < 1 || splits > 8) return cudaErrorInvalidValue;
+}  // namespace
+
+// token boxes of 32 rows (six stages) up to 32 tokens, of 64 rows (five) above
+cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
+                              cudaStream_t s) {
+  if (p.splits < 1 || p.splits > 8 || p.T < 1 || p.T > kQkvDecodeMaxRows) return cudaErrorInvalidValue;
+  return p.T <= 32 ? launch_dc<32, 6>(a, b, p, tiles, s) : launch_dc<64, 5>(a, b, p, tiles, s);
+}
+
+int qkv_decode_box_rows(int64_t T) { return T <= 32 ? 32 : 64; }
+
+// co-resident clusters of `splits` CTAs for the decode kernel variant that
+// serves T tokens (queried once per device, variant and cluster size)
+cudaError_t qkv_decode_clusters(int64_t T, int splits, int* out) {
+  static int cache[64][2][9] = {};  // 0: not yet queried
+  if (splits < 1 || splits > 8 || T < 1 || T > kQkvDecodeMaxRows) return cudaErrorInvalidValue;
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (cache[dev][splits] == 0) {
-    using Cfg = DcCfg<6>;
-    auto kern = kf_qkv_decode_kernel<6>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(splits, 1, 1);
-    cfg.blockDim = dim3(kDcThreads, 1, 1);
-    cfg.dynamicSmemBytes = Cfg::kSmemBytes;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = splits;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
+  const int v = T <= 32 ? 0 : 1;
+  if (cache[dev][v][splits] == 0) {
     int nc = 0;
-    e = cudaOccupancyMaxActiveClusters(&nc, kern, &cfg);
+    cudaError_t e = v == 0 ? clusters_dc<32, 6>(splits, &nc) : clusters_dc<64, 5>(splits, &nc);
     if (e != cudaSuccess) return e;
-    cache[dev][splits] = nc > 0 ? nc : -1;
+    cache[dev][v][splits] = nc > 0 ? nc : -1;
   }
-  *out = cache[dev][splits] > 0 ? cache[dev][splits] : 0;
+  *out = cache[dev][v][splits] > 0 ? cache[dev][v][splits] : 0;
   return cudaSuccess;
 }
 

@@ -1,8 +1,9 @@
 """GPU parity of the QKV projection tail (bias, rotary embedding of query and key
 heads, key / value cache rows; the gpt-oss decode kernel "Bias + RoPE + KV
 update" of Sec. IV-A, here fused with the projection GEMM) against the oracle:
-few-token calls (clusters splitting K, partials reduced in shared memory),
-decode batches up to 128 tokens (one 128-row tile, narrow tiles), prefill (CTA
+few-token calls (clusters splitting K, partials reduced in shared memory; token
+boxes of 32 and 64 rows), decode batches up to 128 tokens (one 128-row tile,
+narrow tiles), prefill (CTA
 pairs, ragged last row tile), 128- and 256-column heads, ragged last column
 tile, fp16 operands, fp32 / fp16 outputs, no bias, out-of-range positions,
 untouched cache rows, repeat runs."""
@@ -50,28 +51,31 @@ def _check(got, ref, idx, what, out_dtype=torch.bfloat16, all_tokens=True):
             assert bool((kc[o] == SENT).all()) and bool((vc[o] == SENT).all()), f"{what}: unnamed rows written"
 
 
-@pytest.mark.parametrize("T", [1, 16, 32, 33, 64, 128])
+@pytest.mark.parametrize("T", [1, 16, 32, 33, 48, 49, 64, 128])
 def test_decode_gpt_oss_shape(T):
-    # <= 32 tokens: clusters splitting K; 33..128: one 128-row tile per CTA
+    # <= 48 tokens: clusters splitting K (32-row token boxes up to 32 tokens,
+    # 64-row ones above); 49..128: one 128-row tile per CTA
     s = kf_workloads.QKV_SHAPE
     inp = kf_workloads.qkv_generate(T, seed=60 + T)
     got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"])
     _check(got, ref, idx, f"decode T={T}")
 
 
+@pytest.mark.parametrize("T", [20, 45])
 @pytest.mark.parametrize("nq,nkv,d", [(8, 2, 128), (2, 1, 256), (3, 2, 64)])
-def test_few_tokens_other_head_sizes_and_ragged_tile(nq, nkv, d):
+def test_few_tokens_other_head_sizes_and_ragged_tile(nq, nkv, d, T):
     # 128- and 256-column heads (two / four pairs per lane), and 7 heads of 64
     # (the last 256-column tile holds three heads)
-    inp = kf_workloads.qkv_generate(20, seed=90 + d + nq, H=640, nq=nq, nkv=nkv, d=d, cache_rows=100)
+    inp = kf_workloads.qkv_generate(T, seed=90 + d + nq + T, H=640, nq=nq, nkv=nkv, d=d, cache_rows=100)
     got, ref, idx = _run(inp, nq, nkv, d)
     _check(got, ref, idx, f"few tokens nq={nq} nkv={nkv} d={d}")
 
 
-def test_few_token_path_repeats_bitwise():
+@pytest.mark.parametrize("T", [7, 45])
+def test_few_token_path_repeats_bitwise(T):
     # the cluster reduction sums the partials in a fixed order
     s = kf_workloads.QKV_SHAPE
-    inp = kf_workloads.qkv_generate(7, seed=95)
+    inp = kf_workloads.qkv_generate(T, seed=95 + T)
     g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
     outs = []
     for _ in range(3):
@@ -123,8 +127,9 @@ def test_no_bias_fp32_output():
     _check(got, ref, idx, "no bias", out_dtype=torch.float32)
 
 
-def test_out_of_range_position_skips_only_that_token():
-    T, nq, nkv, d = 12, 4, 2, 64
+@pytest.mark.parametrize("T", [12, 40, 100])
+def test_out_of_range_position_skips_only_that_token(T):
+    nq, nkv, d = 4, 2, 64
     inp = kf_workloads.qkv_generate(T, seed=92, H=256, nq=nq, nkv=nkv, d=d, max_pos=512, cache_rows=128)
     bad = 7
     inp["positions"][bad] = 512  # one past the tables
