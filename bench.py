@@ -182,15 +182,63 @@ def time_steps(fn, steps, warmup, flush, stream, host_slack=True):
     return sum(a.elapsed_time(b) for a, b in evs) / steps
 
 
+def time_steps_rotating(fns, steps, warmup, stream):
+    """Mean device time (ms) per step of `steps` steps run back to back between
+    one pair of events; step i calls fns[i % len(fns)], each on its own copy of
+    the inputs (the copies together are larger than L2, so no step finds its
+    inputs there).  A device-side sleep before the start event gives the host a
+    head start: it must finish enqueueing every step before the sleep ends, so
+    the device never waits for it (checked; the sleep doubles until it holds).
+    Returns (ms, {"sleep_ms", "host_enqueue_ms"})."""
+    n = len(fns)
+    for i in range(warmup):
+        fns[i % n]()
+    torch.cuda.synchronize()
+    t_end = time.perf_counter() + SETTLE_S
+    i = 0
+    while time.perf_counter() < t_end and i < 4000:
+        fns[i % n]()
+        i += 1
+        if i % 16 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    cycles = 4_000_000
+    for _ in range(4):
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        torch.cuda._sleep(cycles)
+        s1.record(stream)
+        a.record(stream)
+        h0 = time.perf_counter()
+        for j in range(steps):
+            fns[j % n]()
+        host_ms = (time.perf_counter() - h0) * 1e3
+        b.record(stream)
+        torch.cuda.synchronize()
+        sleep_ms = s0.elapsed_time(s1)
+        if host_ms < 0.9 * sleep_ms:
+            break
+        cycles *= 2
+    return a.elapsed_time(b) / steps, {"sleep_ms": round(sleep_ms, 3), "host_enqueue_ms": round(host_ms, 3)}
+
+
+HEADLINE_COPIES = 6  # x 58.7 MB of inputs and output per step: 352 MB, L2 is 129 MB
+
+
 # --------------------------------------------------------------- workloads
+def dense_chain(wl, d):
+    chain = []
+    for kind, prm in kf_workloads.chain_spec(wl):
+        chain.append((kind, {k: (d[v] if k in ("p0", "p1") else v) for k, v in prm.items()}))
+    return chain
+
+
 def dense_setup(name, dev):
     inp = kf_workloads.generate(name, seed=0)
     d = {k: v.to(dev) for k, v in inp.items()}
     wl = kf_workloads.WORKLOADS[name]
-    chain = []
-    for kind, prm in kf_workloads.chain_spec(wl):
-        chain.append((kind, {k: (d[v] if k in ("p0", "p1") else v) for k, v in prm.items()}))
-    return wl, inp, d, chain
+    return wl, inp, d, dense_chain(wl, d)
 
 
 def dense_bytes(name, wl):
@@ -271,18 +319,27 @@ def run_kf(args, rank, world, dev):
         kf.fused_gemm(d["X"], d["W"], chain, out=out)
         hout.copy_(out, non_blocking=True)
 
+    # copies of the inputs and the output for back-to-back steps
+    copies = [d] + [{k2: v.clone() for k2, v in d.items()} for _ in range(HEADLINE_COPIES - 1)]
+    outs = [out] + [torch.empty_like(out) for _ in range(HEADLINE_COPIES - 1)]
+    chains = [chain] + [dense_chain(wl, c) for c in copies[1:]]
+    rot = [(lambda c=c, ch=ch, o=o: kf.fused_gemm(c["X"], c["W"], ch, out=o)) for c, ch, o in zip(copies, chains, outs)]
+
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     with Clocks(dev.index if dev.index is not None else 0) as clk:
-        ms = time_steps(step, args.steps, args.warmup, flush, stream)
+        ms, rot_info = time_steps_rotating(rot, args.steps, args.warmup, stream)
     clocks = clk.summary()
+    ms_iso = time_steps(step, args.steps, args.warmup, flush, stream)
     ms_e2e = time_steps(e2e_step, max(3, args.steps // 2), args.warmup, flush, stream, host_slack=False)
-    ms, ms_e2e = reduce_max_over_ranks([ms, ms_e2e], dev, world)
+    ms, ms_iso, ms_e2e = reduce_max_over_ranks([ms, ms_iso, ms_e2e], dev, world)
     value = whole_job_tflops(flops, ms, world)
     e2e_value = whole_job_tflops(flops, ms_e2e, world)
-    ms_eager = time_steps(eager_dense(MAIN, d), args.steps, args.warmup, flush, stream)
-    ms_cublas = time_steps(lambda: torch.matmul(d["X"], d["W"].t()), args.steps, args.warmup, flush, stream)
+    ms_eager, _ = time_steps_rotating([eager_dense(MAIN, c) for c in copies], args.steps, args.warmup, stream)
+    ms_cublas, _ = time_steps_rotating([(lambda c=c: torch.matmul(c["X"], c["W"].t())) for c in copies],
+                                       args.steps, args.warmup, stream)
+    del copies, outs, chains, rot
     traffic = stored_traffic("dense_store_gelu_1024x4096x4096")
     achieved = flops / (ms * 1e-3) / 1e12
     line = {
@@ -291,7 +348,9 @@ def run_kf(args, rank, world, dev):
         "warmup": args.warmup, "ms_per_step": round(ms, 5), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16 operands, fp32 accumulate", "data": "synthetic (seeded)",
         "config": {"workload": MAIN, "M": wl.M, "N": wl.N, "K": wl.K,
-                   "chain": "bias -> gelu_tanh -> x2.0 -> +R", "l2": "flushed (256 MiB write) before each step",
+                   "chain": "bias -> gelu_tanh -> x2.0 -> +R",
+                   "l2": (f"inputs larger than L2: steps rotate over {HEADLINE_COPIES} copies of the inputs and "
+                          f"output ({HEADLINE_COPIES} x 58.7 MB), run back to back between one pair of events"),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peaks["bf16"],
                      "peak_src": f"{peaks['src']} bf16 burst", "unit": "TFLOP/s",
@@ -301,6 +360,9 @@ def run_kf(args, rank, world, dev):
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "eager": {"ms_per_step": round(ms_eager, 5), "speedup": round(ms_eager / ms, 3),
                   "cublas_gemm_only_ms": round(ms_cublas, 5)},
+        "isolated": {"ms_per_step": round(ms_iso, 5),
+                     "how": "one step at a time after a 256 MiB L2 flush and a 100 us device sleep"},
+        "timing": rot_info,
         "gpu_launches": args.steps,
         "clocks": clocks,
     }
@@ -455,33 +517,47 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
         kc = torch.zeros(rows, nkv * dh, dtype=torch.bfloat16, device=dev)
         vc = torch.zeros_like(kc)
         q = torch.empty(T, nq * dh, dtype=torch.bfloat16, device=dev)
-        fused = lambda: kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"],
-                                       nq, nkv, dh, kc, vc, q_out=q)
         y = torch.empty(T, Nq, dtype=torch.bfloat16, device=dev)
-        pos, crow = g["positions"].long(), g["cache_rows"].long()
-
-        def unfused():
-            kf.fused_gemm(g["X"], g["W"], [("bias", {"p0": g["b"]})], out=y)
-            hd = y.view(T, nq + 2 * nkv, dh)
-            c, sn = g["cos"][pos][:, None, :], g["sin"][pos][:, None, :]
-            x = hd[:, :nq + nkv].float()
-            a, b = x[..., :dh // 2], x[..., dh // 2:]
-            r = torch.cat([a * c - b * sn, b * c + a * sn], -1).to(torch.bfloat16)
-            q.copy_(r[:, :nq].reshape(T, -1))
-            kc.index_copy_(0, crow, r[:, nq:].reshape(T, -1))
-            vc.index_copy_(0, crow, hd[:, nq + nkv:].reshape(T, -1))
-        ms = time_steps(fused, steps, args.warmup, flush, stream)
-        ms_u = time_steps(unfused, steps, args.warmup, flush, stream)
-        ms_c = time_steps(lambda: torch.matmul(g["X"], g["W"].t()), steps, args.warmup, flush, stream)
         byts = Nq * Hq * 2 + T * Hq * 2 + Nq * 2 + T * Nq * 2 + 2 * T * (dh // 2) * 4
         flops = 2.0 * T * Nq * Hq
+        # steps rotate over copies of the inputs, together more than twice L2
+        ncop = max(2, -(-300_000_000 // byts))
+        gs = [g] + [{k2: v.clone() for k2, v in g.items()} for _ in range(ncop - 1)]
+
+        def make_fused(gc):
+            return lambda: kf.qkv_rope_kv(gc["X"], gc["W"], gc["b"], gc["positions"], gc["cache_rows"], gc["cos"],
+                                          gc["sin"], nq, nkv, dh, kc, vc, q_out=q)
+
+        def make_unfused(gc):
+            pos, crow = gc["positions"].long(), gc["cache_rows"].long()
+
+            def unfused():
+                kf.fused_gemm(gc["X"], gc["W"], [("bias", {"p0": gc["b"]})], out=y)
+                hd = y.view(T, nq + 2 * nkv, dh)
+                c, sn = gc["cos"][pos][:, None, :], gc["sin"][pos][:, None, :]
+                x = hd[:, :nq + nkv].float()
+                a, b = x[..., :dh // 2], x[..., dh // 2:]
+                r = torch.cat([a * c - b * sn, b * c + a * sn], -1).to(torch.bfloat16)
+                q.copy_(r[:, :nq].reshape(T, -1))
+                kc.index_copy_(0, crow, r[:, nq:].reshape(T, -1))
+                vc.index_copy_(0, crow, hd[:, nq + nkv:].reshape(T, -1))
+            return unfused
+
+        ms, _ = time_steps_rotating([make_fused(gc) for gc in gs], steps, args.warmup, stream)
+        ms_u, _ = time_steps_rotating([make_unfused(gc) for gc in gs], steps, args.warmup, stream)
+        ms_c, _ = time_steps_rotating([(lambda gc=gc: torch.matmul(gc["X"], gc["W"].t())) for gc in gs], steps,
+                                      args.warmup, stream)
+        ms_iso = time_steps(make_fused(g), steps, args.warmup, flush, stream)
         t_roof = max(flops / (peaks["bf16"] * 1e12), byts / (peaks["hbm"] * 1e9)) * 1e3
         bound = "hbm" if byts / (peaks["hbm"] * 1e9) > flops / (peaks["bf16"] * 1e12) else "tensor"
         res[f"qkv_rope_kv_T{T}"] = {"tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
                                    "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
                                    "cluster_split": T <= 48, "unfused_ms": round(ms_u, 5),
                                    "speedup_vs_unfused": round(ms_u / ms, 3), "cublas_gemm_only_ms": round(ms_c, 5),
+                                   "isolated_ms": round(ms_iso, 5),
+                                   "l2": f"steps rotate over {ncop} copies of the inputs, back to back",
                                    "launches_per_step": 1}
+        del gs
         del g, inp, kc, vc
     return res
 
