@@ -246,7 +246,7 @@ kf_status kf_moe_ffn_act(const void* X, const float* logits, const void* W_gu, c
 /*
  * kf_moe_ffn_add_rmsnorm -- the MoE block tail fused into the MoE finalize
  *                          (Sec. IV-A: the gpt-oss decode kernels "Fused Add +
- *                          RMSNorm" and "MoE finalize"; Sec. VI: optimising the
+ *                          RMSNorm" and "MoE finalize"; Sec. V: optimising the
  *                          kernels of one block together)
  *
  *   The routed expert FFN of kf_moe_ffn_ex (same arguments and flags), whose

@@ -22,7 +22,7 @@
  *     with the intermediate h rounded to bf16 (the down GEMM consumes bf16 h);
  *     the "MoE finalize" kernel of Table 1 is the routing-weighted sum over j.
  *   - the block tail after the MoE FFN (Sec. IV-A: "Fused Add + RMSNorm" and
- *     "MoE finalize" of the gpt-oss decode path; Sec. VI: fusing kernels of one
+ *     "MoE finalize" of the gpt-oss decode path; Sec. V: fusing kernels of one
  *     block) is the residual add and RMS normalisation of the new residual
  *     stream: R_out = bf16(R + Y), normed_j = R_out_j / sqrt(mean(R_out^2) + eps)
  *     * gamma_j -- the norm reads the stored (bf16) residual, as the next layer
