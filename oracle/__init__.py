@@ -19,7 +19,7 @@ FP contraction):
 
 Chains are lists of ``(kind, params)``: kinds ``bias, scale, relu, gelu_tanh,
 silu, sigmoid, residual_add, row_logsumexp, groupnorm, swiglu,
-row_scale_scatter_add, mish, leaky_relu, mul, row_scale``; params ``p0, p1`` (tensors),
+row_scale_scatter_add, mish, leaky_relu, mul, row_scale, row_sum``; params ``p0, p1`` (tensors),
 ``scalar, eps, groups``.
 """
 from __future__ import annotations
@@ -47,6 +47,7 @@ KINDS = {
     "bias": 0, "scale": 1, "relu": 2, "gelu_tanh": 3, "silu": 4, "sigmoid": 5,
     "residual_add": 6, "row_logsumexp": 7, "groupnorm": 8, "swiglu": 9,
     "row_scale_scatter_add": 10, "mish": 11, "leaky_relu": 12, "mul": 13, "row_scale": 14,
+    "row_sum": 15,
 }
 
 
@@ -161,7 +162,8 @@ def fused_gemm(X, W, chain: Sequence[Tuple[str, Dict]], rows: Optional[Sequence[
                nthreads: int = 0) -> np.ndarray:
     """Y = chain(X W^T) in fp64.  X [M, K], W [N, K] (fp32 or bf16).
 
-    Returns float64 [len(rows) or M, N] (or [.., 1] after a row log-sum-exp);
+    Returns float64 [len(rows) or M, N] (or [.., 1] after a row log-sum-exp or
+    a row sum);
     output row r is input row ``rows[r]``."""
     lib = _load()
     keep: list = []
@@ -180,7 +182,7 @@ def fused_gemm(X, W, chain: Sequence[Tuple[str, Dict]], rows: Optional[Sequence[
     lib.orc_fused_gemm(_ptr(x), xt, K, _ptr(w), wt, K, M, N, K, ctypes.cast(ops, ctypes.c_void_p),
                        len(chain), None if rows_a is None else _ptr(rows_a), n_rows, _ptr(Y), N,
                        int(nthreads))
-    if any(k == "row_logsumexp" for k, _ in chain):
+    if any(k in ("row_logsumexp", "row_sum") for k, _ in chain):
         return Y[:, :1].copy()
     return Y
 

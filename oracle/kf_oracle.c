@@ -16,7 +16,8 @@
  *     ("layer-wise fusion", Sec. IV-B: the post-GEMM sequence of operations);
  *   - row log-sum-exp and GroupNorm are the plain two-pass definitions (the
  *     paper's single-pass/online forms, Sec. IV-B, reach the same value up to
- *     rounding order);
+ *     rounding order); the row sum (one reading of the "Sum" that ends the
+ *     chains of Table 3, Sec. IV-B) is the plain sum over the row's columns;
  *   - the MoE expert FFN (gpt-oss decode path, Sec. IV-A) is written per token as
  *     Y_t = sum_j w_tj * W_down[e_tj] (silu(W_gate[e_tj] x_t) * (W_up[e_tj] x_t)),
  *     with the intermediate h rounded to bf16 (the down GEMM consumes bf16 h);
@@ -67,6 +68,7 @@ enum {
   ORC_LEAKY_RELU = 12,   /* s > 0 ? s : scalar * s                        */
   ORC_MUL = 13,          /* s_j *= p0[j]                                  */
   ORC_ROW_SCALE = 14,    /* s_ij *= p0[i]                                 */
+  ORC_ROW_SUM = 15,      /* row -> sum_j s_j                              */
 };
 
 typedef struct {
@@ -80,6 +82,9 @@ typedef struct {
   int32_t pad_;
   int64_t ld;      /* leading dimension of a matrix operand (residual)   */
 } orc_op;
+
+/* Bytes of one stored element: fp32 is 4, the two 16-bit formats 2. */
+static size_t orc_elt_size(int dt) { return dt == ORC_F32 ? 4 : 2; }
 
 /* Widen one stored element to double.  bf16 is the top half of an IEEE
  * binary32 with the low 16 mantissa bits zero, so the widening is exact. */
@@ -186,9 +191,16 @@ static double orc_row_lse(const double *s, int64_t n) {
   return m + log(acc);
 }
 
+/* Row sum: the plain left-to-right sum of the row's n values. */
+static double orc_row_sum(const double *s, int64_t n) {
+  double acc = 0.0;
+  for (int64_t j = 0; j < n; ++j) acc += s[j];
+  return acc;
+}
+
 /* Apply the chain ops[first..n_ops) to the row vector s (length n) of row i.
  * Returns the number of live columns after the chain (1 after a row
- * log-sum-exp, n/2 after SwiGLU).  A scatter op is not applied here. */
+ * log-sum-exp or a row sum, n/2 after SwiGLU).  A scatter op is not applied here. */
 static int64_t orc_apply_chain(const orc_op *ops, int n_ops, double *s, int64_t n, int64_t i) {
   for (int o = 0; o < n_ops; ++o) {
     const orc_op *op = &ops[o];
@@ -198,6 +210,9 @@ static int64_t orc_apply_chain(const orc_op *ops, int n_ops, double *s, int64_t 
       s[0] = orc_row_lse(s, n);
       n = 1;
       /* ops after the reduction act on the scalar (column index 0) */
+    } else if (op->kind == ORC_ROW_SUM) {
+      s[0] = orc_row_sum(s, n);
+      n = 1;
     } else if (op->kind == ORC_GROUPNORM) {
       orc_groupnorm_row(op, s, n);
     } else if (op->kind == ORC_SWIGLU) {
@@ -219,7 +234,7 @@ static int64_t orc_apply_chain(const orc_op *ops, int n_ops, double *s, int64_t 
 /* ------------------------------------------------------------------------- */
 /* Dense fused GEMM: Y = chain(X W^T).  X [M x K] (ld ldx), W [N x K] (ld ldw). */
 /* Output: double Y[M x ldy]; after a row log-sum-exp Y has one value per row   */
-/* (stored at Y[i*ldy]).                                                       */
+/* or a row sum (stored at Y[i*ldy]).                                          */
 /* ------------------------------------------------------------------------- */
 typedef struct {
   const void *X; int xt; int64_t ldx;
@@ -507,7 +522,7 @@ int orc_grouped_gemm(const void *A, int at, int64_t lda, const int32_t *row_inde
   double *a = (double *)malloc(sizeof(double) * (size_t)(K > 0 ? K : 1));
   double *s = (double *)malloc(sizeof(double) * (size_t)(nb > 0 ? nb : 1));
   for (int32_t g = 0; g < G; ++g) {
-    const char *Bg = (const char *)B + (size_t)g * (size_t)b_group_stride * (bt == ORC_BF16 ? 2 : 4);
+    const char *Bg = (const char *)B + (size_t)g * (size_t)b_group_stride * orc_elt_size(bt);
     for (int64_t r = offsets[g]; r < offsets[g + 1]; ++r) {
       int64_t src = row_index ? row_index[r] : r;
       for (int64_t k = 0; k < K; ++k) a[k] = orc_load(A, at, src * lda + k);

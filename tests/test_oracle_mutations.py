@@ -45,6 +45,12 @@ MUTATIONS = {
                                      "y[c] += wt * acc;\n        if (jb->bd) y[c] += orc_load(jb->bd, ORC_BF16, e * H + c);"),
     "moe_up_bias_from_gate": ("u += orc_load(jb->bgu, ORC_BF16, e * 2 * I + I + n);",
                               "u += orc_load(jb->bgu, ORC_BF16, e * 2 * I + n);"),
+    "grouped_f16_stride": ("static size_t orc_elt_size(int dt) { return dt == ORC_F32 ? 4 : 2; }",
+                           "static size_t orc_elt_size(int dt) { return dt == ORC_BF16 ? 2 : 4; }"),
+    "row_sum_drops_last": ("for (int64_t j = 0; j < n; ++j) acc += s[j];\n  return acc;",
+                           "for (int64_t j = 0; j + 1 < n; ++j) acc += s[j];\n  return acc;"),
+    "row_sum_is_mean": ("for (int64_t j = 0; j < n; ++j) acc += s[j];\n  return acc;",
+                        "for (int64_t j = 0; j < n; ++j) acc += s[j];\n  return acc / (double)n;"),
     "residual_dropped": ("case ORC_RESIDUAL_ADD: return v + orc_load", "case ORC_RESIDUAL_ADD: return v + 0 * orc_load"),
 }
 

@@ -340,6 +340,65 @@ def test_grouped_single_group_equals_dense():
     assert np.array_equal(dense, grp)
 
 
+def test_grouped_f16_groups_equal_dense_calls():
+    """fp16 experts: every group of a grouped GEMM reads its own weights, so G
+    groups equal G dense products (this fails if the group stride were taken in
+    the wrong element size)."""
+    g = torch.Generator().manual_seed(21)
+    K, N = 24, 6
+    A = torch.randint(-4, 5, (9, K), generator=g).float().to(torch.float16)
+    B = torch.randint(-4, 5, (2, N, K), generator=g).float().to(torch.float16)
+    off = np.array([0, 4, 9], np.int32)
+    grp = oracle.grouped_gemm(A, B, off, N, [])
+    for e in range(2):
+        dense = oracle.fused_gemm(A[off[e]:off[e + 1]], B[e], [])
+        assert np.array_equal(grp[off[e]:off[e + 1]], dense)
+        exact = A[off[e]:off[e + 1]].double().numpy() @ B[e].double().numpy().T
+        assert np.array_equal(dense, exact)
+    # the same integers in bf16 give the same products
+    grp_bf = oracle.grouped_gemm(A.float().to(torch.bfloat16), B.float().to(torch.bfloat16), off, N, [])
+    assert np.array_equal(grp, grp_bf)
+
+
+# ------------------------------------------------------------------ row sum
+def test_row_sum_closed_forms():
+    # constant row c over N columns sums to N c; rank-1 s_ij = u_i v_j (a.c)
+    # sums to u_i (a.c) sum_j v_j (small integers: exact in fp64)
+    Y, _ = _through_identity(torch.full((3, 64), 1.5), [("row_sum", {})])
+    assert Y.shape == (3, 1) and np.all(Y[:, 0] == 96.0)
+    g = torch.Generator().manual_seed(22)
+    M, N, K = 5, 37, 19
+    u = torch.randint(-3, 4, (M, 1), generator=g).float()
+    a = torch.randint(-3, 4, (1, K), generator=g).float()
+    v = torch.randint(-3, 4, (N, 1), generator=g).float()
+    c = torch.randint(-3, 4, (1, K), generator=g).float()
+    Y = oracle.fused_gemm(bf16(u @ a), bf16(v @ c), [("row_sum", {})])
+    ref = u.double()[:, 0] * float((a.double() * c.double()).sum()) * float(v.double().sum())
+    assert np.array_equal(Y[:, 0], ref.numpy())
+
+
+def test_row_sum_bruteforce_and_linearity():
+    g = torch.Generator().manual_seed(23)
+    M, N, K = 4, 6, 5
+    X = bf16(torch.randn(M, K, generator=g) * 3)
+    W = bf16(torch.randn(N, K, generator=g) * 3)
+    b = bf16(torch.randn(N, generator=g))
+    Y = oracle.fused_gemm(X, W, [("bias", {"p0": b}), ("row_sum", {}), ("scale", {"scalar": 0.5})])
+    xs = [[Fraction(float(t)) for t in row] for row in X.float().tolist()]
+    ws = [[Fraction(float(t)) for t in row] for row in W.float().tolist()]
+    bs = [Fraction(float(t)) for t in b.float().tolist()]
+    for i in range(M):
+        exact = sum(sum(xs[i][k] * ws[j][k] for k in range(K)) + bs[j] for j in range(N)) / 2
+        assert abs(Fraction(Y[i, 0]) - exact) <= abs(exact) * Fraction(1, 2**48) + Fraction(1, 2**200)
+    # linearity: the sum of 2W is twice the sum of W; X W^T summed over j equals
+    # X (sum_j W_j)^T, a matrix-vector product
+    Y1 = oracle.fused_gemm(X, W, [("row_sum", {})])
+    Y2 = oracle.fused_gemm(X, bf16(W.float() * 2), [("row_sum", {})])
+    assert np.allclose(Y2, 2 * Y1, rtol=1e-14, atol=1e-14)
+    mv = f64(X) @ f64(W).sum(axis=0)
+    assert np.allclose(Y1[:, 0], mv, rtol=1e-13, atol=1e-13)
+
+
 def test_row_scale_multiplies_each_row():
     g = torch.Generator().manual_seed(13)
     X = bf16(torch.randint(-3, 4, (5, 8), generator=g).float())
