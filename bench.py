@@ -399,48 +399,171 @@ def cpu_baseline(inp, wl, chain, target_s=8.0):
             "sample": f"{rows} of {wl.M} rows of {wl.name} (fp64 C, {dt:.2f} s)"}
 
 
+def dense_eager_fns(name, d):
+    """Unfused torch eager (separate launches per op) and the bare GEMM (cuBLAS),
+    fp32 with TF32 off."""
+    X, W = d["X"], d["W"]
+    if name == "fp32_relu_linear":
+        return (lambda: F.relu(F.linear(X, W, d["b"]))), (lambda: torch.matmul(X, W.t()))
+    return eager_dense(name, d), (lambda: torch.matmul(X, W.t()))
+
+
+def cpu_oracle_moe(m_cpu, logits_cpu, T, k, target_s):
+    """The oracle's MoE FFN as it stands on all host cores, on a bounded sample of
+    tokens; TFLOP/s counted over the sampled tokens' routed rows."""
+    import oracle
+    oracle.build()
+    cores = os.cpu_count() or 1
+    r = oracle.moe_route(logits_cpu, k)
+    H = m_cpu["W_down"].shape[1]
+    I = m_cpu["W_gu"].shape[1] // 2
+    n = min(T, cores)
+    while True:
+        t0 = time.perf_counter()
+        oracle.moe_ffn(m_cpu["X"], m_cpu["W_gu"], m_cpu["W_down"], r["topk_ids"], r["topk_w"],
+                       tokens=list(range(n)), nthreads=cores)
+        dt = time.perf_counter() - t0
+        if dt >= target_s / 4 or n >= T:
+            break
+        n = min(T, max(n * 2, int(n * target_s / max(dt, 1e-3) / 2)))
+    flops = 2.0 * n * k * (2 * I * H + H * I)
+    return {"value": round(flops / dt / 1e12, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} of {T} tokens (fp64 C, {dt:.2f} s)"}
+
+
+def roofline_block(flops, byts, ms, peaks, traffic=None):
+    """Roofline of one step: tensor-bound (FLOP / bf16 peak) or HBM-bound (bytes /
+    copy peak), whichever takes longer at the peaks."""
+    t_flop = flops / (peaks["bf16"] * 1e12)
+    t_mem = byts / (peaks["hbm"] * 1e9)
+    if t_flop >= t_mem:
+        ach = flops / (ms * 1e-3) / 1e12
+        return {"bound": "tensor", "achieved": round(ach, 2), "peak": peaks["bf16"],
+                "peak_src": f"{peaks['src']} bf16 burst", "unit": "TFLOP/s", "frac": round(ach / peaks["bf16"], 4),
+                "traffic": traffic, "algorithmic_bytes": byts}
+    ach = byts / (ms * 1e-3) / 1e9
+    return {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm"], "peak_src": f"{peaks['src']} copy",
+            "unit": "GB/s", "frac": round(ach / peaks["hbm"], 4), "traffic": traffic, "algorithmic_bytes": byts}
+
+
+DENSE_TRAFFIC_TAGS = {"bf16_scale_rowlse": "dense_lse_2048x8192x8192"}
+
+
+def dense_config_block(name, args, kf, dev, flush, stream, peaks, steps):
+    """One dense configuration with its full record: isolated device time, the
+    roofline of its kernel, unfused eager and bare-GEMM baselines, the end-to-end
+    time through the public API from pinned host buffers, and the oracle on the
+    host cores over a bounded row sample."""
+    import ctypes
+    wl, inp, d, chain = dense_setup(name, dev)
+    M, N, K = wl.M, wl.N, wl.K
+    flops = 2.0 * M * N * K
+    keep = []
+    need = kf.lib().kf_fused_gemm_workspace(M, N, K, ctypes.byref(kf.make_epilogue(chain, keep)))
+    ws = kf.new_workspace(need, dev) if need else None
+    red = any(kk in kf.ROW_REDUCTIONS for kk, _ in chain)
+    out_dt = torch.float32 if (red or wl.dtype == "f32") else torch.bfloat16
+    out = torch.empty((M,) if red else (M, N), dtype=out_dt, device=dev)
+    fn = lambda: kf.fused_gemm(d["X"], d["W"], chain, out=out, workspace=ws)
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    try:
+        ms = time_steps(fn, steps, args.warmup, flush, stream)
+        eager, gemm = dense_eager_fns(name, d)
+        ms_e = time_steps(eager, steps, args.warmup, flush, stream)
+        ms_c = time_steps(gemm, steps, args.warmup, flush, stream)
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+    hin = {k2: v.pin_memory() for k2, v in inp.items()}
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+
+    def e2e():
+        for k2 in hin:
+            d[k2].copy_(hin[k2], non_blocking=True)
+        kf.fused_gemm(d["X"], d["W"], chain, out=out, workspace=ws)
+        hout.copy_(out, non_blocking=True)
+
+    ms_e2e = time_steps(e2e, max(3, steps // 2), args.warmup, flush, stream, host_slack=False)
+    h2d = sum(v.numel() * v.element_size() for v in hin.values())
+    d2h = hout.numel() * hout.element_size()
+    byts = dense_bytes(name, wl)
+    rec = {"workload": name, "M": M, "N": N, "K": K, "ms": round(ms, 5),
+           "tflops": round(flops / ms / 1e9, 3),
+           "roofline": roofline_block(flops, byts, ms, peaks, stored_traffic(DENSE_TRAFFIC_TAGS.get(name, ""))),
+           "eager_ms": round(ms_e, 5), "speedup_vs_eager": round(ms_e / ms, 3),
+           "gemm_only_ms": round(ms_c, 5),
+           "e2e": {"value": round(flops / ms_e2e / 1e9, 3), "unit": "TFLOP/s", "ms_per_step": round(ms_e2e, 4),
+                   "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+           "l2": "256 MiB written between steps (cold L2 for every step)",
+           "launches_per_step": 2 if red else 1}
+    if name == "fp32_relu_linear":
+        rec["us"] = round(ms * 1e3, 2)
+        rec["eager_us"] = round(ms_e * 1e3, 2)
+        rec["note"] = "fp32 FFMA path (exact fp32); eager and the bare GEMM with TF32 off"
+    if not args.no_cpu:
+        rec["cpu_baseline"] = cpu_baseline(inp, wl, chain_cpu(name, inp), target_s=args.cpu_seconds / 2)
+    del d, inp, hin
+    return rec
+
+
+def moe_config_block(T, m, args, kf, dev, flush, stream, peaks, steps, m_cpu):
+    """The routed MoE FFN at T tokens (32 experts, top-4, H = I = 2880): device
+    time, roofline (HBM-bound weight streaming at decode, tensor-bound at
+    prefill), unfused eager, end to end (tokens and logits in, output out; the
+    weights stay resident as in serving) and the oracle on a token sample."""
+    E, k, H, I = 32, 4, 2880, 2880
+    g = torch.Generator("cpu").manual_seed(0)
+    Xc = torch.randn(T, H, generator=g).to(torch.bfloat16)
+    lc = torch.randn(T, E, generator=g)
+    X, logits = Xc.to(dev), lc.to(dev)
+    ws = kf.new_workspace(kf.moe_ffn_workspace_bytes(T, H, I, E, k), dev)
+    out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
+    fn = lambda: kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, out=out, workspace=ws)
+    ms = time_steps(fn, steps, args.warmup, flush, stream)
+    ms_e = time_steps(lambda: moe_eager(X, logits, m["W_gu"], m["W_down"], k), max(3, steps // 2),
+                      args.warmup, flush, stream)
+    hX, hl = Xc.pin_memory(), lc.pin_memory()
+    hout = torch.empty(T, H, dtype=torch.bfloat16).pin_memory()
+
+    def e2e():
+        X.copy_(hX, non_blocking=True)
+        logits.copy_(hl, non_blocking=True)
+        kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, out=out, workspace=ws)
+        hout.copy_(out, non_blocking=True)
+
+    ms_e2e = time_steps(e2e, max(3, steps // 2), args.warmup, flush, stream, host_slack=False)
+    ids = torch.topk(logits, k, dim=1).indices
+    touched = int(torch.unique(ids).numel())
+    wbytes = touched * (2 * I * H + H * I) * 2
+    byts = wbytes + 2 * T * H * 2 + 4 * T * E
+    flops = 2.0 * T * k * (2 * I * H + H * I)
+    rec = {"workload": f"moe_ffn_T{T}", "T": T, "H": H, "I": I, "E": E, "k": k, "ms": round(ms, 5),
+           "tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
+           "roofline": roofline_block(flops, byts, ms, peaks, stored_traffic(f"moe_T{T}")),
+           "experts_touched": touched, "eager_ms": round(ms_e, 5), "speedup_vs_eager": round(ms_e / ms, 3),
+           "e2e": {"value": round(flops / ms_e2e / 1e9, 3), "unit": "TFLOP/s", "ms_per_step": round(ms_e2e, 4),
+                   "h2d_bytes_per_step": hX.numel() * 2 + hl.numel() * 4, "d2h_bytes_per_step": hout.numel() * 2},
+           "l2": "256 MiB written between steps; the 1.59 GB of expert weights exceed L2 anyway",
+           "launches_per_step": 6}
+    if not args.no_cpu:
+        mc = dict(X=Xc, W_gu=m_cpu["W_gu"], W_down=m_cpu["W_down"])
+        rec["cpu_baseline"] = cpu_oracle_moe(mc, lc, T, k, args.cpu_seconds / 2)
+    return rec
+
+
 def other_workloads(args, kf, dev, flush, stream, peaks):
     res = {}
     steps = max(3, min(args.steps, 20))
-    for name in ("bf16_scale_rowlse", "bf16_groupnorm_swish"):
-        wl, inp, d, chain = dense_setup(name, dev)
-        flops = 2.0 * wl.M * wl.N * wl.K
-        ms = time_steps(lambda: kf.fused_gemm(d["X"], d["W"], chain), steps, args.warmup, flush, stream)
-        ms_e = time_steps(eager_dense(name, d), steps, args.warmup, flush, stream)
-        ms_c = time_steps(lambda: torch.matmul(d["X"], d["W"].t()), steps, args.warmup, flush, stream)
-        t_roof = max(flops / (peaks["bf16"] * 1e12), dense_bytes(name, wl) / (peaks["hbm"] * 1e9)) * 1e3
-        res[name] = {"tflops": round(flops / ms / 1e9, 2), "ms": round(ms, 5), "bound": "tensor",
-                     "roofline_frac": round(t_roof / ms, 4), "eager_ms": round(ms_e, 5),
-                     "speedup_vs_eager": round(ms_e / ms, 3), "cublas_gemm_only_ms": round(ms_c, 5),
-                     "launches_per_step": 2 if name == "bf16_scale_rowlse" else 1}
-        del d, inp
+    for name in ("fp32_relu_linear", "bf16_scale_rowlse", "bf16_groupnorm_swish"):
+        res[name] = dense_config_block(name, args, kf, dev, flush, stream, peaks, steps)
     E, k, H, I = 32, 4, 2880, 2880
-    m = None
+    gd = torch.Generator(dev).manual_seed(1)
+    m = dict(W_gu=(torch.randn(E, 2 * I, H, generator=gd, device=dev) * 0.02).to(torch.bfloat16),
+             W_down=(torch.randn(E, H, I, generator=gd, device=dev) * 0.02).to(torch.bfloat16))
+    m_cpu = None if args.no_cpu else {kk: v.cpu() for kk, v in m.items()}
     for T in (64, 4096):
-        g = torch.Generator("cpu").manual_seed(0)
-        X = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
-        logits = torch.randn(T, E, generator=g).to(dev)
-        if m is None:
-            gd = torch.Generator(dev).manual_seed(1)
-            m = dict(W_gu=(torch.randn(E, 2 * I, H, generator=gd, device=dev) * 0.02).to(torch.bfloat16),
-                     W_down=(torch.randn(E, H, I, generator=gd, device=dev) * 0.02).to(torch.bfloat16))
-        ws = torch.empty(kf.moe_ffn_workspace_bytes(T, H, I, E, k), dtype=torch.uint8, device=dev)
-        out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
-        fn = lambda: kf.moe_ffn(X, logits, m["W_gu"], m["W_down"], k, out=out, workspace=ws)
-        ms = time_steps(fn, steps, args.warmup, flush, stream)
-        ms_e = time_steps(lambda: moe_eager(X, logits, m["W_gu"], m["W_down"], k), max(3, steps // 2),
-                          args.warmup, flush, stream)
-        ids = torch.topk(logits, k, dim=1).indices
-        touched = int(torch.unique(ids).numel())
-        wbytes = touched * (2 * I * H + H * I) * 2
-        byts = wbytes + 2 * T * H * 2 + 4 * T * E
-        flops = 2.0 * T * k * (2 * I * H + H * I)
-        t_roof = max(flops / (peaks["bf16"] * 1e12), byts / (peaks["hbm"] * 1e9)) * 1e3
-        bound = "hbm" if byts / (peaks["hbm"] * 1e9) > flops / (peaks["bf16"] * 1e12) else "tensor"
-        res[f"moe_T{T}"] = {"tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
-                            "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
-                            "experts_touched": touched, "eager_ms": round(ms_e, 5),
-                            "speedup_vs_eager": round(ms_e / ms, 3), "launches_per_step": 6}
+        res[f"moe_T{T}"] = moe_config_block(T, m, args, kf, dev, flush, stream, peaks, steps, m_cpu)
+    del m_cpu
     # MoE block tail at decode: residual add + RMSNorm fused into the MoE finalize,
     # against the same MoE FFN followed by torch's add and rms_norm
     T = 64
@@ -449,7 +572,7 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
     logits = torch.randn(T, E, generator=g).to(dev)
     R = torch.randn(T, H, generator=g).to(torch.bfloat16).to(dev)
     gamma = (torch.rand(H, generator=g) + 0.5).to(torch.bfloat16).to(dev)
-    ws = torch.empty(kf.moe_ffn_workspace_bytes(T, H, I, E, k), dtype=torch.uint8, device=dev)
+    ws = kf.new_workspace(kf.moe_ffn_workspace_bytes(T, H, I, E, k), dev)
     y_out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
     r_out = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
     fused = lambda: kf.moe_ffn_add_rmsnorm(X, logits, m["W_gu"], m["W_down"], k, R, gamma, 1e-5, out=y_out,

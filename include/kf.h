@@ -26,10 +26,22 @@
  *     argument returns a status and launches nothing.  A failed launch returns
  *     KF_ERR_CUDA.  No call aborts, exits or throws.
  *   - Device-side waits are bounded.  A kernel whose wait runs out (or that finds
- *     bad device-resident routing data) records an error code in a per-device
- *     error word and returns early; kf_get_device_error reads and clears it.
+ *     bad device-resident indices) records error bits and returns early.  The
+ *     bits go to the error word of the call's workspace when it was given one
+ *     (the first 32-bit word of the workspace's KF_WORKSPACE_HEADER_BYTES
+ *     header; kf_check_device_error reads and clears it), and always to a
+ *     per-device error word (kf_get_device_error reads and clears that one; it
+ *     collects the errors of every call on the device, so a check there by one
+ *     thread can consume another thread's error).
+ *   - Workspaces: a call that takes a workspace and is given one (16-byte
+ *     aligned, at least KF_WORKSPACE_HEADER_BYTES) uses its first
+ *     KF_WORKSPACE_HEADER_BYTES bytes as the header and the rest as scratch.
+ *     The *_workspace size queries include the header.  The header must be zero
+ *     before the workspace's first use (kf_workspace_init, or a zero-filled
+ *     allocation); calls only OR bits into it, kf_check_device_error clears it.
  *   - Calls on distinct streams may run concurrently if they use distinct
- *     workspaces and outputs.
+ *     workspaces and outputs; each then checks its own errors with
+ *     kf_check_device_error on its own workspace.
  */
 #ifndef KF_H_
 #define KF_H_
@@ -53,6 +65,9 @@ typedef enum kf_status {
 } kf_status;
 
 typedef enum kf_dtype { KF_F32 = 0, KF_BF16 = 1, KF_I32 = 2, KF_F16 = 3 } kf_dtype;
+
+/* Bytes at the start of every workspace reserved for its header (error word). */
+#define KF_WORKSPACE_HEADER_BYTES 256
 
 /* Tail ops, applied in list order to the fp32 accumulator (Sec. IV-B: the
  * post-GEMM sequence of operations, fused into one kernel). */
@@ -83,7 +98,13 @@ typedef enum kf_op_kind {
   KF_OP_MISH = 11,         /* v * tanh(log(1 + exp(v)))                                */
   KF_OP_LEAKY_RELU = 12,   /* v > 0 ? v : scalar * v                                   */
   KF_OP_MUL = 13,          /* v *= p0[col]                          (p0: [N])        */
-  KF_OP_ROW_SCALE = 14     /* v *= p0[row]                 (p0: fp32, one per row)     */
+  KF_OP_ROW_SCALE = 14,    /* v *= p0[row]                 (p0: fp32, one per row)     */
+  KF_OP_ROW_SUM = 15       /* row -> sum_j v_j; Y is [M] (fp32, bf16 or fp16).  Ends a
+                              chain of pointwise ops, or follows GROUPNORM (pointwise
+                              ops may sit between); only scalar ops (as after
+                              ROW_LOGSUMEXP) may follow it.  Needs a workspace.  The
+                              "Sum" that ends the paper's Table 3 chains (Sec. IV-B),
+                              read as a reduction over each row.                      */
 } kf_op_kind;
 
 typedef struct kf_epilogue_op {
@@ -107,7 +128,8 @@ typedef struct kf_epilogue {
  * kf_fused_gemm -- Y = chain(X W^T)                    (Sec. IV-B, Table 3)
  *
  *   X [M x K] (row stride ldx), W [N x K] (row stride ldw), Y [M x N] (row
- *   stride ldy), or Y [M] (fp32 or bf16) when the chain holds ROW_LOGSUMEXP.
+ *   stride ldy), or Y [M] (fp32, bf16 or fp16) when the chain holds
+ *   ROW_LOGSUMEXP or ROW_SUM.
  *   Operand dtypes: both KF_BF16 or both KF_F16 (tcgen05 tensor-core path, fp32
  *   accumulation in tensor memory; Y bf16, fp16 or fp32; the paper's B580
  *   kernels ran their matmuls in fp16, Sec. IV-B), or both KF_F32 (element-wise
@@ -120,12 +142,13 @@ typedef struct kf_epilogue {
  *   bf16 path: X, W must be 16-byte aligned with ldx, ldw multiples of 8, else
  *   KF_ERR_MISALIGNED.  M == 0 or N == 0 is a no-op; K must be >= 1.
  *   workspace: kf_fused_gemm_workspace() bytes.  Required for a row
- *   log-sum-exp (per-tile row partials live there).  Optional for GroupNorm over
- *   512-column groups with M > 128: with it, pairs of CTA pairs exchange per-row
- *   statistics through it (all SMs work; the launch is cooperative); with a
- *   smaller or no workspace, clusters of four CTAs exchange them on chip (fewer
- *   SMs can be used).  Same results either way.  0 otherwise.  Calls that share
- *   one workspace must not overlap on the GPU.
+ *   log-sum-exp or row sum (per-tile row partials live there).  Optional for
+ *   GroupNorm over 512-column groups with M > 128 and no row sum: with it, pairs
+ *   of CTA pairs exchange per-row statistics through it (all SMs work; the
+ *   launch is cooperative); with a smaller or no workspace, clusters of four CTAs
+ *   exchange them on chip (fewer SMs can be used).  Same results either way.  0
+ *   otherwise (a KF_WORKSPACE_HEADER_BYTES workspace may still be passed, for
+ *   its error word).  Calls that share one workspace must not overlap on the GPU.
  *   Y must not alias X or W; a RESIDUAL_ADD operand may alias Y (in place).
  */
 kf_status kf_fused_gemm(const void* X, int32_t x_dtype, int64_t ldx, const void* W, int32_t w_dtype,
@@ -173,8 +196,9 @@ kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int
  *   C is [rows_total x N] (stride ldc), bf16 or fp32; with
  *   ROW_SCALE_SCATTER_ADD C is the fp32 scatter target instead.
  *   A, B bf16; alignment rules as kf_fused_gemm (also b_group_stride % 8 == 0).
- *   workspace: kf_grouped_gemm_workspace() bytes (the gathered rows live there).
- *   Bad device-side offsets/indices set KF_ERR_DEVICE_BOUNDS in the error word.
+ *   workspace: kf_grouped_gemm_workspace() bytes (the gathered rows live there;
+ *   0 without a gather).  Bad device-side offsets/indices set
+ *   KF_ERR_DEVICE_BOUNDS in the error words.
  */
 kf_status kf_grouped_gemm(const void* A, int32_t a_dtype, int64_t lda, int64_t a_rows, const int32_t* a_row_index,
                           const void* B, int32_t b_dtype, int64_t ldb, int64_t b_group_stride,
@@ -323,17 +347,35 @@ kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dtype, int64_t
  *   capture.  Every call shares the one array: calls whose executions overlap
  *   on the GPU (different streams, or different host threads) race on it and
  *   must be serialized by the caller.  Each call overwrites every partial it
- *   reads, so no clearing is needed between calls.
+ *   reads, so no clearing is needed between calls.  Operands bf16 or fp16, as
+ *   for kf_fused_gemm.  Device-side errors go to the per-device error word
+ *   (kf_get_device_error).
  */
 kf_status kf_fused_gemm_lse_noalloc(const void* X, int32_t x_dtype, int64_t ldx, const void* W, int32_t w_dtype,
                                     int64_t ldw, void* Y, int32_t y_dtype, int64_t M, int64_t N, int64_t K,
                                     const kf_epilogue* epi, void* stream);
 size_t kf_fused_gemm_lse_noalloc_max_bytes(void);
 
-/* Synchronize `stream`, read and clear this device's error word.  Returns KF_OK,
- * KF_ERR_DEVICE_TIMEOUT or KF_ERR_DEVICE_BOUNDS; *raw (if non-NULL) receives the
- * raw bit set (1 = producer wait, 2 = MMA wait, 4 = epilogue wait, 8 = bounds). */
+/* Synchronize `stream`, read and clear this device's error word (the errors of
+ * every call on the device).  Returns KF_OK, KF_ERR_DEVICE_TIMEOUT or
+ * KF_ERR_DEVICE_BOUNDS (KF_ERR_CUDA for a launch-shape error); *raw (if non-NULL)
+ * receives the raw bit set (1 = producer wait, 2 = MMA wait, 4 = epilogue wait,
+ * 8 = bounds, 16 = launch shape). */
 kf_status kf_get_device_error(void* stream, uint32_t* raw);
+
+/* The same for the error word in `workspace`'s header: only the calls that were
+ * given this workspace write it, so threads that use distinct workspaces see
+ * only their own errors.  `workspace` is the pointer the calls were given
+ * (device memory, 16-byte aligned; KF_ERR_INVALID_ARG otherwise).  Synchronizes
+ * `stream`, which must be the stream of those calls (or one ordered after them).
+ * Returns and reports as kf_get_device_error. */
+kf_status kf_check_device_error(void* workspace, void* stream, uint32_t* raw);
+
+/* Zero `workspace`'s header (cudaMemsetAsync of KF_WORKSPACE_HEADER_BYTES bytes
+ * on `stream`): needed once before a workspace's first use unless it was
+ * allocated zero-filled.  `bytes` >= KF_WORKSPACE_HEADER_BYTES and a 16-byte
+ * aligned pointer, else KF_ERR_INVALID_ARG.  Allocates nothing. */
+kf_status kf_workspace_init(void* workspace, size_t bytes, void* stream);
 
 /* Wall-time limit of every device-side wait, in ns, for later launches
  * (0 restores the default of 2 s).  A short limit makes a kernel give up early

@@ -8,7 +8,13 @@ is no fallback: if ``libkf.so`` is missing the import of the library raises.
 Tail chains are lists of ``(kind, params)``; kinds are the lower-case names of
 ``kf_op_kind`` (``bias, scale, relu, gelu_tanh, silu, sigmoid, residual_add,
 row_logsumexp, groupnorm, swiglu, row_scale_scatter_add, mish, leaky_relu,
-mul``); params ``p0, p1`` (device tensors), ``scalar, eps, groups, ld``.
+mul, row_scale, row_sum``); params ``p0, p1`` (device tensors), ``scalar, eps,
+groups, ld``.
+
+Workspaces start with a ``KF_WORKSPACE_HEADER_BYTES`` header holding the error
+word of the calls given that workspace (``check_device_error``); the header must
+be zero before first use: ``new_workspace`` allocates one that way, and the
+workspaces the functions here allocate themselves are zeroed the same way.
 """
 from __future__ import annotations
 
@@ -28,7 +34,10 @@ OPS = {
     "bias": 0, "scale": 1, "relu": 2, "gelu_tanh": 3, "silu": 4, "sigmoid": 5,
     "residual_add": 6, "row_logsumexp": 7, "groupnorm": 8, "swiglu": 9,
     "row_scale_scatter_add": 10, "mish": 11, "leaky_relu": 12, "mul": 13, "row_scale": 14,
+    "row_sum": 15,
 }
+ROW_REDUCTIONS = ("row_logsumexp", "row_sum")
+KF_WORKSPACE_HEADER_BYTES = 256
 KF_MOE_DETERMINISTIC = 1
 # every entry point declared in include/kf.h
 ABI_SYMBOLS = (
@@ -36,7 +45,7 @@ ABI_SYMBOLS = (
     "kf_grouped_gemm_workspace", "kf_moe_ffn", "kf_moe_ffn_workspace", "kf_get_device_error",
     "kf_set_wait_timeout_ns", "kf_status_string", "kf_abi_version", "kf_fused_gemm_lse_noalloc",
     "kf_fused_gemm_lse_noalloc_max_bytes", "kf_moe_ffn_ex", "kf_moe_ffn_workspace_ex", "kf_moe_ffn_add_rmsnorm",
-    "kf_qkv_rope_kv", "kf_moe_ffn_act", "kf_fused_gemm_ex",
+    "kf_qkv_rope_kv", "kf_moe_ffn_act", "kf_fused_gemm_ex", "kf_check_device_error", "kf_workspace_init",
 )
 KF_GEMM_F32_FFMA, KF_GEMM_F32_TF32X3 = 1, 2
 
@@ -102,6 +111,10 @@ def lib() -> ctypes.CDLL:
     L.kf_moe_ffn_workspace_ex.argtypes = [I64, I64, I64, I32, I32, ctypes.c_uint32]
     L.kf_moe_ffn_workspace_ex.restype = SZ
     L.kf_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
+    L.kf_check_device_error.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
+    L.kf_check_device_error.restype = I32
+    L.kf_workspace_init.argtypes = [P, SZ, P]
+    L.kf_workspace_init.restype = I32
     L.kf_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
     L.kf_fused_gemm_lse_noalloc.argtypes = [P, I32, I64, P, I32, I64, P, I32, I64, I64, I64, EP, P]
     L.kf_fused_gemm_lse_noalloc.restype = I32
@@ -182,11 +195,19 @@ def make_epilogue(chain: Sequence[Tuple[str, Dict]], keep: list, default_ld: int
     return Epilogue(len(chain), ctypes.cast(arr, ctypes.POINTER(EpilogueOp)))
 
 
+def new_workspace(nbytes: int, device, stream=None) -> torch.Tensor:
+    """A workspace of ``nbytes`` (at least the header) with its header zeroed
+    (kf_workspace_init on ``stream``)."""
+    ws = torch.empty(max(int(nbytes), KF_WORKSPACE_HEADER_BYTES), dtype=torch.uint8, device=device)
+    _check(lib().kf_workspace_init(ws.data_ptr(), ws.numel(), _stream(stream)), "kf_workspace_init")
+    return ws
+
+
 def _workspace(nbytes: int, device, workspace: Optional[torch.Tensor]) -> Tuple[Optional[torch.Tensor], int]:
-    if nbytes == 0:
-        return None, 0
     if workspace is None:
-        workspace = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        if nbytes == 0:
+            return None, 0
+        workspace = new_workspace(nbytes, device)
     if workspace.numel() * workspace.element_size() < nbytes:
         raise ValueError("workspace too small")
     return workspace, workspace.numel() * workspace.element_size()
@@ -200,7 +221,7 @@ def fused_gemm(X: torch.Tensor, W: torch.Tensor, chain: Sequence[Tuple[str, Dict
     ``f32_mode`` "ffma" or "tf32x3" forces a path (default: by problem size)."""
     M, K = X.shape
     N = W.shape[0]
-    lse = any(k == "row_logsumexp" for k, _ in chain)
+    lse = any(k in ROW_REDUCTIONS for k, _ in chain)
     if out is None:
         dt = out_dtype or (torch.float32 if (lse or X.dtype == torch.float32) else X.dtype)
         out = torch.empty((M,) if lse else (M, N), dtype=dt, device=X.device)
@@ -371,9 +392,18 @@ def qkv_rope_kv(X: torch.Tensor, W: torch.Tensor, bias: Optional[torch.Tensor], 
 
 
 def get_device_error(stream=None) -> Tuple[int, int]:
-    """(status, raw bits) of this device's error word; synchronizes the stream."""
+    """(status, raw bits) of this device's error word (every call on the
+    device); synchronizes the stream and clears the word."""
     raw = ctypes.c_uint32(0)
     st = lib().kf_get_device_error(_stream(stream), ctypes.byref(raw))
+    return st, raw.value
+
+
+def check_device_error(workspace: torch.Tensor, stream=None) -> Tuple[int, int]:
+    """(status, raw bits) of the error word in ``workspace``'s header (only the
+    calls given that workspace); synchronizes the stream and clears the word."""
+    raw = ctypes.c_uint32(0)
+    st = lib().kf_check_device_error(workspace.data_ptr(), _stream(stream), ctypes.byref(raw))
     return st, raw.value
 
 

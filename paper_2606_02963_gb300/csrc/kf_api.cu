@@ -147,6 +147,12 @@ struct ChainPlan {
   int n_pre = 0, n_post = 0;
   DevOp pre[kMaxOps];
   DevOp post[kMaxOps];
+  // a row reduction's result ([M]): row sum instead of log-sum-exp (kModeLse),
+  // or a row sum after the GroupNorm's post chain (kModeGroupNorm); the scalar
+  // ops after the reduction run in the combine kernel (fin)
+  bool red_sum = false;
+  int n_fin = 0;
+  DevOp fin[kMaxOps];
   DevOp norm;
   int gs = 0;
   const float* row_scale = nullptr;
@@ -184,11 +190,20 @@ kf_status to_devop(const kf_epilogue_op& o, int64_t N, DevOp* d) {
 kf_status plan_chain(const kf_epilogue* epi, int64_t N, bool grouped, ChainPlan* pl) {
   const int n = epi ? epi->num_ops : 0;
   if (n < 0 || n > kMaxOps || (n > 0 && !epi->ops)) return KF_ERR_INVALID_ARG;
-  int special = -1;
+  // one reduction / special op per chain, except that a row sum may end a
+  // GroupNorm chain (GroupNorm, pointwise ops, row sum, scalar ops)
+  int special = -1, gn_sum = -1;
   for (int i = 0; i < n; ++i) {
     const int k = epi->ops[i].kind;
-    if (k == KF_OP_ROW_LOGSUMEXP || k == KF_OP_GROUPNORM || k == KF_OP_SWIGLU || k == KF_OP_ROW_SCALE_SCATTER_ADD) {
-      if (special >= 0) return KF_ERR_UNSUPPORTED;  // one reduction / special op per chain
+    if (k == KF_OP_ROW_LOGSUMEXP || k == KF_OP_GROUPNORM || k == KF_OP_SWIGLU || k == KF_OP_ROW_SCALE_SCATTER_ADD ||
+        k == KF_OP_ROW_SUM) {
+      if (special >= 0) {
+        if (epi->ops[special].kind == KF_OP_GROUPNORM && k == KF_OP_ROW_SUM && gn_sum < 0) {
+          gn_sum = i;
+          continue;
+        }
+        return KF_ERR_UNSUPPORTED;
+      }
       special = i;
     } else if (!is_pointwise_op(k)) {
       return KF_ERR_INVALID_ARG;
@@ -196,23 +211,40 @@ kf_status plan_chain(const kf_epilogue* epi, int64_t N, bool grouped, ChainPlan*
   }
   const int sk = special >= 0 ? epi->ops[special].kind : -1;
   if (!grouped && (sk == KF_OP_SWIGLU || sk == KF_OP_ROW_SCALE_SCATTER_ADD)) return KF_ERR_INVALID_ARG;
-  if (grouped && (sk == KF_OP_ROW_LOGSUMEXP || sk == KF_OP_GROUPNORM)) return KF_ERR_UNSUPPORTED;
+  if (grouped && (sk == KF_OP_ROW_LOGSUMEXP || sk == KF_OP_GROUPNORM || sk == KF_OP_ROW_SUM)) return KF_ERR_UNSUPPORTED;
+  const bool row_red = sk == KF_OP_ROW_LOGSUMEXP || sk == KF_OP_ROW_SUM;
   const int split = special >= 0 ? special : n;
+  const int post_end = gn_sum >= 0 ? gn_sum : n;  // ops the kernel applies after the special op
   pl->n_pre = split;
-  pl->n_post = special >= 0 ? n - special - 1 : 0;
+  pl->n_post = special >= 0 ? post_end - special - 1 : 0;
   for (int i = 0; i < split; ++i) {
     kf_status st = to_devop(epi->ops[i], N, &pl->pre[i]);
     if (st != KF_OK) return st;
   }
   for (int i = 0; i < pl->n_post; ++i) {
     const kf_epilogue_op& o = epi->ops[special + 1 + i];
-    if (sk == KF_OP_ROW_LOGSUMEXP && !is_scalar_op(o.kind)) return KF_ERR_INVALID_ARG;
+    if (row_red && !is_scalar_op(o.kind)) return KF_ERR_INVALID_ARG;
     kf_status st = to_devop(o, N, &pl->post[i]);
     if (st != KF_OK) return st;
   }
+  // scalar ops after a row reduction run on the combined value
+  pl->red_sum = sk == KF_OP_ROW_SUM || gn_sum >= 0;
+  if (row_red) {
+    pl->n_fin = pl->n_post;
+    for (int i = 0; i < pl->n_post; ++i) pl->fin[i] = pl->post[i];
+  } else if (gn_sum >= 0) {
+    pl->n_fin = n - gn_sum - 1;
+    for (int i = 0; i < pl->n_fin; ++i) {
+      const kf_epilogue_op& o = epi->ops[gn_sum + 1 + i];
+      if (!is_scalar_op(o.kind)) return KF_ERR_INVALID_ARG;
+      kf_status st = to_devop(o, N, &pl->fin[i]);
+      if (st != KF_OK) return st;
+    }
+  }
   switch (sk) {
     case -1: pl->mode = kModeStore; break;
-    case KF_OP_ROW_LOGSUMEXP: pl->mode = kModeLse; break;
+    case KF_OP_ROW_LOGSUMEXP:
+    case KF_OP_ROW_SUM: pl->mode = kModeLse; break;
     case KF_OP_SWIGLU:
       pl->mode = kModeSwiglu;
       if (pl->n_pre != 0) return KF_ERR_UNSUPPORTED;  // SwiGLU acts on the raw gate/up accumulators
@@ -249,7 +281,7 @@ kf_status plan_chain(const kf_epilogue* epi, int64_t N, bool grouped, ChainPlan*
   return KF_OK;
 }
 
-void fill_params_common(TcParams& p, const ChainPlan& pl, uint32_t* err) {
+void fill_params_common(TcParams& p, const ChainPlan& pl, uint32_t* err, uint32_t* err_dev) {
   // a single bf16 residual operand in the pre-chain is staged through shared
   // memory with coalesced loads (a second one would need its own buffer)
   int nres = 0, ires = -1;
@@ -270,7 +302,9 @@ void fill_params_common(TcParams& p, const ChainPlan& pl, uint32_t* err) {
   for (int i = 0; i < pl.n_pre; ++i) p.pre[i] = pl.pre[i];
   for (int i = 0; i < pl.n_post; ++i) p.post[i] = pl.post[i];
   p.norm = pl.norm;
+  p.red_sum = pl.red_sum ? 1 : 0;
   p.err = err;
+  p.err_dev = err_dev;
   p.wait_ns = g_wait_ns.load();
   p.drain_ns = std::max<uint64_t>(p.wait_ns, 1000000000ull);
 }
@@ -343,6 +377,25 @@ uint32_t mode_box(int mode, int bn) { return mode == kModeSwiglu ? bn / 2 : bn; 
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// A workspace starts with a header whose first 32-bit word is the error word of
+// the calls given that workspace; the call's scratch (payload) follows it.
+constexpr size_t kWsHeader = KF_WORKSPACE_HEADER_BYTES;
+struct WsView {
+  uint32_t* err = nullptr;  // the header's error word (null: no usable workspace)
+  void* payload = nullptr;
+  size_t bytes = 0;         // payload bytes
+};
+WsView split_ws(void* ws, size_t bytes) {
+  WsView v;
+  if (ws && aligned16(ws) && bytes >= kWsHeader) {
+    v.err = static_cast<uint32_t*>(ws);
+    v.payload = static_cast<char*>(ws) + kWsHeader;
+    v.bytes = bytes - kWsHeader;
+  }
+  return v;
+}
+size_t with_header(size_t payload) { return payload ? kWsHeader + payload : 0; }
+
 // GroupNorm couples: statistics exchange area for up to kMaxCouples couples
 // ([couples][2 slots][2 halves][256 rows] float2, then [couples][2][2][8] flags)
 constexpr int kMaxCouples = 128;
@@ -409,13 +462,14 @@ struct GroupExtras {
 
 // `pdl`: the previous kernel in the stream is one of this library's (MoE chain),
 // so the launches here may be programmatic dependents of it.
-kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cudaStream_t s, const DevInfo& di,
-                       bool pdl, const GroupExtras* ex = nullptr) {
+// `ws`: the payload the gathered rows go to; `werr`: the call's error word.
+kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, uint32_t* werr, cudaStream_t s,
+                       const DevInfo& di, bool pdl, const GroupExtras* ex = nullptr) {
   const void* A = g.A;
   int64_t lda = g.lda;
   if (g.a_row_index) {
-    kf_status st =
-        cuda_status(gather_rows_launch(g.A, g.lda, g.a_rows, g.a_row_index, g.rows_total, g.K, ws, di.err, s, pdl));
+    kf_status st = cuda_status(
+        gather_rows_launch(g.A, g.lda, g.a_rows, g.a_row_index, g.rows_total, g.K, ws, werr, di.err, s, pdl));
     if (st != KF_OK) return st;
     A = ws;
     lda = g.K;
@@ -446,7 +500,7 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, cuda
   p.row_scale = pl.row_scale;
   p.row_dst = pl.row_dst;
   p.dst_rows = static_cast<int32_t>(pl.dst_rows);
-  fill_params_common(p, pl, di.err);
+  fill_params_common(p, pl, werr, di.err);
   p.fast = g.c_dtype == KF_BF16 && pl.mode != kModeScatter;
   if (ex) {
     p.gbias = ex->gbias;
@@ -485,34 +539,56 @@ const char* kf_status_string(int32_t s) {
   }
 }
 
-int32_t kf_abi_version(void) { return 1; }
+int32_t kf_abi_version(void) { return 2; }
 
 kf_status kf_set_wait_timeout_ns(uint64_t ns) {
   g_wait_ns.store(ns == 0 ? kDefaultWaitNs : ns);
   return KF_OK;
 }
 
-kf_status kf_get_device_error(void* stream, uint32_t* raw) {
-  DevInfo di;
-  kf_status st = device_info(&di);
-  if (st != KF_OK) return st;
+}  // extern "C"
+
+namespace {
+// Synchronize `stream`, then read and clear the error word `word` (device memory).
+kf_status read_clear_error(uint32_t* word, void* stream, uint32_t* raw) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return KF_ERR_CUDA;
   uint32_t v = 0, z = 0;
-  if (cudaMemcpy(&v, di.err, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return KF_ERR_CUDA;
-  if (v && cudaMemcpy(di.err, &z, sizeof(z), cudaMemcpyHostToDevice) != cudaSuccess) return KF_ERR_CUDA;
+  if (cudaMemcpy(&v, word, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return KF_ERR_CUDA;
+  if (v && cudaMemcpy(word, &z, sizeof(z), cudaMemcpyHostToDevice) != cudaSuccess) return KF_ERR_CUDA;
   if (raw) *raw = v;
   if (v & (kErrWaitProducer | kErrWaitMma | kErrWaitEpilogue)) return KF_ERR_DEVICE_TIMEOUT;
   if (v & kErrBounds) return KF_ERR_DEVICE_BOUNDS;
   if (v & kErrLaunchShape) return KF_ERR_CUDA;
   return KF_OK;
 }
+}  // namespace
+
+extern "C" {
+
+kf_status kf_get_device_error(void* stream, uint32_t* raw) {
+  DevInfo di;
+  kf_status st = device_info(&di);
+  if (st != KF_OK) return st;
+  return read_clear_error(di.err, stream, raw);
+}
+
+kf_status kf_check_device_error(void* workspace, void* stream, uint32_t* raw) {
+  if (!workspace || !aligned16(workspace)) return KF_ERR_INVALID_ARG;
+  return read_clear_error(static_cast<uint32_t*>(workspace), stream, raw);
+}
+
+kf_status kf_workspace_init(void* workspace, size_t bytes, void* stream) {
+  if (!workspace || !aligned16(workspace) || bytes < kWsHeader) return KF_ERR_INVALID_ARG;
+  return cuda_status(cudaMemsetAsync(workspace, 0, kWsHeader, static_cast<cudaStream_t>(stream)));
+}
 
 size_t kf_fused_gemm_workspace(int64_t M, int64_t N, int64_t K, const kf_epilogue* epi) {
   (void)K;
   if (!epi || M <= 0 || N <= 0) return 0;
   for (int i = 0; i < epi->num_ops && epi->ops; ++i)
-    if (epi->ops[i].kind == KF_OP_ROW_LOGSUMEXP) return lse_ws_bytes(M, N);
-  if (gn512_pairs(epi, M, N)) return couple_ws_bytes(M, N);  // optional: enables the couples
+    if (epi->ops[i].kind == KF_OP_ROW_LOGSUMEXP || epi->ops[i].kind == KF_OP_ROW_SUM)
+      return with_header(lse_ws_bytes(M, N));
+  if (gn512_pairs(epi, M, N)) return with_header(couple_ws_bytes(M, N));  // optional: enables the couples
   return 0;
 }
 
@@ -522,9 +598,15 @@ kf_status kf_fused_gemm(const void* X, int32_t xt, int64_t ldx, const void* W, i
   return kf_fused_gemm_ex(X, xt, ldx, W, wt, ldw, Y, yt, ldy, M, N, K, epi, workspace, ws_bytes, 0u, stream);
 }
 
-kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt, int64_t ldw, void* Y,
-                           int32_t yt, int64_t ldy, int64_t M, int64_t N, int64_t K, const kf_epilogue* epi,
-                           void* workspace, size_t ws_bytes, uint32_t flags, void* stream) {
+}  // extern "C"
+
+namespace {
+// kf_fused_gemm_ex on a split workspace: `payload` / `ws_bytes` is the scratch
+// (row partials, GroupNorm exchange area), `werr` the call's error word (null:
+// the device word only).
+kf_status fused_gemm_impl(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt, int64_t ldw, void* Y,
+                          int32_t yt, int64_t ldy, int64_t M, int64_t N, int64_t K, const kf_epilogue* epi,
+                          void* workspace, size_t ws_bytes, uint32_t* werr, uint32_t flags, void* stream) {
   if (flags & ~(KF_GEMM_F32_FFMA | KF_GEMM_F32_TF32X3)) return KF_ERR_INVALID_ARG;
   if ((flags & KF_GEMM_F32_FFMA) && (flags & KF_GEMM_F32_TF32X3)) return KF_ERR_INVALID_ARG;
   if (M < 0 || N < 0 || K < 1) return KF_ERR_INVALID_ARG;
@@ -536,7 +618,7 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
   ChainPlan pl;
   kf_status st = plan_chain(epi, N, false, &pl);
   if (st != KF_OK) return st;
-  if (pl.mode != kModeLse && ldy < N) return KF_ERR_INVALID_ARG;
+  if (pl.mode != kModeLse && !pl.red_sum && ldy < N) return KF_ERR_INVALID_ARG;
   const bool f32_path = xt == KF_F32 && wt == KF_F32;
   // fp32 operands: FFMA for small problems, three tf32 tensor-core products for
   // large ones (>= 2^30 FLOP), or as the flags say
@@ -556,7 +638,7 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
     // tensor-core path: A and B both bf16 or both fp16 (one operand format per MMA)
     if (xt != wt || (xt != KF_BF16 && xt != KF_F16)) return KF_ERR_UNSUPPORTED;
     if (!aligned16(X) || !aligned16(W) || ldx % 8 != 0 || ldw % 8 != 0) return KF_ERR_MISALIGNED;
-    if (pl.mode == kModeLse &&
+    if ((pl.mode == kModeLse || pl.red_sum) &&
         (!workspace || !aligned16(workspace) || ws_bytes < lse_ws_bytes(M, N)))
       return KF_ERR_WORKSPACE;
   }
@@ -564,6 +646,7 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
   DevInfo di;
   st = device_info(&di);
   if (st != KF_OK) return st;
+  if (!werr) werr = di.err;
 
   if (tf32x3) {
     // tile width: 256 columns (each MMA does twice the work of a 128-wide one
@@ -589,7 +672,8 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
     tp.ldy = ldy;
     tp.y_dtype = yt;
     tp.y_vec_ok = aligned16(Y) && (ldy * elt_size(yt)) % 16 == 0;
-    tp.err = di.err;
+    tp.err = werr;
+    tp.err_dev = di.err;
     tp.wait_ns = g_wait_ns.load();
     tp.drain_ns = std::max<uint64_t>(tp.wait_ns, 1000000000ull);
     const int64_t tiles = static_cast<int64_t>(tp.tiles_m) * tp.tiles_n;
@@ -621,7 +705,7 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
   const bool quad = cta2 && pl.mode == kModeGroupNorm && pl.gs == 512 && di.nsm >= 4 && tc_dense4_has(pl.mode, 256);
   // with a workspace for the statistics exchange: couples of CTA pairs instead
   // (all co-resident pairs work; clusters of four leave SMs idle)
-  const bool couple = quad && tc_couple_has(pl.mode, 256) && workspace && aligned16(workspace) &&
+  const bool couple = quad && !pl.red_sum && tc_couple_has(pl.mode, 256) && workspace && aligned16(workspace) &&
                       ws_bytes >= couple_ws_bytes(M, N);
   int bn = 0, sub = 1;
   int64_t tiles_n = 0;
@@ -656,17 +740,20 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
   p.ldc = ldy;
   p.c_dtype = yt;
   p.c_vec_ok = aligned16(Y) && (ldy * elt_size(yt)) % 16 == 0;
-  if (pl.mode == kModeLse) p.lse_part = static_cast<float2*>(workspace);
-  fill_params_common(p, pl, di.err);
+  if (pl.mode == kModeLse || pl.red_sum) p.lse_part = static_cast<float2*>(workspace);
+  // GroupNorm + row sum: one partial per 256-column block of a row
+  p.red_parts = pl.mode == kModeGroupNorm ? static_cast<int32_t>((N + 255) / 256) : p.tiles_n;
+  fill_params_common(p, pl, werr, di.err);
   CUtensorMap mc;
   std::memset(&mc, 0, sizeof(mc));
-  if ((pl.mode == kModeStore || pl.mode == kModeGroupNorm) && yt == KF_BF16 && p.c_vec_ok) {
+  if ((pl.mode == kModeStore || pl.mode == kModeGroupNorm) && !pl.red_sum && yt == KF_BF16 && p.c_vec_ok) {
     st = make_map_out(&mc, Y, static_cast<uint64_t>(N), static_cast<uint64_t>(M), static_cast<uint64_t>(ldy) * 2);
     if (st != KF_OK) return st;
     p.c_tma = 1;
   }
-  // 16-bit results: reduced-precision activations suffice
-  p.fast = (yt == KF_BF16 || yt == KF_F16) && pl.mode != kModeLse;
+  // 16-bit results: reduced-precision activations suffice (not under a row
+  // reduction: its sum of thousands of values needs each term at fp32)
+  p.fast = (yt == KF_BF16 || yt == KF_F16) && pl.mode != kModeLse && !pl.red_sum;
   p.ab_f16 = xt == KF_F16;
   const int grid = cta2 ? 2 * std::min(p.total_units, di.nsm / 2) : std::min(p.total_units, di.nsm);
   // a compiled chain program, if the chain matches one (bf16 operands staged)
@@ -699,17 +786,28 @@ kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W
     st = cuda_status(tc_dense4_launch(pl.mode, bn, sig, ma, mb, mc, p, s));
   else
     st = cuda_status(tc_dense_launch(pl.mode, bn, cta2, sig, ma, mb, mc, mr, p, sub, grid, s));
-  if (st != KF_OK || pl.mode != kModeLse) return st;
+  if (st != KF_OK || (pl.mode != kModeLse && !pl.red_sum)) return st;
   LseCombineParams cp;
   std::memset(&cp, 0, sizeof(cp));
   cp.part = p.lse_part;
   cp.M = p.M;
-  cp.parts = p.tiles_n;
+  cp.parts = p.red_parts;
   cp.out = Y;
   cp.out_dtype = yt;
-  cp.n_post = pl.n_post;
-  for (int i = 0; i < pl.n_post; ++i) cp.post[i] = pl.post[i];
+  cp.red_sum = pl.red_sum ? 1 : 0;
+  cp.n_post = pl.n_fin;
+  for (int i = 0; i < pl.n_fin; ++i) cp.post[i] = pl.fin[i];
   return cuda_status(lse_combine_launch(cp, s, true));
+}
+}  // namespace
+
+extern "C" {
+
+kf_status kf_fused_gemm_ex(const void* X, int32_t xt, int64_t ldx, const void* W, int32_t wt, int64_t ldw, void* Y,
+                           int32_t yt, int64_t ldy, int64_t M, int64_t N, int64_t K, const kf_epilogue* epi,
+                           void* workspace, size_t ws_bytes, uint32_t flags, void* stream) {
+  const WsView v = split_ws(workspace, ws_bytes);
+  return fused_gemm_impl(X, xt, ldx, W, wt, ldw, Y, yt, ldy, M, N, K, epi, v.payload, v.bytes, v.err, flags, stream);
 }
 
 kf_status kf_moe_route(const float* logits, int64_t T, int32_t E, int32_t k, int32_t* topk_ids, float* topk_w,
@@ -731,7 +829,7 @@ size_t kf_grouped_gemm_workspace(int64_t rows_total, int64_t N, int64_t K, int32
   (void)G;
   (void)epi;
   if (rows_total <= 0 || K <= 0) return 0;
-  return grouped_ws_bytes(rows_total, K, gathered != 0);
+  return with_header(grouped_ws_bytes(rows_total, K, gathered != 0));
 }
 
 kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows, const int32_t* a_row_index,
@@ -755,16 +853,14 @@ kf_status kf_grouped_gemm(const void* A, int32_t at, int64_t lda, int64_t a_rows
   if (!aligned16(A) || !aligned16(B) || lda % 8 != 0 || ldb % 8 != 0 || b_group_stride % 8 != 0)
     return KF_ERR_MISALIGNED;
   if (a_row_index && K % 8 != 0) return KF_ERR_MISALIGNED;
-  if (a_row_index) {
-    if (!workspace || !aligned16(workspace) || ws_bytes < grouped_ws_bytes(rows_total, K, true))
-      return KF_ERR_WORKSPACE;
-  }
+  const WsView v = split_ws(workspace, ws_bytes);
+  if (a_row_index && (!v.payload || v.bytes < grouped_ws_bytes(rows_total, K, true))) return KF_ERR_WORKSPACE;
   DevInfo di;
   st = device_info(&di);
   if (st != KF_OK) return st;
   GroupedArgs g{A, lda, a_row_index ? a_rows : rows_total, a_row_index, B, ldb,
                 G > 1 ? b_group_stride : nb * ldb, offsets, G, rows_total, N, K, C, ct, ldc};
-  return grouped_core(g, pl, workspace, static_cast<cudaStream_t>(stream), di, false);
+  return grouped_core(g, pl, v.payload, v.err ? v.err : di.err, static_cast<cudaStream_t>(stream), di, false);
 }
 
 // Workspace layout of kf_moe_ffn (each region 256-byte aligned):
@@ -809,7 +905,7 @@ size_t kf_moe_ffn_workspace(int64_t T, int64_t H, int64_t I, int32_t E, int32_t 
 
 size_t kf_moe_ffn_workspace_ex(int64_t T, int64_t H, int64_t I, int32_t E, int32_t k, uint32_t flags) {
   if (T < 0 || H < 1 || I < 1 || E < 1 || k < 1) return 0;
-  return moe_layout(T, H, I, E, k, flags).total;
+  return kWsHeader + moe_layout(T, H, I, E, k, flags).total;
 }
 
 kf_status kf_moe_ffn(const void* X, const float* logits, const void* W_gu, const void* W_down, void* Y, int64_t T,
@@ -849,12 +945,14 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
   if (det && H % 4 != 0) return KF_ERR_MISALIGNED;
   if (T == 0) return KF_OK;
   const MoeLayout L = moe_layout(T, H, I, E, k, flags);
-  if (!workspace || !aligned16(workspace) || ws_bytes < L.total) return KF_ERR_WORKSPACE;
+  const WsView v = split_ws(workspace, ws_bytes);
+  if (!v.payload || v.bytes < L.total) return KF_ERR_WORKSPACE;
   DevInfo di;
   kf_status st = device_info(&di);
   if (st != KF_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  char* ws = static_cast<char*>(workspace);
+  char* ws = static_cast<char*>(v.payload);
+  uint32_t* werr = v.err;
   auto* ids = reinterpret_cast<int32_t*>(ws + L.ids);
   auto* w = reinterpret_cast<float*>(ws + L.w);
   auto* off = reinterpret_cast<int32_t*>(ws + L.off);
@@ -895,7 +993,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
       ex.sw_limit = act->limit;
       ex.sw_c = act->linear_offset;
     }
-    st = grouped_core(g, pl, xg, s, di, true, &ex);
+    st = grouped_core(g, pl, xg, werr, s, di, true, &ex);
     if (st != KF_OK) return st;
   }
   if (det) {
@@ -915,7 +1013,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
       ex.gbias = act->b_down;
       ex.gbias_ld = H;
     }
-    st = grouped_core(g, pl, nullptr, s, di, true, &ex);
+    st = grouped_core(g, pl, nullptr, werr, s, di, true, &ex);
     if (st != KF_OK) return st;
     if (tail)
       st = cuda_status(moe_add_rmsnorm_launch(nullptr, yp, pos, k, T, H, tail->R, tail->gamma, tail->eps, tail->R_out, Y,
@@ -941,7 +1039,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
       ex.gbias = act->b_down;
       ex.gbias_ld = H;
     }
-    st = grouped_core(g, pl, nullptr, s, di, true, &ex);
+    st = grouped_core(g, pl, nullptr, werr, s, di, true, &ex);
     if (st != KF_OK) return st;
     if (tail)
       st = cuda_status(moe_add_rmsnorm_launch(yacc, nullptr, nullptr, k, T, H, tail->R, tail->gamma, tail->eps,
@@ -1045,11 +1143,12 @@ extern "C" kf_status kf_fused_gemm_lse_noalloc(const void* X, int32_t xt, int64_
   if (M == 0 || N == 0) return KF_OK;
   const size_t need = kf::lse_ws_bytes(M, N);
   if (need > kf::kNoAllocScratchBytes) return KF_ERR_WORKSPACE;  // problem exceeds the fixed scratch
-  if (xt != KF_BF16 || wt != KF_BF16) return KF_ERR_UNSUPPORTED;
   void* scratch = nullptr;
   kf_status st = kf::noalloc_scratch(&scratch);
   if (st != KF_OK) return st;
-  return kf_fused_gemm(X, xt, ldx, W, wt, ldw, Y, yt, 1, M, N, K, epi, scratch, kf::kNoAllocScratchBytes, stream);
+  // the whole array holds row partials; device-side errors go to the device word
+  return fused_gemm_impl(X, xt, ldx, W, wt, ldw, Y, yt, 1, M, N, K, epi, scratch, kf::kNoAllocScratchBytes, nullptr,
+                         0u, stream);
 }
 
 namespace kf {
@@ -1194,7 +1293,7 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
   p.ldc = ldq;
   p.c_dtype = out_dtype;
   p.c_vec_ok = aligned16(q_out) && (ldq * elt_size(out_dtype)) % 16 == 0;
-  fill_params_common(p, pl, di.err);
+  fill_params_common(p, pl, di.err, di.err);
   p.res_op = -1;
   p.vec_op = -1;
   p.fast = 0;

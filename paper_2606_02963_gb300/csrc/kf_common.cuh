@@ -23,6 +23,13 @@ constexpr uint32_t kErrWaitEpilogue = 4u;
 constexpr uint32_t kErrBounds = 8u;
 constexpr uint32_t kErrLaunchShape = 16u;  // grid or cluster shape not the variant's
 
+// Record error bits in the call's error word and in the device-wide word (the
+// same word when the call has no workspace).
+__device__ __forceinline__ void raise_err(uint32_t* call_word, uint32_t* dev_word, uint32_t bits) {
+  atomicOr(call_word, bits);
+  if (dev_word != nullptr && dev_word != call_word) atomicOr(dev_word, bits);
+}
+
 struct DevOp {
   int32_t kind;
   float scalar;
@@ -70,9 +77,15 @@ struct TcParams {
   const float* row_scale;   // scatter
   const int32_t* row_dst;   // scatter
   int32_t dst_rows;         // scatter: rows of C (bounds)
-  uint32_t* err;
+  uint32_t* err;        // error word of the call: its workspace's header, else the device word
+  uint32_t* err_dev;    // the per-device error word (also written, for the device-wide view)
   uint64_t wait_ns;
   uint64_t drain_ns;
+  // row sum instead of a row log-sum-exp (kModeLse), or after the GroupNorm's
+  // post chain (kModeGroupNorm): per-tile row partials go to lse_part, red_parts
+  // per row (kModeGroupNorm: one per 256-column block), nothing else is stored
+  int32_t red_sum;
+  int32_t red_parts;
   int32_t fast;         // reduced-precision activations (result stored as bf16)
   int32_t res_op;       // index in pre[] of a bf16 RESIDUAL_ADD staged by coalesced loads, or -1
   int32_t vec_op;       // index in pre[] of a bf16 BIAS / MUL whose vector is loaded ahead, or -1
@@ -463,9 +476,14 @@ __device__ __forceinline__ void tanh2_fast(float a, float b, float& ta, float& t
 // c1 = 0.044715 c0 -- each step one f16x2 instruction.  f16 keeps 11
 // significant bits (bf16 keeps 8).  Past |x| ~ 150 the tanh argument overflows
 // to +-inf and tanh saturates at +-1, which is the function's limit.
+// Inputs beyond fp16's range: the conversion saturates to +-65504 (never
+// +-inf, so x < -65504 gives h + h * (-1) = 0, not inf - inf), and the result
+// is max(g, x - 1/2): x - gelu(x) lies in [0, 0.17] for x >= 0 and x - 1/2 <
+// gelu(x) for x < 0, so below 65504 this keeps g, and above it (where g stops
+// at 65504) it gives x - 1/2, which bf16 cannot tell from gelu(x) = x.
 __device__ __forceinline__ void gelu2_f16(float& a, float& b) {
   uint32_t x, g;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(x) : "f"(b), "f"(a));
+  asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(x) : "f"(b), "f"(a));
   asm("{\n\t.reg .b32 u, p, q, t, h;\n\t"
       "mul.rn.f16x2 u, %1, %1;\n\t"
       "fma.rn.f16x2 p, u, %2, %3;\n\t"
@@ -476,8 +494,8 @@ __device__ __forceinline__ void gelu2_f16(float& a, float& b) {
       : "=r"(g)
       : "r"(x), "r"(0x28912891u), "r"(0x3a623a62u), "r"(0x38003800u));  // c1, c0, 1/2 (f16 pairs)
   const __half2 h2 = *reinterpret_cast<const __half2*>(&g);
-  a = __low2float(h2);
-  b = __high2float(h2);
+  a = fmaxf(__low2float(h2), a - 0.5f);
+  b = fmaxf(__high2float(h2), b - 0.5f);
 }
 __device__ __forceinline__ float f_gelu_tanh_fast(float x) {
   const float c = 0.7978845608028654f;

@@ -61,7 +61,8 @@ struct Tf32Params {
   int64_t ldy;
   int32_t y_dtype;
   int32_t y_vec_ok;
-  uint32_t* err;
+  uint32_t* err;        // the call's error word (its workspace's header, else the device word)
+  uint32_t* err_dev;    // the per-device error word
   uint64_t wait_ns;
   uint64_t drain_ns;
 };
@@ -144,6 +145,7 @@ struct LseCombineParams {
   int32_t parts;
   void* out;
   int32_t out_dtype;
+  int32_t red_sum;      // partials are row sums (.y): add them instead of the (max, sum exp) merge
   int32_t n_post;
   DevOp post[kMaxOps];
 };
@@ -170,7 +172,7 @@ cudaError_t moe_add_rmsnorm_launch(const float* yacc, const float* yp, const int
                                    int64_t H, const void* R, const void* gamma, float eps, void* R_out, void* Y,
                                    cudaStream_t s, bool pdl);
 cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
-                               int64_t K, void* out, uint32_t* err, cudaStream_t s, bool pdl);
+                               int64_t K, void* out, uint32_t* err, uint32_t* err_dev, cudaStream_t s, bool pdl);
 cudaError_t cvt_f32_bf16_launch(const float* in, void* out, int64_t n, cudaStream_t s, bool pdl);
 
 }  // namespace kf

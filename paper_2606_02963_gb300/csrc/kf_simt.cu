@@ -83,6 +83,25 @@ __global__ void lse_combine_kernel(const __grid_constant__ LseCombineParams p) {
   const int lane = threadIdx.x & 31;
   if (row >= p.M) return;
   const float2* part = p.part + static_cast<int64_t>(row) * p.parts;
+  if (p.red_sum) {
+    // row sum: the partials' sums, lane-strided then a fixed butterfly (the
+    // same order on every call)
+    float s = 0.f;
+    for (int i = lane; i < p.parts; i += 32) s += part[i].y;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) {
+      float v = s;
+      for (int o = 0; o < p.n_post; ++o) v = apply_scalar_op(p.post[o], v);
+      if (p.out_dtype == KF_BF16)
+        reinterpret_cast<__nv_bfloat16*>(p.out)[row] = __float2bfloat16_rn(v);
+      else if (p.out_dtype == KF_F16)
+        reinterpret_cast<__half*>(p.out)[row] = __float2half_rn(v);
+      else
+        reinterpret_cast<float*>(p.out)[row] = v;
+    }
+    return;
+  }
   float m = -INFINITY, s = 0.f;
   for (int i = lane; i < p.parts; i += 32) {
     const float2 q = part[i];
@@ -513,7 +532,7 @@ cudaError_t moe_add_rmsnorm_launch(const float* yacc, const float* yp, const int
 // range writes a zero row and sets the bounds bit of the error word.
 __global__ void gather_rows_kernel(const uint4* __restrict__ A, int64_t lda_v, int64_t a_rows,
                                    const int32_t* __restrict__ idx, int64_t rows, int64_t kv,
-                                   uint4* __restrict__ out, uint32_t* err) {
+                                   uint4* __restrict__ out, uint32_t* err, uint32_t* err_dev) {
   griddep_wait();  // after the library kernel this one follows (programmatic launch)
   griddep_launch_dependents();
   const int64_t total = rows * kv;
@@ -525,18 +544,18 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ A, int64_t lda_v, i
     if (src >= 0 && src < a_rows)
       v = __ldg(A + src * lda_v + c);
     else if (c == 0)
-      atomicOr(err, kErrBounds);
+      raise_err(err, err_dev, kErrBounds);
     out[i] = v;
   }
 }
 
 cudaError_t gather_rows_launch(const void* A, int64_t lda, int64_t a_rows, const int32_t* idx, int64_t rows,
-                               int64_t K, void* out, uint32_t* err, cudaStream_t s, bool pdl) {
+                               int64_t K, void* out, uint32_t* err, uint32_t* err_dev, cudaStream_t s, bool pdl) {
   if (rows == 0) return cudaSuccess;
   const int64_t kv = K / 8, total = rows * kv;
   int blocks = static_cast<int>(std::min<int64_t>((total + 255) / 256, 148 * 16));
   return launch_k(gather_rows_kernel, dim3(blocks), dim3(256), 0, s, pdl, reinterpret_cast<const uint4*>(A), lda / 8,
-                  a_rows, idx, rows, kv, reinterpret_cast<uint4*>(out), err);
+                  a_rows, idx, rows, kv, reinterpret_cast<uint4*>(out), err, err_dev);
 }
 
 // ------------------------------------------------------------ fp32 -> bf16

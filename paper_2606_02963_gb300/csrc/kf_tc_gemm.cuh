@@ -178,7 +178,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     const uint32_t ncl = CTA2 ? cluster_nctarank() : 1u;
     if (ncl != kCluster || blockDim.x != static_cast<uint32_t>(Cfg::kThr) || gridDim.x % kGridMult != 0 ||
         gridDim.y != 1 || gridDim.z != 1) {
-      if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
+      if (threadIdx.x == 0) raise_err(p.err, p.err_dev, kErrLaunchShape);
       return;
     }
   }
@@ -266,7 +266,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
         prev = o;
       }
       if (!ok) {
-        atomicOr(p.err, kErrBounds);
+        raise_err(p.err, p.err_dev, kErrBounds);
         units = 0;
       }
       if (ok) ustart_s[p.G] = units;
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             const uint32_t ph = (it / STAGES) & 1;
             if (!mbar_wait(&empty[st], ph ^ 1, abort_flag, p.wait_ns)) {
               *abort_flag = 1;
-              atomicOr(p.err, kErrWaitProducer);
+              raise_err(p.err, p.err_dev, kErrWaitProducer);
               ok = false;
               break;
             }
@@ -375,7 +375,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
               const uint32_t ph = (it / STAGES) & 1;
               if (!mbar_wait(&empty[st], ph ^ 1, abort_flag, p.wait_ns)) {
                 *abort_flag = 1;
-                atomicOr(p.err, kErrWaitProducer);
+                raise_err(p.err, p.err_dev, kErrWaitProducer);
                 ok = false;
                 break;
               }
@@ -468,7 +468,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
       }
       if (!ok) {
         *abort_flag = 1;
-        atomicOr(p.err, kErrWaitMma);
+        raise_err(p.err, p.err_dev, kErrWaitMma);
         // arrives once every MMA issued so far has completed
         if constexpr (CTA2)
           tc_commit_pair(drain);
@@ -512,7 +512,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
       w = __all_sync(0xffffffffu, w);
       if (!w) {
         *abort_flag = 1;
-        if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+        if (lane == 0) raise_err(p.err, p.err_dev, kErrWaitEpilogue);
         return false;
       }
       tc_fence_after();
@@ -608,7 +608,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           got = __all_sync(0xffffffffu, got);
           if (!got) {
             *abort_flag = 1;
-            if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+            if (lane == 0) raise_err(p.err, p.err_dev, kErrWaitEpilogue);
             ok = false;
             break;
           }
@@ -627,7 +627,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             rs = p.row_scale[grow];
             dst = p.row_dst[grow];
             if (dst < 0 || dst >= p.dst_rows) {
-              atomicOr(p.err, kErrBounds);
+              raise_err(p.err, p.err_dev, kErrBounds);
               wr = false;
             }
           }
@@ -774,7 +774,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
         if (!wait_acc(tl)) { ok = false; break; }
         bool wr = row_ok;
         if (row_ok && (pos < 0 || pos >= p.rope_max_pos || crow < 0 || crow >= p.dst_rows)) {
-          atomicOr(p.err, kErrBounds);
+          raise_err(p.err, p.err_dev, kErrBounds);
           wr = false;
         }
         const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
@@ -842,6 +842,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
       } else if constexpr (MODE == kModeLse) {
         if (!pair_vote(wait_acc(tl))) { ok = false; break; }
         const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
+        const bool rsum = p.red_sum != 0;  // row sum (s only) instead of (max, sum exp)
         float m = -INFINITY, s = 0.0f;
         for (int c = h; c < BN / 32; c += 2) {
           const int32_t col0 = ui.n0 + c * 32;
@@ -851,6 +852,14 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           float v[32];
           tmem_ld32(tb + c * 32, v);
           run_chain<PRE>(false, p.pre, p.n_pre, v, grow, col0, nvalid, row_ok);
+          if (rsum) {
+            float add = 0.0f;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j < nvalid) add += v[j];
+            s += add;
+            continue;
+          }
           float cm = -INFINITY;
 #pragma unroll
           for (int j = 0; j < 32; ++j)
@@ -870,16 +879,38 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
         pair_sync();
         if (h == 0) {
           const float2 o = xch[row_in_tile];
-          const float nm = fmaxf(m, o.x);
-          float ss = 0.0f;
-          if (nm != -INFINITY)
-            ss = (m == -INFINITY ? 0.f : s * __expf(m - nm)) + (o.x == -INFINITY ? 0.f : o.y * __expf(o.x - nm));
-          if (row_ok) p.lse_part[static_cast<int64_t>(grow) * p.tiles_n + ui.n_blk] = make_float2(nm, ss);
+          float2 part;
+          if (rsum) {
+            part = make_float2(0.0f, s + o.y);  // half 0's columns, then half 1's
+          } else {
+            const float nm = fmaxf(m, o.x);
+            float ss = 0.0f;
+            if (nm != -INFINITY)
+              ss = (m == -INFINITY ? 0.f : s * __expf(m - nm)) + (o.x == -INFINITY ? 0.f : o.y * __expf(o.x - nm));
+            part = make_float2(nm, ss);
+          }
+          if (row_ok) p.lse_part[static_cast<int64_t>(grow) * p.tiles_n + ui.n_blk] = part;
         }
         pair_sync();  // xch is reused by the next tile
       } else if constexpr (MODE == kModeGroupNorm) {
         const int32_t gs = p.norm.groups;  // group size (columns), multiple of 32
         const float eps = p.norm.eps;
+        // a row sum after the post chain (red_sum): each thread adds up the
+        // chunks it finishes instead of storing them; the quadrant's two warps
+        // then merge (half 0 first) and write one partial per 256-column block
+        const bool gn_sum = p.red_sum != 0;
+        float rsum = 0.0f;
+        auto emit_sum = [&](int32_t col_base, int blocks) {
+          xch[h * kBM + row_in_tile] = make_float2(rsum, 0.0f);
+          pair_sync();
+          if (h == 0 && row_ok) {
+            const float tot = rsum + xch[kBM + row_in_tile].x;
+            float2* dst = p.lse_part + static_cast<int64_t>(grow) * p.red_parts + col_base / 256;
+            dst[0] = make_float2(0.0f, tot);
+            for (int b = 1; b < blocks && col_base / 256 + b < p.red_parts; ++b) dst[b] = make_float2(0.0f, 0.0f);
+          }
+          pair_sync();  // xch is reused by the next unit
+        };
         // normalise + affine + post chain + store one 32-column chunk
         // bias / gamma / beta of this warp's chunks of one accumulator, loaded
         // once into the warp's cache (coalesced, lane j = column j) so the
@@ -943,6 +974,13 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             v[4 * k + 3] = (v[4 * k + 3] - mean) * rstd * g.w + t.w;
           }
           run_chain<POST>(fast, p.post, p.n_post, v, grow, col0, 32, row_ok);
+          if (gn_sum) {
+            float add = 0.0f;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) add += v[j];
+            rsum += add;
+            return;
+          }
           if (c_tma)
             store_tile32_tma(stage, lane, v, &tmC, col0, wrow0);
           else if (c_tiles)
@@ -1028,7 +1066,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             got = __all_sync(0xffffffffu, got);
             if (!pair_vote(got)) {
               *abort_flag = 1;
-              if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+              if (lane == 0) raise_err(p.err, p.err_dev, kErrWaitEpilogue);
               ok = false;
               break;
             }
@@ -1061,7 +1099,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             got = __all_sync(0xffffffffu, got);
             if (!pair_vote(got)) {
               *abort_flag = 1;
-              if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+              if (lane == 0) raise_err(p.err, p.err_dev, kErrWaitEpilogue);
               ok = false;
               break;
             }
@@ -1080,9 +1118,13 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           __syncwarp();
           release_acc(tl);
           ++tl;
+          if (gn_sum) emit_sum(ui.n0, 1);
         } else if (gs < BN) {
           // several whole groups per tile: half h takes groups h, h+2, ...
-          if (!wait_acc(tl)) { ok = false; break; }
+          // (a row sum merges the halves after the tile: both vote first)
+          bool got = wait_acc(tl);
+          if (gn_sum) got = pair_vote(got);
+          if (!got) { ok = false; break; }
           const uint32_t tb = tmem + lane_off + (tl & 1) * Cfg::kAccStride;
           const int nch = gs / 32;
           for (int gi = h; gi < BN / gs; gi += 2) {
@@ -1100,6 +1142,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           }
           release_acc(tl);
           ++tl;
+          if (gn_sum) emit_sum(ui.n0, 1);
         } else {
           // one group spans sub_tiles (1 or 2) accumulators of BN columns; the two
           // halves split its chunks and merge their moments through shared memory
@@ -1136,6 +1179,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
             release_acc(tl + st);
           }
           tl += sub_tiles;
+          if (gn_sum) emit_sum(ui.n0, sub_tiles);
         }
       }
     }

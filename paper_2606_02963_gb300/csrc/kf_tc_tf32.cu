@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kTfThreads, 1)
   auto b_lo = [&](int s) { return sm + s * Cfg::kStageBytes + 2 * Cfg::kABytes + Cfg::kBBytes; };
 
   if (blockDim.x != kTfThreads || gridDim.y != 1 || gridDim.z != 1) {
-    if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
+    if (threadIdx.x == 0) raise_err(p.err, p.err_dev, kErrLaunchShape);
     return;
   }
   const int warp = threadIdx.x >> 5;
@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(kTfThreads, 1)
           const int st = it % STAGES;
           if (!mbar_wait(&empty[st], ((it / STAGES) & 1) ^ 1, abort_flag, p.wait_ns)) {
             *abort_flag = 1;
-            atomicOr(p.err, kErrWaitProducer);
+            raise_err(p.err, p.err_dev, kErrWaitProducer);
             ok = false;
             break;
           }
@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(kTfThreads, 1)
       }
       if (!ok) {
         *abort_flag = 1;
-        atomicOr(p.err, kErrWaitMma);
+        raise_err(p.err, p.err_dev, kErrWaitMma);
         tc_commit(drain);  // arrives once every MMA issued so far has completed
         mbar_wait(drain, 0, zero_flag, p.drain_ns);
       }
@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(kTfThreads, 1)
         w = __all_sync(0xffffffffu, w);
         if (!w) {
           *abort_flag = 1;
-          if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+          if (lane == 0) raise_err(p.err, p.err_dev, kErrWaitEpilogue);
           ok = false;
           break;
         }
@@ -250,7 +250,7 @@ __global__ void __launch_bounds__(kTfThreads, 1)
       w = __all_sync(0xffffffffu, w);
       if (!w) {
         *abort_flag = 1;
-        if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
+        if (lane == 0) raise_err(p.err, p.err_dev, kErrWaitEpilogue);
         break;
       }
       tc_fence_after();

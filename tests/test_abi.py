@@ -41,7 +41,7 @@ def test_library_exports_every_declared_symbol(L):
 
 
 def test_status_strings(L):
-    assert L.kf_abi_version() == 1
+    assert L.kf_abi_version() == 2
     for s in range(8):
         assert len(kf.status_string(s)) > 0
     assert "unknown" in kf.status_string(99)
@@ -104,12 +104,43 @@ def test_fused_gemm_chain_errors(L):
     assert need >= 1000 * 8 * 8
     assert fused(L, epi=lse, M=1000, N=1000, ldy=1000) == kf.KF_ERR_WORKSPACE
     assert fused(L, epi=lse, M=1000, N=1000, ws=A16, wsb=need - 1) == kf.KF_ERR_WORKSPACE
+    # row sum: needs the workspace, only scalar ops after it, may follow a
+    # GroupNorm (with pointwise ops between) but nothing else special
+    op = lambda k, **kw: kf.EpilogueOp(kind=k, **kw)
+    ep = lambda *ops: kf.Epilogue(len(ops), ctypes.cast((kf.EpilogueOp * len(ops))(*ops), ctypes.POINTER(kf.EpilogueOp)))
+    rs = ep(op(15))
+    need_rs = L.kf_fused_gemm_workspace(1000, 1000, 64, ctypes.byref(rs))
+    assert need_rs == need and need_rs >= 256 + 1000 * 8 * 8
+    assert fused(L, epi=rs, M=1000, N=1000, ldy=1) == kf.KF_ERR_WORKSPACE
+    assert fused(L, epi=rs, M=1000, N=1000, ws=A16, wsb=need_rs - 1) == kf.KF_ERR_WORKSPACE
+    assert fused(L, epi=ep(op(15), op(0, p0=B16, p_dtype=1)), ws=A16, wsb=1 << 20) == kf.KF_ERR_INVALID_ARG
+    assert fused(L, epi=ep(op(15), op(15))) == kf.KF_ERR_UNSUPPORTED
+    assert fused(L, epi=ep(op(7), op(15))) == kf.KF_ERR_UNSUPPORTED
+    assert fused(L, epi=ep(op(15), op(8, groups=2, eps=1e-5))) == kf.KF_ERR_UNSUPPORTED
+    gn_sum = ep(op(8, groups=2, eps=1e-5), op(12, scalar=0.1), op(15), op(1, scalar=2.0))
+    assert fused(L, epi=gn_sum, N=64, ldy=1) == kf.KF_ERR_WORKSPACE   # planned; needs its partials
+    assert L.kf_fused_gemm_workspace(1000, 1024, 64, ctypes.byref(gn_sum)) >= 256 + 1000 * 8 * 4
+    assert fused(L, epi=ep(op(8, groups=2, eps=1e-5), op(15), op(0, p0=B16, p_dtype=1)), N=64, ldy=1,
+                 ws=A16, wsb=1 << 20) == kf.KF_ERR_INVALID_ARG
     # GroupNorm: N % groups, group size rules
     gn = lambda g: kf.Epilogue(1, ctypes.cast((kf.EpilogueOp * 1)(kf.EpilogueOp(kind=8, groups=g, eps=1e-5)),
                                               ctypes.POINTER(kf.EpilogueOp)))
     assert fused(L, epi=gn(3), N=64, ldy=64) == kf.KF_ERR_INVALID_ARG     # 64 % 3
     assert fused(L, epi=gn(4), N=64, ldy=64) == kf.KF_ERR_UNSUPPORTED     # group of 16 columns
     assert fused(L, epi=gn(0), N=64, ldy=64) == kf.KF_ERR_INVALID_ARG
+
+
+def test_workspace_header_calls_check_arguments(L):
+    # the error-word calls refuse a missing or misaligned workspace before any
+    # device access; the size queries include the header
+    raw = ctypes.c_uint32(0)
+    assert L.kf_check_device_error(None, None, ctypes.byref(raw)) == kf.KF_ERR_INVALID_ARG
+    assert L.kf_check_device_error(A16 + 4, None, ctypes.byref(raw)) == kf.KF_ERR_INVALID_ARG
+    assert L.kf_workspace_init(None, 1 << 20, None) == kf.KF_ERR_INVALID_ARG
+    assert L.kf_workspace_init(A16, 255, None) == kf.KF_ERR_INVALID_ARG
+    assert L.kf_grouped_gemm_workspace(100, 64, 64, 4, 0, None) == 0
+    assert L.kf_grouped_gemm_workspace(100, 64, 64, 4, 1, None) == 256 + 100 * 64 * 2
+    assert L.kf_moe_ffn_workspace(64, 2880, 2880, 32, 4) % 256 == 0
 
 
 def grouped(L, A=A16, at=1, lda=64, a_rows=0, idx=None, B=B16, bt=1, ldb=64, bgs=64 * 64, off=C16, G=4,

@@ -96,6 +96,39 @@ def test_gelu_scale_residual_chain_sweep(dist):
     _no_device_error()
 
 
+@pytest.mark.parametrize("path", ["interpreter", "residual_tile"])
+def test_gelu_far_outside_fp16_range(path):
+    """Pre-activations of +-1e3, +-7e4 and +-3e5 (bf16-exact) among ordinary
+    ones: GELU gives x above zero and ~0 below, never inf or NaN, on the packed
+    fp16 path bf16 outputs take.  X = I makes X W^T = W^T exactly."""
+    g = torch.Generator().manual_seed(31)
+    M = K = 256
+    N = 512
+    big = torch.tensor([1e3, -1e3, 7e4, -7e4, 3e5, -3e5]).to(torch.bfloat16).float()
+    vals = torch.randn(M, N, generator=g) * 3
+    idx = torch.randperm(M * N, generator=g)[:M * N // 7]
+    vals.view(-1)[idx] = big[torch.arange(idx.numel()) % big.numel()]
+    vals = vals.to(torch.bfloat16)
+    X = torch.eye(K).to(torch.bfloat16)
+    W = vals.t().contiguous()
+    if path == "interpreter":
+        chain = [("gelu_tanh", {})]
+    else:  # the headline's compiled chain on CTA pairs (residual tile in shared memory)
+        chain = [("bias", {"p0": torch.zeros(N).to(torch.bfloat16)}), ("gelu_tanh", {}), ("scale", {"scalar": 2.0}),
+                 ("residual_add", {"p0": torch.zeros(M, N).to(torch.bfloat16)})]
+    Y = kf.fused_gemm(X.to(DEV), W.to(DEV), chain_to(chain, DEV))
+    ref = oracle.fused_gemm(X, W, chain)
+    y = to_np(Y)
+    assert np.isfinite(y).all()
+    check_bf16(Y, ref, path)
+    f = 1.0 if path == "interpreter" else 2.0
+    x = vals.double().numpy()
+    hi, lo = x >= 1e3, x <= -1e3
+    assert np.all(np.abs(y[hi] - f * x[hi]) <= 1e-2 * f * x[hi])
+    assert np.all(np.abs(y[lo]) <= 1e-2)
+    _no_device_error()
+
+
 @pytest.mark.parametrize("in_place", [False, True])
 def test_gelu_chain_more_tiles_than_cta_pairs(in_place):
     # 4 ragged 256-row tiles x 20 column tiles of 224 = 80 tiles: more than the

@@ -4,6 +4,8 @@ is not already satisfied gives up; the kernel records a timeout bit in the
 device error word, drains its in-flight copies and MMAs, frees tensor memory and
 returns.  The host reads KF_ERR_DEVICE_TIMEOUT, and the context stays usable: the
 next (normal) call is correct."""
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -62,3 +64,34 @@ def test_grouped_wait_timeout_is_reported():
     C = kf.grouped_gemm(A, B, off, 256, [])
     ref = oracle.grouped_gemm(A.cpu(), B.cpu(), off.cpu().numpy(), 256, [])
     check_bf16(C, ref, "grouped after timeout")
+
+
+def test_error_words_are_per_workspace():
+    """Two streams, two workspaces: the call whose waits are limited to 1 ns
+    reports the timeout in its own workspace's error word; the other call's
+    word stays clean (the device-wide word sees the timeout as well)."""
+    inp = kf_workloads.generate("bf16_scale_rowlse", seed=23, M=512, N=2048, K=512)
+    X, W = inp["X"].to(DEV), inp["W"].to(DEV)
+    chain = [("scale", {"scalar": 0.125}), ("row_logsumexp", {})]
+    need = kf.lib().kf_fused_gemm_workspace(512, 2048, 512, ctypes.byref(kf.make_epilogue(chain, [])))
+    wa, wb = kf.new_workspace(need, DEV), kf.new_workspace(need, DEV)
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    torch.cuda.synchronize()
+    assert kf.get_device_error()[0] == kf.KF_OK
+    try:
+        kf.set_wait_timeout_ns(1)
+        kf.fused_gemm(X, W, chain, workspace=wa, stream=sa)
+    finally:
+        kf.set_wait_timeout_ns(0)
+    yb = kf.fused_gemm(X, W, chain, workspace=wb, stream=sb)
+    stb, rawb = kf.check_device_error(wb, sb)
+    sta, rawa = kf.check_device_error(wa, sa)
+    assert stb == kf.KF_OK, hex(rawb)
+    assert sta == kf.KF_ERR_DEVICE_TIMEOUT and rawa & 0x7, (sta, hex(rawa))
+    assert kf.check_device_error(wa, sa)[0] == kf.KF_OK  # cleared by the read
+    assert kf.get_device_error()[0] == kf.KF_ERR_DEVICE_TIMEOUT
+    assert kf.get_device_error()[0] == kf.KF_OK
+    torch.cuda.synchronize()
+    ref = oracle.fused_gemm(inp["X"], inp["W"], chain)[:, 0]
+    from tests._util import check_f32
+    check_f32(yb, ref, "the other stream's call")

@@ -25,17 +25,19 @@ def _noalloc(X, W, chain, out):
     epi = kf.make_epilogue(chain, keep)
     M, K = X.shape
     N = W.shape[0]
+    dt = kf.KF_F16 if X.dtype == torch.float16 else kf.KF_BF16
     return kf.lib().kf_fused_gemm_lse_noalloc(
-        X.data_ptr(), kf.KF_BF16, X.stride(0), W.data_ptr(), kf.KF_BF16, W.stride(0), out.data_ptr(),
+        X.data_ptr(), dt, X.stride(0), W.data_ptr(), dt, W.stride(0), out.data_ptr(),
         kf.KF_F32, M, N, K, ctypes.byref(epi), torch.cuda.current_stream().cuda_stream)
 
 
-def test_noalloc_lse_matches_workspace_entry_point_on_two_calls():
+@pytest.mark.parametrize("op_dtype", [torch.bfloat16, torch.float16])
+def test_noalloc_lse_matches_workspace_entry_point_on_two_calls(op_dtype):
     problems = [dict(seed=1, M=300, N=2500, K=264, dist="unscaled"),
                 dict(seed=2, M=2048, N=8192, K=8192, dist="default")]
     for pr in problems:
         inp = kf_workloads.generate("bf16_scale_rowlse", **pr)
-        X, W = inp["X"].to(DEV), inp["W"].to(DEV)
+        X, W = inp["X"].to(op_dtype).to(DEV), inp["W"].to(op_dtype).to(DEV)
         chain = [("scale", {"scalar": 0.125}), ("row_logsumexp", {})]
         ref = kf.fused_gemm(X, W, chain)                       # caller-provided workspace
         out = torch.full((X.shape[0],), float("nan"), dtype=torch.float32, device=DEV)
