@@ -22,8 +22,9 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  kern<<<grid, Cfg::kThr, Cfg::kSmemBytes, s>>>(a, b, c, r, p, sub);
-  return cudaGetLastError();
+  // a programmatic dependent of the previous kernel in the stream (see the
+  // CTA-pair launcher): set-up overlaps a preceding call's tail
+  return launch_k(kern, dim3(grid), dim3(Cfg::kThr), Cfg::kSmemBytes, s, true, a, b, c, r, p, static_cast<int32_t>(sub));
 }
 
 }  // namespace

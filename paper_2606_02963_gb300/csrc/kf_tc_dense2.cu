@@ -32,13 +32,20 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtens
   cfg.blockDim = dim3(Cfg::kThr, 1, 1);
   cfg.dynamicSmemBytes = Cfg::kSmemBytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // a programmatic dependent of the previous kernel in the stream: when that
+  // one is also a launch of this library (back-to-back calls), this grid's
+  // barrier set-up and tensor-memory allocation overlap its tail; the kernel
+  // waits for it to complete (griddepcontrol.wait) before any global access.
+  // After any other kernel this is an ordinary stream-ordered launch.
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, a, b, c, r, p, static_cast<int32_t>(sub));
 }
 
