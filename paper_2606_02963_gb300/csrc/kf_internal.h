@@ -1,6 +1,7 @@
 // kf_internal.h -- host-side declarations shared by the library's translation
 // units (kernel launchers); not part of the public ABI.
 #pragma once
+#include <atomic>
 #include <cuda.h>
 #include <cuda_runtime.h>
 

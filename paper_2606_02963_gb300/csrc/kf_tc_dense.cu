@@ -13,7 +13,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
                        const TcParams& p, int sub, int grid, cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, kClOne>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClOne>;
-  static bool configured[64] = {};  // the attribute is per device
+  static std::atomic<bool> configured[64];  // the attribute is per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;

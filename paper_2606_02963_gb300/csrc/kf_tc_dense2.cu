@@ -17,7 +17,7 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, const CUtens
                         const TcParams& p, int sub, int grid, cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, kClPair, kResTileFor<MODE, false, kClPair, PRE>>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClPair, PRE, POST>;
-  static bool configured[64] = {};
+  static std::atomic<bool> configured[64];
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
@@ -57,7 +57,7 @@ cudaError_t launch_quad(const CUtensorMap& a, const CUtensorMap& b, const CUtens
                         cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, kClQuad>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClQuad, PRE, POST>;
-  static int max_clusters[64] = {};  // per device; 0 = not yet queried
+  static std::atomic<int> max_clusters[64];  // per device; 0 = not yet queried
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
@@ -82,7 +82,7 @@ cudaError_t launch_quad(const CUtensorMap& a, const CUtensorMap& b, const CUtens
     if (nc < 1) return cudaErrorInvalidConfiguration;
     max_clusters[dev] = nc;
   }
-  const int clusters = std::min(p.total_units, max_clusters[dev]);
+  const int clusters = std::min(p.total_units, max_clusters[dev].load());
   if (clusters < 1) return cudaSuccess;
   cfg.gridDim = dim3(4 * clusters, 1, 1);
   static const CUtensorMap none = {};  // GroupNorm stages no residual tile
@@ -97,7 +97,7 @@ cudaError_t launch_couple(const CUtensorMap& a, const CUtensorMap& b, const CUte
                           int max_couples, cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, MODE, false, kClCouple>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, false, kClCouple, PRE, POST>;
-  static int max_pairs[64] = {};  // per device; 0 = not yet queried
+  static std::atomic<int> max_pairs[64];  // per device; 0 = not yet queried
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
@@ -124,7 +124,7 @@ cudaError_t launch_couple(const CUtensorMap& a, const CUtensorMap& b, const CUte
     if (nc < 2) return cudaErrorInvalidConfiguration;
     max_pairs[dev] = nc;
   }
-  const int couples = std::min(std::min(p_in.total_units, max_pairs[dev] / 2), max_couples);
+  const int couples = std::min(std::min(p_in.total_units, max_pairs[dev].load() / 2), max_couples);
   if (couples < 1) return cudaSuccess;
   TcParams p = p_in;
   p.gx_couples = couples;

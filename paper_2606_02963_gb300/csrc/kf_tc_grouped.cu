@@ -11,7 +11,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
                        bool pdl) {
   using Cfg = TcCfg<BN, STAGES, MODE, true, kClOne>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, kClOne>;
-  static bool configured[64] = {};  // the attribute is per device
+  static std::atomic<bool> configured[64];  // the attribute is per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;

@@ -344,7 +344,7 @@ cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecod
                       cudaStream_t s) {
   using Cfg = DcCfg<ROWS, STAGES>;
   auto kern = kf_qkv_decode_kernel<ROWS, STAGES>;
-  static bool configured[64] = {};
+  static std::atomic<bool> configured[64];
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
@@ -403,7 +403,7 @@ int qkv_decode_box_rows(int64_t T) { return T <= 32 ? 32 : 64; }
 // co-resident clusters of `splits` CTAs for the decode kernel variant that
 // serves T tokens (queried once per device, variant and cluster size)
 cudaError_t qkv_decode_clusters(int64_t T, int splits, int* out) {
-  static int cache[64][2][9] = {};  // 0: not yet queried
+  static std::atomic<int> cache[64][2][9];  // 0: not yet queried
   if (splits < 1 || splits > 8 || T < 1 || T > kQkvDecodeMaxRows) return cudaErrorInvalidValue;
   int dev = 0;
   cudaGetDevice(&dev);
@@ -415,7 +415,8 @@ cudaError_t qkv_decode_clusters(int64_t T, int splits, int* out) {
     if (e != cudaSuccess) return e;
     cache[dev][v][splits] = nc > 0 ? nc : -1;
   }
-  *out = cache[dev][v][splits] > 0 ? cache[dev][v][splits] : 0;
+  const int c = cache[dev][v][splits].load();
+  *out = c > 0 ? c : 0;
   return cudaSuccess;
 }
 

@@ -17,7 +17,7 @@ template <int BN, int STAGES, int CL>
 cudaError_t launch_rope(const CUtensorMap& a, const CUtensorMap& b, const TcParams& p, int grid, cudaStream_t s) {
   using Cfg = TcCfg<BN, STAGES, kModeRope, false, CL>;
   auto kern = kf_tc_gemm_kernel<BN, STAGES, kModeRope, false, CL>;
-  static bool configured[64] = {};  // the attribute is per device
+  static std::atomic<bool> configured[64];  // the attribute is per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;

@@ -286,7 +286,7 @@ template <int BN, int STAGES>
 cudaError_t launch_tf32(const CUtensorMap& a, const CUtensorMap& b, const Tf32Params& p, int grid, cudaStream_t s) {
   using Cfg = Tf32Cfg<BN, STAGES>;
   auto kern = kf_tf32x3_gemm_kernel<BN, STAGES>;
-  static bool configured[64] = {};
+  static std::atomic<bool> configured[64];
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;

@@ -50,9 +50,13 @@ def test_wait_timeout_is_reported_and_context_survives(M):
 
 
 def test_grouped_wait_timeout_is_reported():
+    # K = 2048 (32 k-blocks): the epilogue's wait for the accumulator outlasts
+    # the hardware's own suspension inside one mbarrier try_wait, so at least
+    # one wait must give up (with two k-blocks every wait could be satisfied
+    # within a single try_wait)
     g = torch.Generator().manual_seed(3)
-    A = torch.randn(300, 128, generator=g).to(torch.bfloat16).to(DEV)
-    B = (torch.randn(3, 256, 128, generator=g) * 0.1).to(torch.bfloat16).to(DEV)
+    A = torch.randn(300, 2048, generator=g).to(torch.bfloat16).to(DEV)
+    B = (torch.randn(3, 256, 2048, generator=g) * 0.02).to(torch.bfloat16).to(DEV)
     off = torch.tensor([0, 100, 100, 300], dtype=torch.int32, device=DEV)
     try:
         kf.set_wait_timeout_ns(1)
@@ -70,10 +74,10 @@ def test_error_words_are_per_workspace():
     """Two streams, two workspaces: the call whose waits are limited to 1 ns
     reports the timeout in its own workspace's error word; the other call's
     word stays clean (the device-wide word sees the timeout as well)."""
-    inp = kf_workloads.generate("bf16_scale_rowlse", seed=23, M=512, N=2048, K=512)
+    inp = kf_workloads.generate("bf16_scale_rowlse", seed=23, M=512, N=2048, K=2048)
     X, W = inp["X"].to(DEV), inp["W"].to(DEV)
     chain = [("scale", {"scalar": 0.125}), ("row_logsumexp", {})]
-    need = kf.lib().kf_fused_gemm_workspace(512, 2048, 512, ctypes.byref(kf.make_epilogue(chain, [])))
+    need = kf.lib().kf_fused_gemm_workspace(512, 2048, 2048, ctypes.byref(kf.make_epilogue(chain, [])))
     wa, wb = kf.new_workspace(need, DEV), kf.new_workspace(need, DEV)
     sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
     torch.cuda.synchronize()
