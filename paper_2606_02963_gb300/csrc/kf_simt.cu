@@ -29,46 +29,108 @@ __device__ __forceinline__ float apply_chain1(const DevOp* ops, int n, float v, 
 }
 
 // ------------------------------------------------------------------ fp32 GEMM
-// 32x32 output tile per 256-thread block, 2x2 outputs per thread, K in steps
-// of 32 through shared memory (both operands K-contiguous in global memory).
-constexpr int kSB = 32;
-__global__ void __launch_bounds__(256) simt_gemm_f32_kernel(const __grid_constant__ SimtParams p) {
-  __shared__ float xs[kSB][kSB + 1];  // [k][m]
-  __shared__ float ws[kSB][kSB + 1];  // [k][n]
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const int m0 = blockIdx.y * kSB, n0 = blockIdx.x * kSB;
-  float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
-  for (int k0 = 0; k0 < p.K; k0 += kSB) {
-    for (int i = threadIdx.x; i < kSB * kSB; i += 256) {
-      const int r = i / kSB, c = i % kSB;  // c runs along K: coalesced
-      const int gm = m0 + r, gn = n0 + r, gk = k0 + c;
-      xs[c][r] = (gm < p.M && gk < p.K) ? p.X[static_cast<int64_t>(gm) * p.ldx + gk] : 0.f;
-      ws[c][r] = (gn < p.N && gk < p.K) ? p.W[static_cast<int64_t>(gn) * p.ldw + gk] : 0.f;
+// 16 x 16 output tile per 256-thread block; the four warp pairs take a quarter
+// of each 128-wide K chunk each (2 x 2 outputs per thread), and the quarters
+// are added in a fixed order at the end.  Chunks are double-buffered: the next
+// chunk's loads are in flight while the current one is multiplied, so a small
+// problem (the launch-bound sizes this path serves) pays about one memory round
+// trip instead of one per chunk, and 16 x 16 tiles give many blocks.
+constexpr int kFT = 16;    // output tile edge
+constexpr int kFK = 128;   // K chunk
+constexpr int kFPad = 129; // shared row stride (floats): distinct banks per row
+__device__ __forceinline__ void f32_chunk_load(const float* __restrict__ src, int64_t ld, int32_t rows, int32_t r0,
+                                               int32_t K, int32_t k0, bool vec, int t, float (&r)[8]) {
+  // 16 rows x 128 columns = 512 groups of 4 columns; thread t takes groups t, t + 256
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int gi = t + 256 * h;
+    const int row = gi >> 5, kq = (gi & 31) * 4;
+    const int32_t gr = r0 + row, gk = k0 + kq;
+    const float* q = src + static_cast<int64_t>(gr) * ld + gk;
+    if (gr < rows && vec && gk + 3 < K) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(q));
+      r[4 * h] = v.x;
+      r[4 * h + 1] = v.y;
+      r[4 * h + 2] = v.z;
+      r[4 * h + 3] = v.w;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) r[4 * h + j] = (gr < rows && gk + j < K) ? __ldg(q + j) : 0.0f;
     }
-    __syncthreads();
+  }
+}
+__device__ __forceinline__ void f32_chunk_store(float (*dst)[kFPad], int t, const float (&r)[8]) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int gi = t + 256 * h;
+    const int row = gi >> 5, kq = (gi & 31) * 4;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) dst[row][kq + j] = r[4 * h + j];
+  }
+}
+
+__global__ void __launch_bounds__(256) simt_gemm_f32_kernel(const __grid_constant__ SimtParams p) {
+  __shared__ float xs[2][kFT][kFPad];
+  __shared__ float ws[2][kFT][kFPad];
+  const int t = threadIdx.x;
+  const int kq = t >> 6;            // K quarter of each chunk
+  const int o = t & 63;
+  const int om = (o >> 3) * 2, on = (o & 7) * 2;
+  const int32_t m0 = blockIdx.y * kFT, n0 = blockIdx.x * kFT;
+  const bool xvec = (reinterpret_cast<uintptr_t>(p.X) & 15) == 0 && (p.ldx & 3) == 0;
+  const bool wvec = (reinterpret_cast<uintptr_t>(p.W) & 15) == 0 && (p.ldw & 3) == 0;
+  const int nchunks = (p.K + kFK - 1) / kFK;
+  float rx[8], rw[8];
+  f32_chunk_load(p.X, p.ldx, p.M, m0, p.K, 0, xvec, t, rx);
+  f32_chunk_load(p.W, p.ldw, p.N, n0, p.K, 0, wvec, t, rw);
+  f32_chunk_store(xs[0], t, rx);
+  f32_chunk_store(ws[0], t, rw);
+  __syncthreads();
+  float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+  for (int c = 0; c < nchunks; ++c) {
+    const int b = c & 1;
+    const bool more = c + 1 < nchunks;
+    if (more) {  // next chunk in flight during this one's products
+      f32_chunk_load(p.X, p.ldx, p.M, m0, p.K, (c + 1) * kFK, xvec, t, rx);
+      f32_chunk_load(p.W, p.ldw, p.N, n0, p.K, (c + 1) * kFK, wvec, t, rw);
+    }
 #pragma unroll 8
-    for (int k = 0; k < kSB; ++k) {
-      const float a0 = xs[k][ty * 2], a1 = xs[k][ty * 2 + 1];
-      const float b0 = ws[k][tx * 2], b1 = ws[k][tx * 2 + 1];
+    for (int k = kq * 32; k < kq * 32 + 32; ++k) {
+      const float a0 = xs[b][om][k], a1 = xs[b][om + 1][k];
+      const float b0 = ws[b][on][k], b1 = ws[b][on + 1][k];
       acc[0][0] = fmaf(a0, b0, acc[0][0]);
       acc[0][1] = fmaf(a0, b1, acc[0][1]);
       acc[1][0] = fmaf(a1, b0, acc[1][0]);
       acc[1][1] = fmaf(a1, b1, acc[1][1]);
     }
+    if (more) {
+      f32_chunk_store(xs[b ^ 1], t, rx);
+      f32_chunk_store(ws[b ^ 1], t, rw);
+    }
     __syncthreads();
   }
+  // the four quarters' partial sums, added in quarter order by quarter 0
+  float* red = &xs[0][0][0];  // [4][16 x 16] after the last chunk
 #pragma unroll
   for (int i = 0; i < 2; ++i)
 #pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const int gm = m0 + ty * 2 + i, gn = n0 + tx * 2 + j;
-      if (gm < p.M && gn < p.N)
-        p.Y[static_cast<int64_t>(gm) * p.ldy + gn] = apply_chain1(p.ops, p.n_ops, acc[i][j], gm, gn);
-    }
+    for (int j = 0; j < 2; ++j) red[kq * 256 + (om + i) * kFT + on + j] = acc[i][j];
+  __syncthreads();
+  if (kq == 0) {
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int e = (om + i) * kFT + on + j;
+        const float v = ((red[e] + red[256 + e]) + red[512 + e]) + red[768 + e];
+        const int32_t gm = m0 + om + i, gn = n0 + on + j;
+        if (gm < p.M && gn < p.N) p.Y[static_cast<int64_t>(gm) * p.ldy + gn] = apply_chain1(p.ops, p.n_ops, v, gm, gn);
+      }
+  }
 }
 
 cudaError_t simt_gemm_f32_launch(const SimtParams& p, cudaStream_t s) {
-  dim3 grid((p.N + kSB - 1) / kSB, (p.M + kSB - 1) / kSB);
+  dim3 grid((p.N + kFT - 1) / kFT, (p.M + kFT - 1) / kFT);
   simt_gemm_f32_kernel<<<grid, 256, 0, s>>>(p);
   return cudaGetLastError();
 }

@@ -73,29 +73,59 @@ def test_grouped_wait_timeout_is_reported():
 def test_error_words_are_per_workspace():
     """Two streams, two workspaces: the call whose waits are limited to 1 ns
     reports the timeout in its own workspace's error word; the other call's
-    word stays clean (the device-wide word sees the timeout as well)."""
-    inp = kf_workloads.generate("bf16_scale_rowlse", seed=23, M=512, N=2048, K=2048)
-    X, W = inp["X"].to(DEV), inp["W"].to(DEV)
-    chain = [("scale", {"scalar": 0.125}), ("row_logsumexp", {})]
-    need = kf.lib().kf_fused_gemm_workspace(512, 2048, 2048, ctypes.byref(kf.make_epilogue(chain, [])))
-    wa, wb = kf.new_workspace(need, DEV), kf.new_workspace(need, DEV)
+    word stays clean (the device-wide word sees the timeout as well).  A store
+    chain needs no scratch, so each call is given a header-only workspace for
+    its error word (the same problem as the timeout test above)."""
+    inp, d = _problem()
+    chain = chain_to(wl_chain("bf16_gelu_scale_residual", inp), DEV)
+    wa = kf.new_workspace(kf.KF_WORKSPACE_HEADER_BYTES, DEV)
+    wb = kf.new_workspace(kf.KF_WORKSPACE_HEADER_BYTES, DEV)
     sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
     torch.cuda.synchronize()
     assert kf.get_device_error()[0] == kf.KF_OK
     try:
         kf.set_wait_timeout_ns(1)
-        kf.fused_gemm(X, W, chain, workspace=wa, stream=sa)
+        kf.fused_gemm(d["X"], d["W"], chain, workspace=wa, stream=sa)
     finally:
         kf.set_wait_timeout_ns(0)
-    yb = kf.fused_gemm(X, W, chain, workspace=wb, stream=sb)
+    yb = kf.fused_gemm(d["X"], d["W"], chain, workspace=wb, stream=sb)
+    stb, rawb = kf.check_device_error(wb, sb)
+    sta, rawa = kf.check_device_error(wa, sa)
+    assert stb == kf.KF_OK, ("other stream", stb, hex(rawb))
+    assert sta == kf.KF_ERR_DEVICE_TIMEOUT and rawa & 0x7, ("timed-out stream", sta, hex(rawa))
+    assert kf.check_device_error(wa, sa)[0] == kf.KF_OK  # cleared by the read
+    dst, draw = kf.get_device_error()
+    assert dst == kf.KF_ERR_DEVICE_TIMEOUT, ("device word", dst, hex(draw))
+    assert kf.get_device_error()[0] == kf.KF_OK
+    torch.cuda.synchronize()
+    check_bf16(yb, oracle.fused_gemm(inp["X"], inp["W"], wl_chain("bf16_gelu_scale_residual", inp)),
+               "the other stream's call")
+
+
+def test_bounds_errors_are_per_workspace():
+    """The same isolation with a deterministic error: a gathered grouped GEMM
+    whose row index points outside A sets the bounds bit in its own
+    workspace's word only; a correct call on another stream reports KF_OK."""
+    g = torch.Generator().manual_seed(4)
+    A = torch.randn(64, 128, generator=g).to(torch.bfloat16).to(DEV)
+    B = (torch.randn(2, 256, 128, generator=g) * 0.1).to(torch.bfloat16).to(DEV)
+    off = torch.tensor([0, 40, 96], dtype=torch.int32, device=DEV)
+    good = torch.randint(0, 64, (96,), generator=g, dtype=torch.int32)
+    bad = good.clone()
+    bad[17] = 1 << 20
+    need = kf.lib().kf_grouped_gemm_workspace(96, 256, 128, 2, 1, None)
+    wa, wb = kf.new_workspace(need, DEV), kf.new_workspace(need, DEV)
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    gi, bi = good.to(DEV), bad.to(DEV)
+    torch.cuda.synchronize()
+    kf.get_device_error()
+    kf.grouped_gemm(A, B, off, 256, [], row_index=bi, workspace=wa, stream=sa)
+    C = kf.grouped_gemm(A, B, off, 256, [], row_index=gi, workspace=wb, stream=sb)
     stb, rawb = kf.check_device_error(wb, sb)
     sta, rawa = kf.check_device_error(wa, sa)
     assert stb == kf.KF_OK, hex(rawb)
-    assert sta == kf.KF_ERR_DEVICE_TIMEOUT and rawa & 0x7, (sta, hex(rawa))
-    assert kf.check_device_error(wa, sa)[0] == kf.KF_OK  # cleared by the read
-    assert kf.get_device_error()[0] == kf.KF_ERR_DEVICE_TIMEOUT
-    assert kf.get_device_error()[0] == kf.KF_OK
+    assert sta == kf.KF_ERR_DEVICE_BOUNDS and rawa == 0x8, (sta, hex(rawa))
+    assert kf.get_device_error()[0] == kf.KF_ERR_DEVICE_BOUNDS
     torch.cuda.synchronize()
-    ref = oracle.fused_gemm(inp["X"], inp["W"], chain)[:, 0]
-    from tests._util import check_f32
-    check_f32(yb, ref, "the other stream's call")
+    ref = oracle.grouped_gemm(A.cpu(), B.cpu(), off.cpu().numpy(), 256, [], row_index=good.numpy())
+    check_bf16(C, ref, "the other stream's grouped call")
