@@ -48,23 +48,24 @@ def _peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
 
 
-KERNEL_FILES = ("kf_ptx.cuh", "kf_common.cuh", "kf_tc_gemm.cuh", "kf_internal.h", "kf_tc_dense.cu", "kf_tc_dense2.cu")
-
-
 def kernel_source_hash() -> str:
-    """Hash of the sources of the dense tensor-core kernel; a stored ncu traffic
-    figure is used only while they are unchanged since it was captured."""
+    """Hash of the library's sources (every file under csrc/ and the C header); a
+    stored ncu traffic figure is used only while they are unchanged since it was
+    captured."""
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2606_02963_gb300", "csrc")
-    for fn in KERNEL_FILES:
-        h.update(fn.encode())
-        h.update(open(os.path.join(d, fn), "rb").read())
+    files = sorted(os.path.join(d, fn) for fn in os.listdir(d) if fn.endswith((".cu", ".cuh", ".h")))
+    files.append(os.path.join(ROOT, "include", "kf.h"))
+    for fp in files:
+        h.update(os.path.basename(fp).encode())
+        h.update(open(fp, "rb").read())
     return h.hexdigest()[:16]
 
 
 def stored_traffic(kernel_tag: str):
-    """Per-launch DRAM bytes from profiles/ncu_traffic.txt (lines:
-    '<tag> <source-hash> <bytes>'), or None if absent or stale."""
+    """Per-step DRAM bytes (read + write, all of the path's kernels of one step)
+    from profiles/ncu_traffic.txt (lines: '<tag> <source-hash> <bytes>'), or None
+    if absent or stale."""
     p = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     if not os.path.exists(p):
         return None
@@ -242,14 +243,18 @@ def dense_setup(name, dev):
 
 
 def dense_bytes(name, wl):
+    """Algorithmic bytes of one call: every input read once, the output written once."""
     M, N, K = wl.M, wl.N, wl.K
-    b = 2 * (M * K + N * K)
+    e = 4 if wl.dtype == "f32" else 2
+    b = e * (M * K + N * K)
     if name == MAIN:
-        b += 2 * N + 2 * M * N + 2 * M * N          # bias, R, Y
+        b += e * (N + M * N + M * N)                # bias, R, Y
     elif name == "bf16_scale_rowlse":
-        b += 4 * M
+        b += 4 * M                                  # fp32 [M]
     elif name == "bf16_groupnorm_swish":
-        b += 2 * N + 4 * N * 2 + 2 * M * N          # bias, gamma/beta (fp32), Y
+        b += e * (3 * N + M * N)                    # bias, gamma, beta, Y
+    elif name == "fp32_relu_linear":
+        b += e * (N + M * N)                        # bias, Y
     return b
 
 
@@ -340,7 +345,7 @@ def run_kf(args, rank, world, dev):
     ms_cublas, _ = time_steps_rotating([(lambda c=c: torch.matmul(c["X"], c["W"].t())) for c in copies],
                                        args.steps, args.warmup, stream)
     del copies, outs, chains, rot
-    traffic = stored_traffic("dense_store_gelu_1024x4096x4096")
+    traffic = stored_traffic(MAIN)
     achieved = flops / (ms * 1e-3) / 1e12
     line = {
         "metric": "fused GEMM+tail TFLOP/s & % of GB300 roofline; speedup vs unfused torch eager",
@@ -446,9 +451,6 @@ def roofline_block(flops, byts, ms, peaks, traffic=None):
             "unit": "GB/s", "frac": round(ach / peaks["hbm"], 4), "traffic": traffic, "algorithmic_bytes": byts}
 
 
-DENSE_TRAFFIC_TAGS = {"bf16_scale_rowlse": "dense_lse_2048x8192x8192"}
-
-
 def dense_config_block(name, args, kf, dev, flush, stream, peaks, steps):
     """One dense configuration with its full record: isolated device time, the
     roofline of its kernel, unfused eager and bare-GEMM baselines, the end-to-end
@@ -489,7 +491,7 @@ def dense_config_block(name, args, kf, dev, flush, stream, peaks, steps):
     byts = dense_bytes(name, wl)
     rec = {"workload": name, "M": M, "N": N, "K": K, "ms": round(ms, 5),
            "tflops": round(flops / ms / 1e9, 3),
-           "roofline": roofline_block(flops, byts, ms, peaks, stored_traffic(DENSE_TRAFFIC_TAGS.get(name, ""))),
+           "roofline": roofline_block(flops, byts, ms, peaks, stored_traffic(name)),
            "eager_ms": round(ms_e, 5), "speedup_vs_eager": round(ms_e / ms, 3),
            "gemm_only_ms": round(ms_c, 5),
            "e2e": {"value": round(flops / ms_e2e / 1e9, 3), "unit": "TFLOP/s", "ms_per_step": round(ms_e2e, 4),
