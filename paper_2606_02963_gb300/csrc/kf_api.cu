@@ -1157,10 +1157,12 @@ namespace {
 // Tile width of the QKV projection: whole heads per tile (a multiple of d),
 // then the fewest tile-widths on the busiest SM (or CTA pair) + a fixed cost
 // per tile, as for the dense store variants.
-// Calls of at most this many tokens take the cluster-split decode kernel; above
-// it the per-token reduction costs more than the whole-tile kernel's MMAs
-// (gpt-oss-20b shape: 48 tokens 20.5 against 22.5 us, 64 tokens 24.6 against 22.5)
-constexpr int64_t kQkvClusterMaxT = 48;
+// Calls of at most this many tokens (the decode kernel's largest token box) take
+// the cluster-split decode kernel; with both kernels launched as programmatic
+// dependents that prefetch their weights, it is the faster one up to there
+// (gpt-oss-20b shape, back to back: 56 tokens 17.0 against 18.8 us, 64 tokens
+// 17.1 against 19.0 us)
+constexpr int64_t kQkvClusterMaxT = 64;
 static_assert(kQkvClusterMaxT <= kQkvDecodeMaxRows, "the decode kernel's token box");
 
 int pick_rope_bn(int64_t M, int64_t N, int d, int nsm, bool cta2) {

@@ -231,6 +231,17 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
     if constexpr (RT) tma_prefetch_desc(&tmR);
+    if constexpr (MODE == kModeRope) {
+      // the QKV projection at decode sizes streams its weights: this CTA's first
+      // weight tile goes to L2 while a preceding kernel may still run (a
+      // prefetch reads memory without changing it, and L2 is where that
+      // kernel's writes land, so the loads after the dependency wait below see
+      // current values either way)
+      if (p.M <= kBM && unit0 < p.total_units) {
+        const int32_t nb0 = (unit0 / p.tiles_m) * Cfg::kOutN + static_cast<int32_t>(prank) * Cfg::kBRows;
+        for (int32_t kb = 0; kb < p.num_kb; ++kb) tma_prefetch_3d(&tmB, kb * kBK, nb0, 0);
+      }
+    }
   }
   if (warp == 1) {
     __syncwarp();

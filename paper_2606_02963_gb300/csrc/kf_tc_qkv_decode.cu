@@ -163,12 +163,21 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    // this CTA's weights into L2 while a preceding kernel may still run: a
+    // prefetch reads memory without changing it and L2 is where that kernel's
+    // writes land, so the loads after the dependency wait below see current
+    // values either way; the weights are the bytes this kernel is bound by
+    for (int32_t kb = kb0; kb < kb1; ++kb) tma_prefetch_3d(&tmB, kb * kDcBK, n0, 0);
   }
   if (warp == 1) {
     __syncwarp();
     tmem_alloc(tmem_slot, kDcBN);
     tmem_relinquish();
   }
+  // launched as a programmatic dependent of the previous kernel in the stream:
+  // wait for it before any operand, position or table is read
+  griddep_wait();
+  griddep_launch_dependents();
   tc_fence_before();
   __syncwarp();
   __syncthreads();
@@ -358,13 +367,17 @@ cudaError_t launch_dc(const CUtensorMap& a, const CUtensorMap& b, const QkvDecod
   cfg.blockDim = dim3(kDcThreads, 1, 1);
   cfg.dynamicSmemBytes = Cfg::kSmemBytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = p.splits;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // a programmatic dependent of the previous kernel in the stream (the kernel
+  // waits for it before reading anything it may have written)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, a, b, p);
 }
 

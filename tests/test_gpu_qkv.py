@@ -51,10 +51,10 @@ def _check(got, ref, idx, what, out_dtype=torch.bfloat16, all_tokens=True):
             assert bool((kc[o] == SENT).all()) and bool((vc[o] == SENT).all()), f"{what}: unnamed rows written"
 
 
-@pytest.mark.parametrize("T", [1, 16, 32, 33, 48, 49, 64, 128])
+@pytest.mark.parametrize("T", [1, 16, 32, 33, 48, 49, 64, 65, 128])
 def test_decode_gpt_oss_shape(T):
-    # <= 48 tokens: clusters splitting K (32-row token boxes up to 32 tokens,
-    # 64-row ones above); 49..128: one 128-row tile per CTA
+    # <= 64 tokens: clusters splitting K (32-row token boxes up to 32 tokens,
+    # 64-row ones above); 65..128: one 128-row tile per CTA
     s = kf_workloads.QKV_SHAPE
     inp = kf_workloads.qkv_generate(T, seed=60 + T)
     got, ref, idx = _run(inp, s["nq"], s["nkv"], s["d"])
