@@ -100,7 +100,8 @@ struct TcCfg {
   // per-warp 1 KB tile buffers (1 KB aligned, right after the stages): two for
   // the asynchronous TMA stores, plus (store mode) one for the residual
   // transposition, which must not reuse a buffer a TMA store may still read
-  // (residual tile: 256 B per warp, the bias of its chunks)
+  // (residual tile: 256 B per warp, the bias of its chunks; scatter-add: 64 B
+  // per lane, the row segment a bulk reduction adds to the destination row)
   static constexpr int kWarpStaging = RT ? 256 : (MODE == kModeStore) ? 3072 : (MODE == kModeRope) ? 0 : 2048;
   // residual tile: BN / 32 chunks x 4 row blocks of 32 x 32 bf16 (2 KB, 64-byte
   // swizzle), placed in the A then B regions of two ring slots
@@ -736,18 +737,29 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
           if constexpr (RT) {
             // stored above
           } else if constexpr (MODE == kModeScatter) {
-            if (wr) {
-              float* dstp = reinterpret_cast<float*>(p.C) + static_cast<int64_t>(dst) * p.ldc + col0;
-              if (nvalid == 32 && p.c_vec_ok) {
+            float* dstp = reinterpret_cast<float*>(p.C) + static_cast<int64_t>(dst) * p.ldc + col0;
+            if (nvalid == 32 && p.c_vec_ok) {
+              // row = lane: the scaled row segment passes through this lane's
+              // 64 bytes of the warp buffer, 16 columns at a time, and the TMA
+              // unit adds it to the destination row
+              float4* sb = reinterpret_cast<float4*>(stage) + lane * 4;
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                  atomicAdd(reinterpret_cast<float4*>(dstp) + j,
-                            make_float4(v[4 * j] * rs, v[4 * j + 1] * rs, v[4 * j + 2] * rs, v[4 * j + 3] * rs));
-              } else {
+              for (int hf = 0; hf < 2; ++hf) {
+                bulk_wait_group_read<0>();  // this lane's previous segment has been read
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  if (j < nvalid) atomicAdd(dstp + j, v[j] * rs);
+                for (int u = 0; u < 4; ++u)
+                  sb[u] = make_float4(v[16 * hf + 4 * u] * rs, v[16 * hf + 4 * u + 1] * rs,
+                                      v[16 * hf + 4 * u + 2] * rs, v[16 * hf + 4 * u + 3] * rs);
+                fence_proxy_async_smem();
+                if (wr) {
+                  bulk_reduce_add_f32(dstp + 16 * hf, sb, 64);
+                  bulk_commit_group();
+                }
               }
+            } else if (wr) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (j < nvalid) atomicAdd(dstp + j, v[j] * rs);
             }
           } else if (c_tma) {
             store_tile32_tma(stage, lane, v, &tmC, col0, wrow0);
@@ -1197,7 +1209,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
   }
 
   // ---------------------------------------------------------------- teardown
-  if (warp >= 2 && lane == 0) bulk_wait_group_all();  // this warp's TMA stores have completed
+  if (warp >= 2 && (lane == 0 || MODE == kModeScatter)) bulk_wait_group_all();  // this warp's bulk copies have completed
   tc_fence_before();
   __syncwarp();  // lane 0 of the producer / MMA warps arrives after lanes 1-31
   __syncthreads();
