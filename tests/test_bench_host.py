@@ -2,6 +2,7 @@
 nvidia-smi samples (median SM clock, throttle reasons), the traffic figure keyed
 to the kernel sources' hash, and the whole-job throughput."""
 import os
+import shutil
 
 import pytest
 
@@ -50,11 +51,25 @@ def test_stored_traffic_is_keyed_to_the_kernel_sources(tmp_path, monkeypatch):
     assert bench.stored_traffic("dense_store_x") is None  # stale once the sources change
 
 
-def test_kernel_source_hash_covers_the_dense_kernel_files():
-    d = os.path.join(bench.ROOT, "paper_2606_02963_gb300", "csrc")
-    assert all(os.path.exists(os.path.join(d, f)) for f in bench.KERNEL_FILES)
+def test_kernel_source_hash_covers_every_library_source(tmp_path, monkeypatch):
+    # a stored ncu traffic figure stays valid only while no source of the
+    # library changed: the hash covers every file under csrc/ and the C header
     h = bench.kernel_source_hash()
     assert len(h) == 16 and h == bench.kernel_source_hash()
+    src = os.path.join(bench.ROOT, "paper_2606_02963_gb300", "csrc")
+    dst = tmp_path / "paper_2606_02963_gb300" / "csrc"
+    shutil.copytree(src, dst, ignore=shutil.ignore_patterns("*.o", "*.so"))
+    (tmp_path / "include").mkdir()
+    shutil.copy(os.path.join(bench.ROOT, "include", "kf.h"), tmp_path / "include" / "kf.h")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.kernel_source_hash() == h
+    for f in sorted(os.listdir(dst)) + ["../../include/kf.h"]:
+        fp = dst / f
+        old = fp.read_bytes()
+        fp.write_bytes(old + b"\n")
+        assert bench.kernel_source_hash() != h, f
+        fp.write_bytes(old)
+    assert bench.kernel_source_hash() == h
 
 
 def test_whole_job_throughput_and_single_rank_max():
