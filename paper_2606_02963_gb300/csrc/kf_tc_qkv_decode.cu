@@ -289,10 +289,23 @@ __global__ void __launch_bounds__(kDcThreads, 1)
           if (batch[j].ok && m < npl) {
             const int i = lane + 32 * m;
             const uint32_t off = static_cast<uint32_t>((batch[j].t * kDcPartStride + (batch[j].hcol - n0) + i) * 4);
-            for (uint32_t s2 = 0; s2 < S; ++s2) {
-              const uint32_t bs = mapa_shared(part_base, s2);
-              a[j][m] += ld_cluster_f32(bs + off);
-              b[j][m] += ld_cluster_f32(bs + off + static_cast<uint32_t>(half * 4));
+            // all 2S loads in flight before the first add (their round trips
+            // overlap), then the sums in CTA-rank order
+            float va[8], vb[8];
+#pragma unroll
+            for (uint32_t s2 = 0; s2 < 8; ++s2) {
+              if (s2 < S) {
+                const uint32_t bs = mapa_shared(part_base, s2);
+                va[s2] = ld_cluster_f32(bs + off);
+                vb[s2] = ld_cluster_f32(bs + off + static_cast<uint32_t>(half * 4));
+              }
+            }
+#pragma unroll
+            for (uint32_t s2 = 0; s2 < 8; ++s2) {
+              if (s2 < S) {
+                a[j][m] += va[s2];
+                b[j][m] += vb[s2];
+              }
             }
           }
         }
