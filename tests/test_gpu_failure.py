@@ -129,3 +129,41 @@ def test_bounds_errors_are_per_workspace():
     torch.cuda.synchronize()
     ref = oracle.grouped_gemm(A.cpu(), B.cpu(), off.cpu().numpy(), 256, [], row_index=good.numpy())
     check_bf16(C, ref, "the other stream's grouped call")
+
+
+@pytest.mark.parametrize("T", [1, 32])  # the weight stream (<= 8 tokens) and the K-splitting clusters
+def test_qkv_decode_wait_timeout_is_reported_and_context_survives(T):
+    s = kf_workloads.QKV_SHAPE
+    inp = kf_workloads.qkv_generate(T, seed=400 + T, cache_rows=512)
+    g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
+    rows = int(inp["rows"])
+
+    def run():
+        kc = torch.zeros(rows, s["nkv"] * s["d"], dtype=torch.bfloat16, device=DEV)
+        vc = torch.zeros_like(kc)
+        q = kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"], s["nq"],
+                           s["nkv"], s["d"], kc, vc)
+        return q, kc, vc
+
+    assert kf.get_device_error()[0] == kf.KF_OK
+    try:
+        kf.set_wait_timeout_ns(1)
+        run()
+        st, raw = kf.get_device_error()
+    finally:
+        kf.set_wait_timeout_ns(0)
+    if T > 8:
+        # the epilogue warps wait for the accumulator through the whole mainloop
+        assert st == kf.KF_ERR_DEVICE_TIMEOUT, (st, hex(raw))
+    else:
+        # the stream's waits are for stages that land within microseconds; a
+        # blocking try-wait may see them land before the first check of the
+        # limit, so the call may also complete normally
+        assert st in (kf.KF_ERR_DEVICE_TIMEOUT, kf.KF_OK), (st, hex(raw))
+    q, kc, vc = run()
+    assert kf.get_device_error()[0] == kf.KF_OK
+    rq, rk, rv = oracle.qkv_rope_kv(inp["X"], inp["W"], inp["b"], inp["positions"], inp["cache_rows"], inp["cos"],
+                                    inp["sin"], s["nq"], s["nkv"], s["d"], rows)
+    check_bf16(q, rq, f"qkv after timeout T={T}")
+    named = np.flatnonzero(~np.isnan(rk[:, 0]))
+    check_bf16(kc[torch.as_tensor(named, device=DEV)], rk[named], f"k after timeout T={T}")
