@@ -458,6 +458,8 @@ struct GroupExtras {
   int64_t gbias_ld = 0;
   bool sw_ext = false;
   float sw_alpha = 1.0f, sw_limit = 0.0f, sw_c = 0.0f;
+  void* zero_ptr = nullptr;  // SwiGLU: cleared while its first units run (see TcParams)
+  int64_t zero_bytes = 0;
 };
 
 // `pdl`: the previous kernel in the stream is one of this library's (MoE chain),
@@ -509,6 +511,8 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, uint
     p.sw_alpha = ex->sw_alpha;
     p.sw_limit = ex->sw_limit;
     p.sw_c = ex->sw_c;
+    p.zero_ptr = ex->zero_ptr;
+    p.zero_bytes = ex->zero_bytes;
   }
   const int64_t ub = ((g.rows_total + kBM - 1) / kBM + g.G) * p.tiles_n;
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(ub, di.nsm)));
@@ -964,9 +968,10 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
   const int64_t P = T * k;
 
   int32_t* pos = det ? reinterpret_cast<int32_t*>(ws + L.pos) : nullptr;
-  // the fp32 scatter target is cleared first, so that the kernels of the chain
-  // below follow one another directly (each a programmatic dependent of the last)
-  if (!det && cudaMemsetAsync(yacc, 0, static_cast<size_t>(T) * H * 4, s) != cudaSuccess) return KF_ERR_CUDA;
+  // the fp32 scatter target is cleared by the gate/up GEMM's epilogue warps
+  // while its first units run (the down GEMM starts after that grid completes),
+  // so no separate pass over it and the kernels of the chain follow one another
+  // directly (each a programmatic dependent of the last)
   st = cuda_status(route_topk_launch(logits, static_cast<int32_t>(T), E, k, ids, w, s));
   if (st != KF_OK) return st;
   if (P >= kSortMultiBlockPairs)
@@ -985,6 +990,10 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     if (st != KF_OK) return st;
     GroupedArgs g{X, H, T, stok, W_gu, H, 2 * I * H, off, E, P, I, H, h, KF_BF16, I};
     GroupExtras ex;
+    if (!det) {
+      ex.zero_ptr = yacc;
+      ex.zero_bytes = T * H * 4;
+    }
     if (act) {
       ex.gbias = act->b_gu;
       ex.gbias_ld = 2 * I;

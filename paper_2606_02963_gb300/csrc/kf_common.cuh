@@ -127,6 +127,12 @@ struct TcParams {
   float sw_alpha;
   float sw_limit;
   float sw_c;
+  // grouped SwiGLU (the MoE gate/up GEMM): zero_bytes (a multiple of 16) at
+  // zero_ptr are cleared by the epilogue warps while the first unit's mainloop
+  // runs -- the down GEMM's fp32 scatter target, which that GEMM only touches
+  // after this grid has completed
+  void* zero_ptr;
+  int64_t zero_bytes;
 };
 
 // ---------------------------------------------------------------- loads/stores

@@ -499,6 +499,16 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     const int q = warp & 3;
     const int h = ew >> 2;
     const int32_t row_in_tile = q * 32 + lane;
+    if constexpr (GROUPED && MODE == kModeSwiglu) {
+      if (p.zero_ptr) {
+        // this CTA's share of the scatter target, 16 bytes per thread and step
+        const int64_t n16 = p.zero_bytes >> 4;
+        const int64_t per = (n16 + gridDim.x - 1) / gridDim.x;
+        const int64_t z0 = static_cast<int64_t>(blockIdx.x) * per, z1 = min(n16, z0 + per);
+        uint4* zp = static_cast<uint4*>(p.zero_ptr);
+        for (int64_t i = z0 + ew * 32 + lane; i < z1; i += 32 * Cfg::kEpiW) zp[i] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const bool fast = p.fast != 0;
     float2* xch = reinterpret_cast<float2*>(misc + 16);  // [2 halves][128 rows]
