@@ -10,15 +10,15 @@
 // 64-column heads): CTA r multiplies the k-blocks [r K / S, (r + 1) K / S),
 // writes the T token rows of its 128 x 256 fp32 partial from TMEM into its own
 // shared memory (the operand ring, free by then), and after a cluster barrier the epilogue warps
-// of all S CTAs take the tile's (token, head) items in turn: a warp sums the S
-// partials of its item (lane j: columns j and j + d/2 of the head, read from
-// each CTA's shared memory through DSMEM), adds the bias, rotates query and key
-// heads and stores the row to q_out or to the token's cache row.  No global
-// workspace, no atomics, no waits between CTAs other than the two hardware
-// cluster barriers.  While the MMAs run, the epilogue warps already load what
-// their first items need besides the sums (positions, cache rows, bias, the
-// table rows of the positions), so that after the barrier only the partial sums
-// are read.
+// of all S CTAs take the tile's token rows in turn: a warp sums the S partials
+// of its row (lane j: the four rotation pairs 4j .. 4j + 3 of the tile, read as
+// 16-byte loads from each CTA's shared memory through DSMEM), adds the bias,
+// rotates query and key heads and stores the row's heads to q_out or to the
+// token's cache row.  No global workspace, no atomics, no waits between CTAs
+// other than the two hardware cluster barriers.  While the MMAs run, the
+// epilogue warps already load what their rows need besides the sums (bias,
+// positions, cache rows, the first row's table entries), so that after the
+// barrier mostly the partial sums are read.
 //
 // Token rows are staged in boxes of ROWS = 32 (six-stage ring) or 64 rows
 // (five stages): the box is what limits the tokens of a call.
@@ -33,7 +33,7 @@ constexpr int kDcThreads = 320;
 constexpr int kDcBM = 128;          // rows of the MMA (only the first T are tokens)
 constexpr int kDcBK = 64;           // K elements per 128-byte row
 constexpr int kDcBN = 256;          // tile columns
-constexpr int kDcPartStride = 257;  // floats per partial row (odd: conflict-free row-per-lane stores)
+constexpr int kDcPartStride = 260;  // floats per partial row (4 banks apart: conflict-free 16-byte row-per-lane stores)
 
 template <int ROWS, int STAGES>
 struct DcCfg {
@@ -56,51 +56,105 @@ struct DcCfg {
   static_assert(kSmemBytes <= 232448, "shared memory");
 };
 
-__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+__device__ __forceinline__ float4 ld_cluster_f32x4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
   return v;
 }
 
-// Operands of one (token, head) item that do not depend on the sums: lane j
-// holds pairs j + 32 m of the head (d / 2 <= 128: m < 4).
-constexpr int kBatch = 4, kMaxPl = 4;
-struct DcItem {
-  int32_t t, hcol, pos, crow;
-  bool live, ok, rotate;
-  float b0[kMaxPl], b1[kMaxPl], c[kMaxPl], s[kMaxPl];
+// A tile row (one token, 256 columns) is reduced by one warp: lane j takes the
+// rotation pairs 4j .. 4j + 3 of the tile, i.e. four consecutive columns of one
+// head's first half and the four that pair with them in its second half (a
+// head's half is a multiple of 32 columns, so the four never straddle heads).
+// These operands of the lane do not depend on the token.
+struct DcLane {
+  int32_t hcol;  // first column of the lane's head
+  int32_t i;     // first of the lane's four pair indices within the head
+  bool live, rotate;
+  float b0[4], b1[4];
+};
+// The token-dependent operands of a row.
+struct DcRow {
+  int32_t pos, crow;
+  bool ok;
+  float c[4], s[4];
 };
 
-// Items it = base + stride j (j < kBatch) of a tile: token it / heads, head
-// it % heads.  All loads are issued before any is used.  A position or cache row
-// out of range clears `ok` (the item is then reported and skipped, and no table
-// row is read for it).
-__device__ __forceinline__ void dc_load_items(const QkvDecodeParams& p, int32_t n0, int32_t base, int32_t stride,
-                                              int32_t items, int heads, int lane, DcItem (&it)[kBatch]) {
-  const int d = p.rope_d, half = d >> 1, npl = half >> 5;
+__device__ __forceinline__ void dc_lane(const QkvDecodeParams& p, int32_t n0, int lane, DcLane& L) {
+  const int d = p.rope_d, half = d >> 1;
+  const int pr = 4 * lane;
+  L.hcol = n0 + (pr / half) * d;
+  L.i = pr % half;
+  L.live = L.hcol < p.N;
+  L.rotate = L.hcol < p.rot_cols;
 #pragma unroll
-  for (int j = 0; j < kBatch; ++j) {
-    const int32_t idx = base + stride * j;
-    const int32_t hl = idx % heads;
-    it[j].t = idx / heads;
-    it[j].hcol = n0 + hl * d;
-    it[j].live = idx < items && it[j].hcol < p.N;
-    it[j].pos = it[j].live ? p.positions[it[j].t] : 0;
-    it[j].crow = it[j].live ? p.cache_rows[it[j].t] : 0;
+  for (int m = 0; m < 4; ++m) {
+    const bool use = L.live && p.bias;
+    L.b0[m] = use ? ld_elem(p.bias, p.bias_dtype, L.hcol + L.i + m) : 0.0f;
+    L.b1[m] = use ? ld_elem(p.bias, p.bias_dtype, L.hcol + L.i + m + half) : 0.0f;
   }
-#pragma unroll
-  for (int j = 0; j < kBatch; ++j) {
-    it[j].ok = it[j].live && it[j].pos >= 0 && it[j].pos < p.max_pos && it[j].crow >= 0 && it[j].crow < p.rows;
-    it[j].rotate = it[j].hcol < p.rot_cols;
-#pragma unroll
-    for (int m = 0; m < kMaxPl; ++m) {
-      const int i = lane + 32 * m;
-      const bool use = it[j].ok && m < npl;
-      it[j].b0[m] = use && p.bias ? ld_elem(p.bias, p.bias_dtype, it[j].hcol + i) : 0.0f;
-      it[j].b1[m] = use && p.bias ? ld_elem(p.bias, p.bias_dtype, it[j].hcol + i + half) : 0.0f;
-      const bool tab = use && it[j].rotate;
-      it[j].c[m] = tab ? __ldg(p.cos_t + static_cast<int64_t>(it[j].pos) * half + i) : 1.0f;
-      it[j].s[m] = tab ? __ldg(p.sin_t + static_cast<int64_t>(it[j].pos) * half + i) : 0.0f;
+}
+
+// A position or cache row out of range clears `ok` (the row is then reported
+// and skipped, and no table row is read for it).
+__device__ __forceinline__ void dc_row(const QkvDecodeParams& p, const DcLane& L, int32_t pos, int32_t crow,
+                                       DcRow& R) {
+  const int half = p.rope_d >> 1;
+  R.pos = pos;
+  R.crow = crow;
+  R.ok = pos >= 0 && pos < p.max_pos && crow >= 0 && crow < p.rows;
+  // the tables start on 16 bytes and half and i are multiples of 4: one
+  // 16-byte load per table
+  float4 c = make_float4(1.0f, 1.0f, 1.0f, 1.0f), s = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  if (R.ok && L.live && L.rotate) {
+    const int64_t o = static_cast<int64_t>(pos) * half + L.i;
+    c = __ldg(reinterpret_cast<const float4*>(p.cos_t + o));
+    s = __ldg(reinterpret_cast<const float4*>(p.sin_t + o));
+  }
+  R.c[0] = c.x;
+  R.c[1] = c.y;
+  R.c[2] = c.z;
+  R.c[3] = c.w;
+  R.s[0] = s.x;
+  R.s[1] = s.y;
+  R.s[2] = s.z;
+  R.s[3] = s.w;
+}
+
+// four consecutive outputs from element o on: one vector store where o and the
+// base allow it, else four scalar stores
+__device__ __forceinline__ void dc_store4(void* dst, int dt, int64_t o, float x0, float x1, float x2, float x3) {
+  const uintptr_t base = reinterpret_cast<uintptr_t>(dst);
+  if (dt == KF_F32) {
+    float* d = reinterpret_cast<float*>(dst) + o;
+    if ((o & 3) == 0 && (base & 15) == 0) {
+      *reinterpret_cast<float4*>(d) = make_float4(x0, x1, x2, x3);
+    } else {
+      d[0] = x0;
+      d[1] = x1;
+      d[2] = x2;
+      d[3] = x3;
+    }
+  } else {
+    uint32_t w0, w1;
+    if (dt == KF_BF16) {
+      w0 = pack_bf16x2(x0, x1);
+      w1 = pack_bf16x2(x2, x3);
+    } else {
+      w0 = pack_f16x2(x0, x1);
+      w1 = pack_f16x2(x2, x3);
+    }
+    uint16_t* d = reinterpret_cast<uint16_t*>(dst) + o;
+    if ((o & 3) == 0 && (base & 7) == 0) {
+      *reinterpret_cast<uint2*>(d) = make_uint2(w0, w1);
+    } else {
+      d[0] = static_cast<uint16_t>(w0);
+      d[1] = static_cast<uint16_t>(w0 >> 16);
+      d[2] = static_cast<uint16_t>(w1);
+      d[3] = static_cast<uint16_t>(w1 >> 16);
     }
   }
 }
@@ -140,13 +194,14 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   const int32_t kb1 = static_cast<int32_t>(r + 1) * p.num_kb / static_cast<int32_t>(S);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // (token, head) items of the tile go to the cluster's epilogue warps in turn;
-  // a warp takes up to kBatch items at a time
-  const int heads = kDcBN / p.rope_d;
-  const int32_t items = p.T * heads;
+  // the tile's token rows go to the cluster's epilogue warps in turn: rows
+  // first, first + stride, ... of the call's T
   const int32_t stride = static_cast<int32_t>(S) * 8;
   const int32_t first = static_cast<int32_t>(r) + static_cast<int32_t>(S) * (warp - 2);
-  DcItem batch[kBatch];  // the epilogue warp's current items
+  const int32_t nrows = warp >= 2 && first < p.T ? (p.T - first + stride - 1) / stride : 0;
+  DcLane L;       // the epilogue lane's columns and bias
+  DcRow cur;      // the warp's current row
+  int32_t my_pos = 0, my_crow = 0;  // lane k < nrows: row k's position and cache row
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -240,8 +295,16 @@ __global__ void __launch_bounds__(kDcThreads, 1)
     const int q = warp & 3;                      // TMEM lane quadrant
     const int hh = ew >> 2;                      // column half: [128 hh, 128 hh + 128)
     const int32_t row = q * 32 + lane;
-    // the first batch's operands load while the MMAs run
-    if (first < items) dc_load_items(p, n0, first, stride, items, heads, lane, batch);
+    // while the MMAs run: the lane's bias, the positions and cache rows of all
+    // the warp's rows (at most 8: T <= 64 and stride >= 8), the first row's
+    // table entries
+    dc_lane(p, n0, lane, L);
+    if (lane < nrows) {
+      my_pos = p.positions[first + lane * stride];
+      my_crow = p.cache_rows[first + lane * stride];
+    }
+    if (nrows > 0)
+      dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, 0), __shfl_sync(0xffffffffu, my_crow, 0), cur);
     bool w = mbar_wait(accf, 0, abort_flag, p.wait_ns);
     w = __all_sync(0xffffffffu, w);
     if (!w) {
@@ -256,9 +319,9 @@ __global__ void __launch_bounds__(kDcThreads, 1)
           float v[32];
           tmem_ld32(tmem + lane_off + hh * 128 + c * 32, v);
           if (row < p.T) {
-            float* dst = part + row * kDcPartStride + hh * 128 + c * 32;
+            float4* dst = reinterpret_cast<float4*>(part + row * kDcPartStride + hh * 128 + c * 32);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) dst[j] = v[j];
+            for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
           }
         }
       }
@@ -272,84 +335,71 @@ __global__ void __launch_bounds__(kDcThreads, 1)
 
   if (warp >= 2 && !*abort_flag) {
     // --------------------- epilogue part 2: reduce S partials, bias, rotate, store
-    // A warp issues the DSMEM loads of all its batch's partial sums before any
-    // arithmetic or store, so their latencies overlap; the other operands of
-    // the first batch are in registers already.
-    const int d = p.rope_d, half = d >> 1, npl = half >> 5;
+    // Per row a lane issues the DSMEM loads of all S partials of its 8 columns
+    // (2 S 16-byte loads) before any add, so their latencies overlap, and the
+    // next row's table entries load meanwhile.
+    const int half = p.rope_d >> 1;
     const uint32_t part_base = smem_u32(part);
-    for (int32_t base = first; base < items; base += stride * kBatch) {
-      if (base != first) dc_load_items(p, n0, base, stride, items, heads, lane, batch);
-      float a[kBatch][kMaxPl], b[kBatch][kMaxPl];
+    for (int32_t k = 0; k < nrows; ++k) {
+      const int32_t t = first + k * stride;
+      DcRow nxt = cur;
+      if (k + 1 < nrows)
+        dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, k + 1), __shfl_sync(0xffffffffu, my_crow, k + 1), nxt);
+      if (!cur.ok) {
+        if (lane == 0) atomicOr(p.err, kErrBounds);
+      } else if (L.live) {
+        const int32_t c0 = L.hcol - n0 + L.i;
+        const uint32_t off = static_cast<uint32_t>((t * kDcPartStride + c0) * 4);
+        float4 va[8], vb[8];
 #pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-#pragma unroll
-        for (int m = 0; m < kMaxPl; ++m) {
-          a[j][m] = 0.0f;
-          b[j][m] = 0.0f;
-          if (batch[j].ok && m < npl) {
-            const int i = lane + 32 * m;
-            const uint32_t off = static_cast<uint32_t>((batch[j].t * kDcPartStride + (batch[j].hcol - n0) + i) * 4);
-            // all 2S loads in flight before the first add (their round trips
-            // overlap), then the sums in CTA-rank order
-            float va[8], vb[8];
-#pragma unroll
-            for (uint32_t s2 = 0; s2 < 8; ++s2) {
-              if (s2 < S) {
-                const uint32_t bs = mapa_shared(part_base, s2);
-                va[s2] = ld_cluster_f32(bs + off);
-                vb[s2] = ld_cluster_f32(bs + off + static_cast<uint32_t>(half * 4));
-              }
-            }
-#pragma unroll
-            for (uint32_t s2 = 0; s2 < 8; ++s2) {
-              if (s2 < S) {
-                a[j][m] += va[s2];
-                b[j][m] += vb[s2];
-              }
-            }
+        for (uint32_t s2 = 0; s2 < 8; ++s2) {
+          if (s2 < S) {
+            const uint32_t bs = mapa_shared(part_base, s2);
+            va[s2] = ld_cluster_f32x4(bs + off);
+            vb[s2] = ld_cluster_f32x4(bs + off + static_cast<uint32_t>(half * 4));
           }
         }
-      }
+        // the sums in CTA-rank order
+        float a[4] = {0.0f, 0.0f, 0.0f, 0.0f}, b[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        if (!batch[j].live) continue;
-        if (!batch[j].ok) {
-          if (lane == 0) atomicOr(p.err, kErrBounds);
-          continue;
+        for (uint32_t s2 = 0; s2 < 8; ++s2) {
+          if (s2 < S) {
+            a[0] += va[s2].x;
+            a[1] += va[s2].y;
+            a[2] += va[s2].z;
+            a[3] += va[s2].w;
+            b[0] += vb[s2].x;
+            b[1] += vb[s2].y;
+            b[2] += vb[s2].z;
+            b[3] += vb[s2].w;
+          }
         }
-        const int32_t hcol = batch[j].hcol;
+        float y0[4], y1[4];
+#pragma unroll
+        for (int m = 0; m < 4; ++m) {
+          float x0 = a[m] + L.b0[m], x1 = b[m] + L.b1[m];
+          if (L.rotate) {
+            const float c = cur.c[m], sn = cur.s[m];
+            const float r0 = fmaf(x0, c, -x1 * sn), r1 = fmaf(x1, c, x0 * sn);
+            x0 = r0;
+            x1 = r1;
+          }
+          y0[m] = x0;
+          y1[m] = x1;
+        }
         void* dst;
         int64_t dst0;
-        if (hcol < p.q_cols) {
+        if (L.hcol < p.q_cols) {
           dst = p.q_out;
-          dst0 = static_cast<int64_t>(batch[j].t) * p.ldq + hcol;
+          dst0 = static_cast<int64_t>(t) * p.ldq + L.hcol;
         } else {
-          dst = batch[j].rotate ? p.k_cache : p.v_cache;
-          dst0 = static_cast<int64_t>(batch[j].crow) * p.ld_cache + hcol - (batch[j].rotate ? p.q_cols : p.rot_cols);
+          dst = L.rotate ? p.k_cache : p.v_cache;
+          dst0 = static_cast<int64_t>(cur.crow) * p.ld_cache + L.hcol - (L.rotate ? p.q_cols : p.rot_cols);
         }
-#pragma unroll
-        for (int m = 0; m < kMaxPl; ++m) {
-          if (m >= npl) break;
-          const int i = lane + 32 * m;
-          float x0 = a[j][m] + batch[j].b0[m], x1 = b[j][m] + batch[j].b1[m];
-          if (batch[j].rotate) {
-            const float c = batch[j].c[m], sn = batch[j].s[m];
-            const float y0 = fmaf(x0, c, -x1 * sn), y1 = fmaf(x1, c, x0 * sn);
-            x0 = y0;
-            x1 = y1;
-          }
-          if (p.out_dtype == KF_F32) {
-            reinterpret_cast<float*>(dst)[dst0 + i] = x0;
-            reinterpret_cast<float*>(dst)[dst0 + i + half] = x1;
-          } else if (p.out_dtype == KF_BF16) {
-            reinterpret_cast<__nv_bfloat16*>(dst)[dst0 + i] = __float2bfloat16_rn(x0);
-            reinterpret_cast<__nv_bfloat16*>(dst)[dst0 + i + half] = __float2bfloat16_rn(x1);
-          } else {
-            reinterpret_cast<__half*>(dst)[dst0 + i] = __float2half_rn(x0);
-            reinterpret_cast<__half*>(dst)[dst0 + i + half] = __float2half_rn(x1);
-          }
-        }
+        dc_store4(dst, p.out_dtype, dst0 + L.i, y0[0], y0[1], y0[2], y0[3]);
+        dc_store4(dst, p.out_dtype, dst0 + L.i + half, y1[0], y1[1], y1[2], y1[3]);
       }
+      cur = nxt;
     }
   }
   // no CTA leaves while another may still read its shared memory

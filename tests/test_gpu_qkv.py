@@ -5,8 +5,8 @@ few-token calls (clusters splitting K, partials reduced in shared memory; token
 boxes of 32 and 64 rows), decode batches up to 128 tokens (one 128-row tile,
 narrow tiles), prefill (CTA
 pairs, ragged last row tile), 128- and 256-column heads, ragged last column
-tile, fp16 operands, fp32 / fp16 outputs, no bias, out-of-range positions,
-untouched cache rows, repeat runs."""
+tile, fp16 operands, fp32 / fp16 outputs, outputs at odd offsets and strides,
+no bias, out-of-range positions, untouched cache rows, repeat runs."""
 import numpy as np
 import pytest
 import torch
@@ -125,6 +125,31 @@ def test_no_bias_fp32_output():
     inp = kf_workloads.qkv_generate(10, seed=91, H=384, nq=4, nkv=1, d=128, cache_rows=64)
     got, ref, idx = _run(inp, 4, 1, 128, out_dtype=torch.float32, bias=False)
     _check(got, ref, idx, "no bias", out_dtype=torch.float32)
+
+
+@pytest.mark.parametrize("T", [3, 20, 64, 100])
+@pytest.mark.parametrize("out_dtype", [torch.bfloat16, torch.float32])
+def test_outputs_at_odd_offsets_and_strides(out_dtype, T):
+    # q_out and the caches one element past an aligned start, rows an odd number
+    # of elements apart: no vector store is legal, every output goes through
+    # the element-wise stores (weight stream, clusters, one tile)
+    s = kf_workloads.QKV_SHAPE
+    nq, nkv, d = s["nq"], s["nkv"], s["d"]
+    inp = kf_workloads.qkv_generate(T, seed=95 + T, cache_rows=256)
+    rows = int(inp["rows"])
+    qb = torch.full((T, nq * d + 3), SENT, dtype=out_dtype, device=DEV)
+    kb = torch.full((rows, nkv * d + 3), SENT, dtype=out_dtype, device=DEV)
+    vb = torch.full((rows, nkv * d + 3), SENT, dtype=out_dtype, device=DEV)
+    q, kc, vc = qb[:, 1:1 + nq * d], kb[:, 1:1 + nkv * d], vb[:, 1:1 + nkv * d]
+    g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
+    kf.qkv_rope_kv(g["X"], g["W"], g["b"], g["positions"], g["cache_rows"], g["cos"], g["sin"], nq, nkv, d, kc, vc,
+                   q_out=q)
+    assert kf.get_device_error()[0] == kf.KF_OK
+    for buf in (qb, kb, vb):  # the columns around the views stay untouched
+        assert bool((buf[:, 0] == SENT).all()) and bool((buf[:, -2:] == SENT).all())
+    rq, rk, rv = oracle.qkv_rope_kv(inp["X"], inp["W"], inp["b"], inp["positions"], inp["cache_rows"], inp["cos"],
+                                    inp["sin"], nq, nkv, d, rows)
+    _check((q, kc, vc), (rq, rk, rv), torch.arange(T), f"odd offsets T={T}", out_dtype=out_dtype)
 
 
 @pytest.mark.parametrize("T", [12, 40, 100])
