@@ -232,6 +232,16 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
+// The two halves of a cluster barrier: arrive without ordering (e.g. "this CTA
+// has started") and wait for every thread of the cluster to have arrived.
+__device__ __forceinline__ void cluster_arrive_relaxed() { asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait;" ::: "memory"); }
+// 16-byte store into (possibly another CTA's) shared memory of the cluster.
+__device__ __forceinline__ void st_cluster_f4(uint32_t cluster_addr, float a, float b, float c, float d) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(cluster_addr), "f"(a), "f"(b), "f"(c),
+               "f"(d)
+               : "memory");
+}
 // Arrive on an mbarrier of another CTA of the cluster (shared::cluster address).
 // Programmatic dependent launch: wait until the grids this one depends on have
 // completed and their writes are visible (no-op without such a dependency), and

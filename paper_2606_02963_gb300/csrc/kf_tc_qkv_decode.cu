@@ -7,21 +7,24 @@
 // A decode GEMM reads each weight once; one 256-column tile per CTA over the
 // whole K would keep only N / 256 SMs busy and pay 4 MMAs per 64-wide k-block
 // for all of K.  Here a cluster of S CTAs shares one 256-column tile (four
-// 64-column heads): CTA r multiplies the k-blocks [r K / S, (r + 1) K / S),
-// writes the T token rows of its 128 x 256 fp32 partial from TMEM into its own
-// shared memory (the operand ring, free by then), and after a cluster barrier the epilogue warps
-// of all S CTAs take the tile's token rows in turn: a warp sums the S partials
-// of its row (lane j: the four rotation pairs 4j .. 4j + 3 of the tile, read as
-// 16-byte loads from each CTA's shared memory through DSMEM), adds the bias,
-// rotates query and key heads and stores the row's heads to q_out or to the
-// token's cache row.  No global workspace, no atomics, no waits between CTAs
-// other than the two hardware cluster barriers.  While the MMAs run, the
-// epilogue warps already load what their rows need besides the sums (bias,
-// positions, cache rows, the first row's table entries), so that after the
-// barrier mostly the partial sums are read.
+// 64-column heads): CTA r multiplies the k-blocks [r K / S, (r + 1) K / S).
+// The tile's T token rows are dealt out to the cluster's CTAs in runs of
+// RPO = ceil(T / S) rows; each CTA sends every row of its 128 x 256 fp32
+// partial straight from TMEM to the shared memory of the row's owner (16-byte
+// DSMEM stores, which need no reply and overlap the other CTAs' mainloops; its
+// own rows go to its operand ring, free by then).  After one cluster barrier an
+// owner's epilogue warps reduce its rows from local shared memory alone: a warp
+// sums the S partials of a row in CTA-rank order (lane j: the four rotation
+// pairs 4j .. 4j + 3 of the tile), adds the bias, rotates query and key heads
+// and stores the row's heads to q_out or to the token's cache row.  No global
+// workspace, no atomics, no waits between CTAs other than the hardware cluster
+// barriers (one that every CTA has started before any DSMEM store, one after
+// the stores), and no CTA waits for the others to exit.  While the MMAs run,
+// the epilogue warps already load what their rows need besides the sums (bias,
+// positions, cache rows, the first row's table entries).
 //
-// Token rows are staged in boxes of ROWS = 32 (six-stage ring) or 64 rows
-// (five stages): the box is what limits the tokens of a call.
+// Token rows are staged in boxes of ROWS = 32 (five-stage ring) or 64 rows
+// (four stages): the box is what limits the tokens of a call.
 //
 // Warp roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 epilogue.
 #include "kf_internal.h"
@@ -46,24 +49,22 @@ struct DcCfg {
   static constexpr int kBBytes = kDcBN * kDcBK * 2;    // 32 KB
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr uint32_t kTxBytes = kStageBytes;
-  static constexpr int kPartBytes = ROWS * kDcPartStride * 4;
   static constexpr int kRingBytes = STAGES * kStageBytes;
-  static_assert(kPartBytes <= kRingBytes, "the partial fits the ring");
+  // after the mainloop the ring holds the CTA's own partial of the rows it
+  // owns; the other CTAs' partials of those rows land in a region of their own
+  // (written while this CTA may still be in its mainloop): (S - 1) ceil(T / S)
+  // rows, at most 60 (ROWS = 64) or 30 (ROWS = 32) for S <= 8
+  static constexpr int kRecvRows = ROWS == 64 ? 60 : 30;
+  static constexpr int kRowBytes = kDcPartStride * 4;
+  static_assert(ROWS * kRowBytes <= kRingBytes, "the own partial fits the ring");
   static_assert(STAGES * kABytes + kBBytes >= kDcBM * kDcBK * 2, "the MMA's 128-row reads stay in the ring");
-  static constexpr int kBarBytes = 8 * (2 * STAGES + 2);
-  static constexpr int kSmemBytes = 1024 + kRingBytes + kBarBytes + 64;
+  static constexpr int kBarBytes = 256;  // 2 STAGES + 2 barriers and three words
+  static_assert(8 * (2 * STAGES + 2) + 16 <= kBarBytes, "barrier block");
+  static constexpr int kRecvOff = kRingBytes + kBarBytes;
+  static constexpr int kSmemBytes = 1024 + kRecvOff + kRecvRows * kRowBytes;
   static constexpr uint32_t kIdesc = idesc_bf16_f32(kDcBM, kDcBN);
   static_assert(kSmemBytes <= 232448, "shared memory");
 };
-
-__device__ __forceinline__ float4 ld_cluster_f32x4(uint32_t addr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(addr)
-               : "memory");
-  return v;
-}
 
 // A tile row (one token, 256 columns) is reduced by one warp: lane j takes the
 // rotation pairs 4j .. 4j + 3 of the tile, i.e. four consecutive columns of one
@@ -168,7 +169,8 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* smA = sm;                                   // A stages first (see DcCfg)
   uint8_t* smB = sm + STAGES * Cfg::kABytes;
-  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: [ROWS][257] fp32
+  float* part = reinterpret_cast<float*>(sm);          // after the mainloop: own partial, [RPO][260] fp32
+  float* recv = reinterpret_cast<float*>(sm + Cfg::kRecvOff);  // other CTAs' partials, [S - 1][RPO][260]
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kRingBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
@@ -183,7 +185,8 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   // any barrier, TMEM allocation or copy
   const uint32_t S = cluster_nctarank();
   if (S != static_cast<uint32_t>(p.splits) || blockDim.x != kDcThreads || gridDim.x % S != 0 || gridDim.y != 1 ||
-      gridDim.z != 1 || p.T > ROWS) {
+      gridDim.z != 1 || p.T < 1 || p.T > ROWS ||
+      (static_cast<int32_t>(S) - 1) * ((p.T + static_cast<int32_t>(S) - 1) / static_cast<int32_t>(S)) > Cfg::kRecvRows) {
     if (threadIdx.x == 0) atomicOr(p.err, kErrLaunchShape);
     return;
   }
@@ -194,11 +197,12 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   const int32_t kb1 = static_cast<int32_t>(r + 1) * p.num_kb / static_cast<int32_t>(S);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // the tile's token rows go to the cluster's epilogue warps in turn: rows
-  // first, first + stride, ... of the call's T
-  const int32_t stride = static_cast<int32_t>(S) * 8;
-  const int32_t first = static_cast<int32_t>(r) + static_cast<int32_t>(S) * (warp - 2);
-  const int32_t nrows = warp >= 2 && first < p.T ? (p.T - first + stride - 1) / stride : 0;
+  // CTA o of the cluster owns the token rows [o RPO, (o + 1) RPO) of the tile
+  // and reduces them; its epilogue warp ew takes the owned rows ew, ew + 8, ...
+  const int32_t rpo = (p.T + static_cast<int32_t>(S) - 1) / static_cast<int32_t>(S);
+  const int32_t own0 = static_cast<int32_t>(r) * rpo;
+  const int32_t nown = max(0, min(rpo, p.T - own0));
+  const int32_t nrows = warp >= 2 && warp - 2 < nown ? (nown - (warp - 2) + 7) / 8 : 0;
   DcLane L;       // the epilogue lane's columns and bias
   DcRow cur;      // the warp's current row
   int32_t my_pos = 0, my_crow = 0;  // lane k < nrows: row k's position and cache row
@@ -239,6 +243,9 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
+  // this CTA has started: the other CTAs of the cluster may write its shared
+  // memory once every CTA has arrived here
+  cluster_arrive_relaxed();
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
@@ -290,18 +297,13 @@ __global__ void __launch_bounds__(kDcThreads, 1)
       }
     }
   } else {
-    // ------------------------------------- epilogue part 1: partial -> own smem
-    const int ew = warp - 2;
-    const int q = warp & 3;                      // TMEM lane quadrant
-    const int hh = ew >> 2;                      // column half: [128 hh, 128 hh + 128)
-    const int32_t row = q * 32 + lane;
-    // while the MMAs run: the lane's bias, the positions and cache rows of all
-    // the warp's rows (at most 8: T <= 64 and stride >= 8), the first row's
-    // table entries
+    // ------------------ epilogue: operands while the MMAs run, the accumulator
+    // the lane's bias, the positions and cache rows of all the warp's rows (at
+    // most 8: T <= 64 and 8 warps), the first row's table entries
     dc_lane(p, n0, lane, L);
     if (lane < nrows) {
-      my_pos = p.positions[first + lane * stride];
-      my_crow = p.cache_rows[first + lane * stride];
+      my_pos = p.positions[own0 + warp - 2 + 8 * lane];
+      my_crow = p.cache_rows[own0 + warp - 2 + 8 * lane];
     }
     if (nrows > 0)
       dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, 0), __shfl_sync(0xffffffffu, my_crow, 0), cur);
@@ -310,38 +312,66 @@ __global__ void __launch_bounds__(kDcThreads, 1)
     if (!w) {
       *abort_flag = 1;
       if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
-    } else {
-      tc_fence_after();
-      fence_proxy_async_smem();  // the ring's last copies were async-proxy writes
-      const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-      if (q * 32 < p.T) {  // quadrants past the last token have nothing to keep
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(tmem + lane_off + hh * 128 + c * 32, v);
-          if (row < p.T) {
-            float4* dst = reinterpret_cast<float4*>(part + row * kDcPartStride + hh * 128 + c * 32);
+    }
+  }
+  // every CTA of the cluster has started
+  cluster_wait();
+  if (warp >= 2 && !*abort_flag) {
+    // ------------- epilogue part 1: partial rows -> the owning CTA's shared memory
+    // Own rows go to the ring (idle: all copies landed and all MMAs completed
+    // before the accumulator was signalled), the others to slot r (r - 1 past
+    // the owner's rank) of the owner's receive region, as 16-byte DSMEM stores
+    // that need no reply.
+    const int ew = warp - 2;
+    const int q = warp & 3;  // TMEM lane quadrant
+    const int hh = ew >> 2;  // column half: [128 hh, 128 hh + 128)
+    const int32_t row = q * 32 + lane;
+    tc_fence_after();
+    fence_proxy_async_smem();  // the ring's last copies were async-proxy writes
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    if (q * 32 < p.T) {  // quadrants past the last token have nothing to keep
+      const int32_t rr = min(row, p.T - 1);  // lanes past the last token store nothing
+      const uint32_t o = static_cast<uint32_t>(rr / rpo);
+      const int32_t lr = rr - static_cast<int32_t>(o) * rpo;
+      uint32_t dst;
+      if (o == r) {
+        dst = smem_u32(part) + static_cast<uint32_t>(lr * Cfg::kRowBytes);
+      } else {
+        const uint32_t slot = r < o ? r : r - 1;
+        dst = mapa_shared(smem_u32(recv), o) + static_cast<uint32_t>((slot * rpo + lr) * Cfg::kRowBytes);
+      }
+      dst += static_cast<uint32_t>((hh * 128) * 4);
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        tmem_ld32(tmem + lane_off + hh * 128 + c * 32, v);
+        if (row < p.T) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-          }
+          for (int j = 0; j < 8; ++j)
+            st_cluster_f4(dst + static_cast<uint32_t>((c * 32 + 4 * j) * 4), v[4 * j], v[4 * j + 1], v[4 * j + 2],
+                          v[4 * j + 3]);
         }
       }
     }
   }
-  // every CTA's partial is in its shared memory (the ring is idle: all copies
-  // landed and all MMAs completed before the accumulator was signalled)
+  // every partial row is in its owner's shared memory; after this barrier no
+  // CTA touches another's shared memory, so none waits for the others to exit
   tc_fence_before();
   __syncwarp();
   cluster_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kDcBN);
+  }
 
   if (warp >= 2 && !*abort_flag) {
-    // --------------------- epilogue part 2: reduce S partials, bias, rotate, store
-    // Per row a lane issues the DSMEM loads of all S partials of its 8 columns
-    // (2 S 16-byte loads) before any add, so their latencies overlap, and the
-    // next row's table entries load meanwhile.
+    // ---------- epilogue part 2: reduce the S partials of the owned rows, bias,
+    // rotate, store (all from this CTA's shared memory); the next row's table
+    // entries load meanwhile
     const int half = p.rope_d >> 1;
-    const uint32_t part_base = smem_u32(part);
     for (int32_t k = 0; k < nrows; ++k) {
-      const int32_t t = first + k * stride;
+      const int32_t lr = warp - 2 + 8 * k;
+      const int32_t t = own0 + lr;
       DcRow nxt = cur;
       if (k + 1 < nrows)
         dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, k + 1), __shfl_sync(0xffffffffu, my_crow, k + 1), nxt);
@@ -349,14 +379,15 @@ __global__ void __launch_bounds__(kDcThreads, 1)
         if (lane == 0) atomicOr(p.err, kErrBounds);
       } else if (L.live) {
         const int32_t c0 = L.hcol - n0 + L.i;
-        const uint32_t off = static_cast<uint32_t>((t * kDcPartStride + c0) * 4);
         float4 va[8], vb[8];
 #pragma unroll
         for (uint32_t s2 = 0; s2 < 8; ++s2) {
           if (s2 < S) {
-            const uint32_t bs = mapa_shared(part_base, s2);
-            va[s2] = ld_cluster_f32x4(bs + off);
-            vb[s2] = ld_cluster_f32x4(bs + off + static_cast<uint32_t>(half * 4));
+            // rank s2's partial: the ring for this CTA's own, else its slot
+            const float* src = s2 == r ? part + lr * kDcPartStride
+                                       : recv + ((s2 < r ? s2 : s2 - 1) * rpo + lr) * kDcPartStride;
+            va[s2] = *reinterpret_cast<const float4*>(src + c0);
+            vb[s2] = *reinterpret_cast<const float4*>(src + c0 + half);
           }
         }
         // the sums in CTA-rank order
@@ -401,13 +432,6 @@ __global__ void __launch_bounds__(kDcThreads, 1)
       }
       cur = nxt;
     }
-  }
-  // no CTA leaves while another may still read its shared memory
-  cluster_sync();
-  if (warp == 1) {
-    __syncwarp();
-    tc_fence_after();
-    tmem_dealloc(tmem, kDcBN);
   }
 }
 
@@ -467,11 +491,11 @@ cudaError_t clusters_dc(int splits, int* out) {
 
 }  // namespace
 
-// token boxes of 32 rows (six stages) up to 32 tokens, of 64 rows (five) above
+// token boxes of 32 rows (five stages) up to 32 tokens, of 64 rows (four) above
 cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,
                               cudaStream_t s) {
   if (p.splits < 1 || p.splits > 8 || p.T < 1 || p.T > kQkvDecodeMaxRows) return cudaErrorInvalidValue;
-  return p.T <= 32 ? launch_dc<32, 6>(a, b, p, tiles, s) : launch_dc<64, 5>(a, b, p, tiles, s);
+  return p.T <= 32 ? launch_dc<32, 5>(a, b, p, tiles, s) : launch_dc<64, 4>(a, b, p, tiles, s);
 }
 
 int qkv_decode_box_rows(int64_t T) { return T <= 32 ? 32 : 64; }
@@ -487,7 +511,7 @@ cudaError_t qkv_decode_clusters(int64_t T, int splits, int* out) {
   const int v = T <= 32 ? 0 : 1;
   if (cache[dev][v][splits] == 0) {
     int nc = 0;
-    cudaError_t e = v == 0 ? clusters_dc<32, 6>(splits, &nc) : clusters_dc<64, 5>(splits, &nc);
+    cudaError_t e = v == 0 ? clusters_dc<32, 5>(splits, &nc) : clusters_dc<64, 4>(splits, &nc);
     if (e != cudaSuccess) return e;
     cache[dev][v][splits] = nc > 0 ? nc : -1;
   }
