@@ -677,8 +677,7 @@ def other_workloads(args, kf, dev, flush, stream, peaks):
         bound = "hbm" if byts / (peaks["hbm"] * 1e9) > flops / (peaks["bf16"] * 1e12) else "tensor"
         res[f"qkv_rope_kv_T{T}"] = {"tflops": round(flops / ms / 1e9, 2), "gbs": round(byts / ms / 1e6, 1),
                                    "ms": round(ms, 5), "bound": bound, "roofline_frac": round(t_roof / ms, 4),
-                                   "path": ("weight stream, one CTA per SM, warp-level MMAs" if T <= 8 else
-                                            "clusters splitting K" if T <= 64 else "tcgen05 tiles"),
+                                   "path": "clusters splitting K" if T <= 64 else "tcgen05 tiles",
                                    "unfused_ms": round(ms_u, 5),
                                    "speedup_vs_unfused": round(ms_u / ms, 3), "cublas_gemm_only_ms": round(ms_c, 5),
                                    "isolated_ms": round(ms_iso, 5),

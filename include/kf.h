@@ -317,13 +317,10 @@ kf_status kf_moe_ffn_add_rmsnorm(const void* X, const float* logits, const void*
  *   q_out [T x ldq], k_cache / v_cache [cache_rows_n x ld_cache]: out_dtype
  *     (KF_BF16, KF_F16 or KF_F32); ldq >= nq d, ld_cache >= nkv d.
  *   d: a multiple of 64, at most 256 (KF_ERR_UNSUPPORTED otherwise); nq, nkv >= 1.
- *   Calls of at most 8 tokens with H a multiple of 8, H <= 4096, stream the
- *   weights: the heads' rotation pairs are dealt out in contiguous runs to one
- *   CTA per SM, each CTA holds all of its weight rows in shared memory at once
- *   (when they fit) and adds its dot products in a fixed order.  Other calls of
- *   at most 64 tokens with d dividing 256 run as clusters of CTAs that split K
- *   over each 256-column tile and add their partial sums in shared memory.
- *   Either way repeated calls are bitwise identical.
+ *   Calls of at most 64 tokens with d dividing 256 run as clusters of CTAs
+ *   that split K over each 256-column tile and add their partial sums in
+ *   shared memory in a fixed order; larger calls run as tensor-core tiles over
+ *   the whole K.  Either way repeated calls are bitwise identical.
  *   T = 0 writes nothing.  All buffers are the caller's; nothing is allocated.
  */
 kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dtype, int64_t ldx, int64_t ldw, const void* bias,

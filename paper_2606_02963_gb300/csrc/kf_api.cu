@@ -1233,8 +1233,26 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
   if (st != KF_OK) return st;
   const bool cta2 = T > kBM && di.nsm >= 2;
   const int64_t num_kb = (H + kBK - 1) / kBK;
-  // the fields the few-token kernels share
-  auto fill_decode = [&](QkvDecodeParams& dp) {
+  if (T <= kQkvClusterMaxT && 256 % d == 0) {
+    // few tokens: clusters of S CTAs split K over one 256-column tile and
+    // reduce through distributed shared memory; S as large as keeps every
+    // cluster of the call resident at once
+    const int64_t tiles = (N + 255) / 256;
+    int S = 1;
+    for (int cand : {8, 6, 4, 2}) {
+      int nc = 0;
+      if (cand <= num_kb && qkv_decode_clusters(T, cand, &nc) == cudaSuccess && nc >= tiles) {
+        S = cand;
+        break;
+      }
+    }
+    const CUtensorMapDataType dt = xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    CUtensorMap ma, mb;
+    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, qkv_decode_box_rows(T), 2, dt);  // token boxes of 32 or 64 rows
+    if (st != KF_OK) return st;
+    st = make_map(&mb, W, H, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, 256, 3, dt);
+    if (st != KF_OK) return st;
+    QkvDecodeParams dp;
     std::memset(&dp, 0, sizeof(dp));
     dp.T = static_cast<int32_t>(T);
     dp.N = static_cast<int32_t>(N);
@@ -1261,43 +1279,6 @@ extern "C" kf_status kf_qkv_rope_kv(const void* X, const void* W, int32_t xw_dty
     dp.err = di.err;
     dp.wait_ns = g_wait_ns.load();
     dp.drain_ns = std::max<uint64_t>(dp.wait_ns, 1000000000ull);
-  };
-  if (T <= kQkvGemvMaxT) {
-    // one or two tokens: a weight stream on the CUDA cores, one CTA per head
-    // (or per part of its rotation pairs)
-    QkvGemvParams gp;
-    std::memset(&gp, 0, sizeof(gp));
-    size_t smem = 0;
-    if (qkv_gemv_plan(T, H, nq + 2 * nkv, d, di.nsm, &gp, &smem)) {
-      fill_decode(gp.q);
-      gp.X = X;
-      gp.ldx = ldx;
-      gp.W = W;
-      gp.ldw = ldw;
-      return cuda_status(qkv_gemv_launch(gp, smem, s));
-    }
-  }
-  if (T <= kQkvClusterMaxT && 256 % d == 0) {
-    // few tokens: clusters of S CTAs split K over one 256-column tile and
-    // reduce through distributed shared memory; S as large as keeps every
-    // cluster of the call resident at once
-    const int64_t tiles = (N + 255) / 256;
-    int S = 1;
-    for (int cand : {8, 6, 4, 2}) {
-      int nc = 0;
-      if (cand <= num_kb && qkv_decode_clusters(T, cand, &nc) == cudaSuccess && nc >= tiles) {
-        S = cand;
-        break;
-      }
-    }
-    const CUtensorMapDataType dt = xw_dtype == KF_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
-    CUtensorMap ma, mb;
-    st = make_map(&ma, X, H, T, ldx * 2, 1, 0, qkv_decode_box_rows(T), 2, dt);  // token boxes of 32 or 64 rows
-    if (st != KF_OK) return st;
-    st = make_map(&mb, W, H, N, ldw * 2, 1, static_cast<uint64_t>(N) * ldw * 2, 256, 3, dt);
-    if (st != KF_OK) return st;
-    QkvDecodeParams dp;
-    fill_decode(dp);
     dp.splits = S;
     return cuda_status(qkv_decode_launch(ma, mb, dp, static_cast<int>(tiles), s));
   }

@@ -92,26 +92,6 @@ struct QkvDecodeParams {
   uint64_t wait_ns;
   uint64_t drain_ns;
 };
-// Up to eight tokens: the projection as a weight stream, the heads' rotation
-// pairs dealt out in contiguous runs to one CTA per SM, all of a CTA's weight
-// rows in shared memory at once, warp-level MMAs; `g.q` as for the cluster
-// kernel (its T, K, ab_f16, bias, rotation and output fields).
-constexpr int kQkvGemvMaxT = 8;
-struct QkvGemvParams {
-  QkvDecodeParams q;
-  const void* X;
-  int64_t ldx;
-  const void* W;
-  int64_t ldw;
-  int32_t ctas, pairs;       // CTA c takes pairs [c pairs / ctas, (c + 1) pairs / ctas)
-  int32_t max_stages;        // stages of 8 rows of the CTA with the most pairs
-  int32_t max_pairs;         // pairs of that CTA
-  int32_t buf_rows, stride;  // weight rows in shared memory, bytes between them
-};
-// Tile the call (false: T, H or d outside what the kernel serves, or a CTA's
-// rows do not fit its shared memory); fills the launch fields of *g and *smem.
-bool qkv_gemv_plan(int64_t T, int64_t H, int32_t heads, int32_t d, int nsm, QkvGemvParams* g, size_t* smem);
-cudaError_t qkv_gemv_launch(const QkvGemvParams& g, size_t smem, cudaStream_t s);
 // few-token QKV tail: at most this many tokens; A boxes of qkv_decode_box_rows(T) rows
 constexpr int kQkvDecodeMaxRows = 64;
 cudaError_t qkv_decode_launch(const CUtensorMap& a, const CUtensorMap& b, const QkvDecodeParams& p, int tiles,

@@ -132,7 +132,8 @@ def test_no_bias_fp32_output():
 def test_outputs_at_odd_offsets_and_strides(out_dtype, T):
     # q_out and the caches one element past an aligned start, rows an odd number
     # of elements apart: no vector store is legal, every output goes through
-    # the element-wise stores (weight stream, clusters, one tile)
+    # the element-wise stores (clusters with direct and with staged partial
+    # rows, one tcgen05 tile)
     s = kf_workloads.QKV_SHAPE
     nq, nkv, d = s["nq"], s["nkv"], s["d"]
     inp = kf_workloads.qkv_generate(T, seed=95 + T, cache_rows=256)

@@ -1,11 +1,11 @@
-"""GPU parity of the QKV projection tail for up to eight tokens (the weight
-stream: rotation pairs dealt out to one CTA per SM, all of a CTA's weight rows
-in shared memory at once, warp-level MMAs, bias, rotary embedding, key / value
+"""GPU parity of the QKV projection tail for one to eight tokens (clusters of
+CTAs splitting K over 256-column tiles, partial rows pushed to their owning
+CTA through distributed shared memory, bias, rotary embedding, key / value
 cache rows; the gpt-oss decode kernel "Bias + RoPE + KV update" of Sec. IV-A)
-against the oracle: the gpt-oss shape, 128- and 256-column heads, CTAs with
-fewer rows than a stage and with 17 stages, rows of one 16-byte chunk, fp16
-operands, fp32 / fp16 outputs, fp32 and absent bias, strided weight rows,
-out-of-range positions and cache rows, repeats."""
+against the oracle: the gpt-oss shape, 128- and 256-column heads, K of one
+partial k-block and of four k-blocks, many heads, fp16 operands, fp32 / fp16
+outputs, fp32 and absent bias, strided weight rows, out-of-range positions and
+cache rows, repeats."""
 import numpy as np
 import pytest
 import torch
@@ -54,39 +54,39 @@ def test_gpt_oss_shape(T):
     s = kf_workloads.QKV_SHAPE
     inp = kf_workloads.qkv_generate(T, seed=300 + T, cache_rows=4096)
     got, ref = _run(inp, s["nq"], s["nkv"], s["d"])
-    _check(got, ref, f"gemv T={T}")
+    _check(got, ref, f"few T={T}")
 
 
 @pytest.mark.parametrize("T", [1, 8])
 @pytest.mark.parametrize("nq,nkv,d,H", [(8, 2, 128, 640), (2, 1, 256, 512), (32, 8, 128, 4096), (3, 2, 64, 8),
                                          (64, 8, 128, 512), (72, 4, 256, 256)])
 def test_head_sizes_row_widths(nq, nkv, d, H, T):
-    # 128- and 256-column heads; few pairs per CTA (fewer rows than a stage)
-    # and many (up to 68 pairs, 17 stages); 8-wide rows (one 16-byte chunk,
-    # half a k-step); 48 heads of 128 at H = 4096 do not fit one CTA's shared
-    # memory per SM and take the cluster path
+    # 128- and 256-column heads; K of 8 (one partial k-block: clusters of one
+    # CTA) and 256 (four k-blocks: clusters of at most four); 48 heads of 128
+    # at H = 4096 (24 tiles); 80 heads of 128 and of 256 (40 and 80 tiles)
     inp = kf_workloads.qkv_generate(T, seed=310 + d + nq + T + H, H=H, nq=nq, nkv=nkv, d=d, cache_rows=64)
     got, ref = _run(inp, nq, nkv, d)
-    _check(got, ref, f"gemv nq={nq} nkv={nkv} d={d} H={H} T={T}")
+    _check(got, ref, f"few nq={nq} nkv={nkv} d={d} H={H} T={T}")
 
 
 @pytest.mark.parametrize("out_dtype", [torch.float32, torch.float16])
 def test_fp16_operands_and_wide_outputs(out_dtype):
     inp = kf_workloads.qkv_generate(5, seed=320, H=2880, nq=16, nkv=4, d=64, dtype="f16", cache_rows=300)
     got, ref = _run(inp, 16, 4, 64, out_dtype=out_dtype)
-    _check(got, ref, f"gemv f16 -> {out_dtype}", out_dtype=out_dtype)
+    _check(got, ref, f"few f16 -> {out_dtype}", out_dtype=out_dtype)
 
 
 def test_no_bias_fp32_output_and_fp32_bias():
     inp = kf_workloads.qkv_generate(1, seed=321, H=384, nq=4, nkv=1, d=128, cache_rows=64)
     got, ref = _run(inp, 4, 1, 128, out_dtype=torch.float32, bias=False)
-    _check(got, ref, "gemv no bias", out_dtype=torch.float32)
+    _check(got, ref, "few no bias", out_dtype=torch.float32)
     got, ref = _run(inp, 4, 1, 128, bias_f32=True)
-    _check(got, ref, "gemv fp32 bias")
+    _check(got, ref, "few fp32 bias")
 
 
 def test_strided_weight_rows():
-    # W rows 8 elements apart from the next row's start: one bulk copy per row
+    # W rows 8 elements apart from the next row's start (the tensor map's row
+    # stride)
     s = kf_workloads.QKV_SHAPE
     inp = kf_workloads.qkv_generate(4, seed=322, cache_rows=128)
     N, H = inp["W"].shape
@@ -96,7 +96,7 @@ def test_strided_weight_rows():
     Wd = big.to(DEV)[:, :H]
     assert Wd.stride(0) == H + 8
     got, ref = _run(inp, s["nq"], s["nkv"], s["d"], W=Wd)
-    _check(got, ref, "gemv strided W")
+    _check(got, ref, "few strided W")
 
 
 @pytest.mark.parametrize("bad_field", ["position", "cache_row"])
@@ -125,17 +125,17 @@ def test_out_of_range_token_skips_only_that_token(bad_field):
     good = torch.tensor([t for t in range(T) if t != bad])
     rq, rk, rv = oracle.qkv_rope_kv(inp["X"][good], inp["W"], inp["b"], inp["positions"][good],
                                     inp["cache_rows"][good], inp["cos"], inp["sin"], nq, nkv, d, rows)
-    check_bf16(q[good.to(DEV)], rq, "gemv good tokens q")
+    check_bf16(q[good.to(DEV)], rq, "few good tokens q")
     named = np.flatnonzero(~np.isnan(rk[:, 0]))
-    check_bf16(kc[torch.as_tensor(named, device=DEV)], rk[named], "gemv good tokens k")
-    check_bf16(vc[torch.as_tensor(named, device=DEV)], rv[named], "gemv good tokens v")
+    check_bf16(kc[torch.as_tensor(named, device=DEV)], rk[named], "few good tokens k")
+    check_bf16(vc[torch.as_tensor(named, device=DEV)], rv[named], "few good tokens v")
     assert kf.get_device_error()[0] == kf.KF_OK  # the read cleared the word
 
 
 @pytest.mark.parametrize("T", [1, 8])
 def test_repeats_bitwise(T):
-    # each row's dot product has a fixed order (k-steps per warp, then the
-    # warps' partials in warp order)
+    # each output's sum has a fixed order (k-blocks within a CTA, then the
+    # CTAs' partials in cluster-rank order)
     s = kf_workloads.QKV_SHAPE
     inp = kf_workloads.qkv_generate(T, seed=324 + T)
     g = {k: v.to(DEV) for k, v in inp.items() if k != "rows"}
