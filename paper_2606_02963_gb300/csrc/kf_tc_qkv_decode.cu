@@ -10,18 +10,20 @@
 // 64-column heads): CTA r multiplies the k-blocks [r K / S, (r + 1) K / S).
 // The tile's T token rows are dealt out to the cluster's CTAs in runs of
 // RPO = ceil(T / S) rows; each CTA sends every row of its 128 x 256 fp32
-// partial straight from TMEM to the shared memory of the row's owner (16-byte
-// DSMEM stores, which need no reply and overlap the other CTAs' mainloops; its
-// own rows go to its operand ring, free by then).  After one cluster barrier an
-// owner's epilogue warps reduce its rows from local shared memory alone: a warp
-// sums the S partials of a row in CTA-rank order (lane j: the four rotation
-// pairs 4j .. 4j + 3 of the tile), adds the bias, rotates query and key heads
-// and stores the row's heads to q_out or to the token's cache row.  No global
-// workspace, no atomics, no waits between CTAs other than the hardware cluster
-// barriers (one that every CTA has started before any DSMEM store, one after
-// the stores), and no CTA waits for the others to exit.  While the MMAs run,
-// the epilogue warps already load what their rows need besides the sums (bias,
-// positions, cache rows, the first row's table entries).
+// partial to the shared memory of the row's owner as 16-byte DSMEM stores,
+// which need no reply and overlap the other CTAs' mainloops: up to 32 tokens
+// straight from TMEM (lane = row), above that staged in its operand ring (free
+// by then) and sent as whole 512-byte warp stores by all ten warps.  After one
+// cluster barrier an owner's epilogue warps reduce its rows from local shared
+// memory alone (its own rows from its ring): a warp sums the S partials of a
+// row in CTA-rank order (lane j: the four rotation pairs 4j .. 4j + 3 of the
+// tile), adds the bias, rotates query and key heads and stores the row's heads
+// to q_out or to the token's cache row.  No global workspace, no atomics, no
+// waits between CTAs other than the hardware cluster barriers (one that every
+// CTA has started before any DSMEM store, one after the stores), and no CTA
+// waits for the others to exit.  While the MMAs run, the epilogue warps already
+// load what their rows need besides the sums (bias, positions, cache rows, the
+// first two rows' table entries).
 //
 // Token rows are staged in boxes of ROWS = 32 (five-stage ring) or 64 rows
 // (four stages): the box is what limits the tokens of a call.
@@ -36,6 +38,7 @@ constexpr int kDcThreads = 320;
 constexpr int kDcBM = 128;          // rows of the MMA (only the first T are tokens)
 constexpr int kDcBK = 64;           // K elements per 128-byte row
 constexpr int kDcBN = 256;          // tile columns
+constexpr int kDcDirectMaxT = 32;  // up to this many tokens partial rows leave TMEM for their owners directly
 constexpr int kDcPartStride = 260;  // floats per partial row (4 banks apart: conflict-free 16-byte row-per-lane stores)
 
 template <int ROWS, int STAGES>
@@ -84,6 +87,30 @@ struct DcRow {
   float c[4], s[4];
 };
 
+// A 16-byte load of read-only data issued exactly here: a plain __ldg may be
+// moved to its first use (read-only loads are free to move), which would put
+// its latency back after the cluster barrier that this prefetch is meant to
+// hide it behind.
+__device__ __forceinline__ float4 ldg_f4_here(const float* ptr) {
+  float4 v;
+  asm volatile("ld.global.nc.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(ptr));
+  return v;
+}
+// one bias element (fp32, bf16 or fp16), issued exactly here likewise
+__device__ __forceinline__ float ld_bias_here(const void* ptr, int dt, int64_t i) {
+  uint32_t b;
+  if (dt == KF_F32) {
+    asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(b) : "l"(static_cast<const uint32_t*>(ptr) + i));
+  } else {
+    uint16_t h;
+    asm volatile("ld.global.nc.b16 %0, [%1];" : "=h"(h) : "l"(static_cast<const uint16_t*>(ptr) + i));
+    b = h;
+  }
+  return cvt_raw(b, dt);
+}
+
 __device__ __forceinline__ void dc_lane(const QkvDecodeParams& p, int32_t n0, int lane, DcLane& L) {
   const int d = p.rope_d, half = d >> 1;
   const int pr = 4 * lane;
@@ -94,9 +121,21 @@ __device__ __forceinline__ void dc_lane(const QkvDecodeParams& p, int32_t n0, in
 #pragma unroll
   for (int m = 0; m < 4; ++m) {
     const bool use = L.live && p.bias;
-    L.b0[m] = use ? ld_elem(p.bias, p.bias_dtype, L.hcol + L.i + m) : 0.0f;
-    L.b1[m] = use ? ld_elem(p.bias, p.bias_dtype, L.hcol + L.i + m + half) : 0.0f;
+    L.b0[m] = use ? ld_bias_here(p.bias, p.bias_dtype, L.hcol + L.i + m) : 0.0f;
+    L.b1[m] = use ? ld_bias_here(p.bias, p.bias_dtype, L.hcol + L.i + m + half) : 0.0f;
   }
+}
+
+// 16 bytes of this CTA's shared memory (explicit state space: the partial
+// buffers are addressed through an aligned integer, which a plain pointer
+// access would turn into a generic load or store)
+__device__ __forceinline__ float4 lds_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ void sts_f4(uint32_t addr, float a, float b, float c, float d) {
+  asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d) : "memory");
 }
 
 // A position or cache row out of range clears `ok` (the row is then reported
@@ -112,8 +151,8 @@ __device__ __forceinline__ void dc_row(const QkvDecodeParams& p, const DcLane& L
   float4 c = make_float4(1.0f, 1.0f, 1.0f, 1.0f), s = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   if (R.ok && L.live && L.rotate) {
     const int64_t o = static_cast<int64_t>(pos) * half + L.i;
-    c = __ldg(reinterpret_cast<const float4*>(p.cos_t + o));
-    s = __ldg(reinterpret_cast<const float4*>(p.sin_t + o));
+    c = ldg_f4_here(p.cos_t + o);
+    s = ldg_f4_here(p.sin_t + o);
   }
   R.c[0] = c.x;
   R.c[1] = c.y;
@@ -204,7 +243,7 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   const int32_t nown = max(0, min(rpo, p.T - own0));
   const int32_t nrows = warp >= 2 && warp - 2 < nown ? (nown - (warp - 2) + 7) / 8 : 0;
   DcLane L;       // the epilogue lane's columns and bias
-  DcRow cur;      // the warp's current row
+  DcRow cur, nxt;  // the warp's current and next row
   int32_t my_pos = 0, my_crow = 0;  // lane k < nrows: row k's position and cache row
 
   if (threadIdx.x == 0) {
@@ -243,6 +282,7 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
+  bool acc_ok = false;  // epilogue warps: the accumulator is complete
   // this CTA has started: the other CTAs of the cluster may write its shared
   // memory once every CTA has arrived here
   cluster_arrive_relaxed();
@@ -299,7 +339,7 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   } else {
     // ------------------ epilogue: operands while the MMAs run, the accumulator
     // the lane's bias, the positions and cache rows of all the warp's rows (at
-    // most 8: T <= 64 and 8 warps), the first row's table entries
+    // most 8: T <= 64 and 8 warps), the first two rows' table entries
     dc_lane(p, n0, lane, L);
     if (lane < nrows) {
       my_pos = p.positions[own0 + warp - 2 + 8 * lane];
@@ -307,21 +347,28 @@ __global__ void __launch_bounds__(kDcThreads, 1)
     }
     if (nrows > 0)
       dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, 0), __shfl_sync(0xffffffffu, my_crow, 0), cur);
+    if (nrows > 1)
+      dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, 1), __shfl_sync(0xffffffffu, my_crow, 1), nxt);
     bool w = mbar_wait(accf, 0, abort_flag, p.wait_ns);
-    w = __all_sync(0xffffffffu, w);
-    if (!w) {
+    acc_ok = __all_sync(0xffffffffu, w);
+    if (!acc_ok) {
       *abort_flag = 1;
       if (lane == 0) atomicOr(p.err, kErrWaitEpilogue);
     }
   }
   // every CTA of the cluster has started
   cluster_wait();
-  if (warp >= 2 && !*abort_flag) {
-    // ------------- epilogue part 1: partial rows -> the owning CTA's shared memory
-    // Own rows go to the ring (idle: all copies landed and all MMAs completed
-    // before the accumulator was signalled), the others to slot r (r - 1 past
-    // the owner's rank) of the owner's receive region, as 16-byte DSMEM stores
-    // that need no reply.
+  // Few rows go straight from TMEM to their owners (lane = row: the warps of
+  // the token quadrants alone send); more rows are staged in this CTA's ring
+  // first and sent by all ten warps as whole 512-byte warp stores, which the
+  // DSMEM path moves much faster.
+  const bool direct = p.T <= kDcDirectMaxT;
+  if (warp >= 2 && acc_ok) {
+    // -------------------------------- epilogue part 1: partial rows out of TMEM
+    // Own rows (all rows when staging) go to the ring (idle: all copies landed
+    // and all MMAs completed before the accumulator was signalled), row t at
+    // t * 260 floats; the others to slot r (r - 1 past the owner's rank) of the
+    // owner's receive region.  DSMEM stores need no reply.
     const int ew = warp - 2;
     const int q = warp & 3;  // TMEM lane quadrant
     const int hh = ew >> 2;  // column half: [128 hh, 128 hh + 128)
@@ -332,23 +379,50 @@ __global__ void __launch_bounds__(kDcThreads, 1)
     if (q * 32 < p.T) {  // quadrants past the last token have nothing to keep
       const int32_t rr = min(row, p.T - 1);  // lanes past the last token store nothing
       const uint32_t o = static_cast<uint32_t>(rr / rpo);
-      const int32_t lr = rr - static_cast<int32_t>(o) * rpo;
-      uint32_t dst;
-      if (o == r) {
-        dst = smem_u32(part) + static_cast<uint32_t>(lr * Cfg::kRowBytes);
-      } else {
+      uint32_t dst = smem_u32(part) + static_cast<uint32_t>(rr * Cfg::kRowBytes);
+      if (direct && o != r) {
         const uint32_t slot = r < o ? r : r - 1;
+        const int32_t lr = rr - static_cast<int32_t>(o) * rpo;
         dst = mapa_shared(smem_u32(recv), o) + static_cast<uint32_t>((slot * rpo + lr) * Cfg::kRowBytes);
       }
       dst += static_cast<uint32_t>((hh * 128) * 4);
       for (int c = 0; c < 4; ++c) {
         float v[32];
         tmem_ld32(tmem + lane_off + hh * 128 + c * 32, v);
-        if (row < p.T) {
+        // sent directly: one store path for the warp's own and remote rows
+        // alike (splitting the lanes over two paths costs more than it saves)
+        if (row < p.T && direct) {
 #pragma unroll
           for (int j = 0; j < 8; ++j)
             st_cluster_f4(dst + static_cast<uint32_t>((c * 32 + 4 * j) * 4), v[4 * j], v[4 * j + 1], v[4 * j + 2],
                           v[4 * j + 3]);
+        } else if (row < p.T) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            sts_f4(dst + static_cast<uint32_t>((c * 32 + 4 * j) * 4), v[4 * j], v[4 * j + 1], v[4 * j + 2],
+                   v[4 * j + 3]);
+        }
+      }
+    }
+  }
+  if (!direct) {
+    __syncthreads();
+    if (!*abort_flag) {
+      // ----------- epilogue part 2: staged rows other CTAs own -> their shared memory
+      // warp w sends rows w, w + 10, ... (a row is 1 KB: two 512-byte warp
+      // stores, lane j: 16 bytes)
+      for (int32_t t = warp; t < p.T; t += kDcThreads / 32) {
+        const uint32_t o = static_cast<uint32_t>(t / rpo);
+        if (o == r) continue;  // reduced in place
+        const uint32_t slot = r < o ? r : r - 1;
+        const int32_t lr = t - static_cast<int32_t>(o) * rpo;
+        const uint32_t dst =
+            mapa_shared(smem_u32(recv), o) + static_cast<uint32_t>((slot * rpo + lr) * Cfg::kRowBytes);
+        const uint32_t src = smem_u32(part) + static_cast<uint32_t>(t * Cfg::kRowBytes);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const float4 v = lds_f4(src + static_cast<uint32_t>((h * 128 + 4 * lane) * 4));
+          st_cluster_f4(dst + static_cast<uint32_t>((h * 128 + 4 * lane) * 4), v.x, v.y, v.z, v.w);
         }
       }
     }
@@ -365,16 +439,16 @@ __global__ void __launch_bounds__(kDcThreads, 1)
   }
 
   if (warp >= 2 && !*abort_flag) {
-    // ---------- epilogue part 2: reduce the S partials of the owned rows, bias,
-    // rotate, store (all from this CTA's shared memory); the next row's table
-    // entries load meanwhile
+    // ---------- epilogue part 3: reduce the S partials of the owned rows, bias,
+    // rotate, store (all from this CTA's shared memory); the table entries of
+    // the row after the next load meanwhile
     const int half = p.rope_d >> 1;
     for (int32_t k = 0; k < nrows; ++k) {
       const int32_t lr = warp - 2 + 8 * k;
       const int32_t t = own0 + lr;
-      DcRow nxt = cur;
-      if (k + 1 < nrows)
-        dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, k + 1), __shfl_sync(0xffffffffu, my_crow, k + 1), nxt);
+      DcRow nn = nxt;  // the row after the next one, loaded while this one is reduced
+      if (k + 2 < nrows)
+        dc_row(p, L, __shfl_sync(0xffffffffu, my_pos, k + 2), __shfl_sync(0xffffffffu, my_crow, k + 2), nn);
       if (!cur.ok) {
         if (lane == 0) atomicOr(p.err, kErrBounds);
       } else if (L.live) {
@@ -384,10 +458,11 @@ __global__ void __launch_bounds__(kDcThreads, 1)
         for (uint32_t s2 = 0; s2 < 8; ++s2) {
           if (s2 < S) {
             // rank s2's partial: the ring for this CTA's own, else its slot
-            const float* src = s2 == r ? part + lr * kDcPartStride
-                                       : recv + ((s2 < r ? s2 : s2 - 1) * rpo + lr) * kDcPartStride;
-            va[s2] = *reinterpret_cast<const float4*>(src + c0);
-            vb[s2] = *reinterpret_cast<const float4*>(src + c0 + half);
+            const uint32_t src =
+                s2 == r ? smem_u32(part) + static_cast<uint32_t>(t * Cfg::kRowBytes)
+                        : smem_u32(recv) + static_cast<uint32_t>(((s2 < r ? s2 : s2 - 1) * rpo + lr) * Cfg::kRowBytes);
+            va[s2] = lds_f4(src + static_cast<uint32_t>(c0 * 4));
+            vb[s2] = lds_f4(src + static_cast<uint32_t>((c0 + half) * 4));
           }
         }
         // the sums in CTA-rank order
@@ -431,6 +506,7 @@ __global__ void __launch_bounds__(kDcThreads, 1)
         dc_store4(dst, p.out_dtype, dst0 + L.i + half, y1[0], y1[1], y1[2], y1[3]);
       }
       cur = nxt;
+      nxt = nn;
     }
   }
 }
