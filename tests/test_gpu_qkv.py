@@ -2,7 +2,7 @@
 heads, key / value cache rows; the gpt-oss decode kernel "Bias + RoPE + KV
 update" of Sec. IV-A, here fused with the projection GEMM) against the oracle:
 few-token calls (clusters splitting K, partials reduced in shared memory; token
-boxes of 32 and 64 rows), decode batches up to 128 tokens (one 128-row tile,
+boxes of 32 and 64 rows; clusters of one to three CTAs owning many rows), decode batches up to 128 tokens (one 128-row tile,
 narrow tiles), prefill (CTA
 pairs, ragged last row tile), 128- and 256-column heads, ragged last column
 tile, fp16 operands, fp32 / fp16 outputs, outputs at odd offsets and strides,
@@ -125,6 +125,17 @@ def test_no_bias_fp32_output():
     inp = kf_workloads.qkv_generate(10, seed=91, H=384, nq=4, nkv=1, d=128, cache_rows=64)
     got, ref, idx = _run(inp, 4, 1, 128, out_dtype=torch.float32, bias=False)
     _check(got, ref, idx, "no bias", out_dtype=torch.float32)
+
+
+@pytest.mark.parametrize("nq,nkv,d,H,T", [(3, 2, 64, 8, 45), (3, 2, 64, 8, 64), (8, 2, 64, 128, 64),
+                                           (8, 2, 128, 192, 33), (4, 4, 64, 64, 17)])
+def test_few_k_blocks_many_rows_per_cta(nq, nkv, d, H, T):
+    # K of one to three k-blocks: clusters of one to three CTAs, so a CTA owns
+    # up to 64 of the tile's token rows and an epilogue warp reduces up to 8 of
+    # them (positions of all, table rows two ahead), staged and direct
+    inp = kf_workloads.qkv_generate(T, seed=70 + H + T, H=H, nq=nq, nkv=nkv, d=d, cache_rows=256)
+    got, ref, idx = _run(inp, nq, nkv, d)
+    _check(got, ref, idx, f"H={H} T={T}")
 
 
 @pytest.mark.parametrize("T", [3, 20, 64, 100])
