@@ -460,6 +460,7 @@ struct GroupExtras {
   float sw_alpha = 1.0f, sw_limit = 0.0f, sw_c = 0.0f;
   void* zero_ptr = nullptr;  // SwiGLU: cleared while its first units run (see TcParams)
   int64_t zero_bytes = 0;
+  int64_t max_group_rows = 0;  // an upper bound on every group's rows, when the caller knows one (0: none)
 };
 
 // `pdl`: the previous kernel in the stream is one of this library's (MoE chain),
@@ -480,8 +481,11 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, uint
   if (bn == 0) return KF_ERR_UNSUPPORTED;
   const int outn = pl.mode == kModeSwiglu ? bn / 2 : bn;
   const int64_t nb = pl.mode == kModeSwiglu ? 2 * g.N : g.N;
+  // groups known to hold at most 64 rows take the variant with 64-row A slots
+  // (and a deeper ring), where there is one
+  const int ar = ex && ex->max_group_rows > 0 && ex->max_group_rows <= 64 && tc_grouped_has(pl.mode, bn, 64) ? 64 : kBM;
   CUtensorMap ma, mb;
-  kf_status st = make_map(&ma, A, g.K, g.rows_total, lda * 2, 1, 0, kBM, 2);
+  kf_status st = make_map(&ma, A, g.K, g.rows_total, lda * 2, 1, 0, ar, 2);
   if (st != KF_OK) return st;
   st = make_map(&mb, g.B, g.K, nb, g.ldb * 2, g.G, g.b_group_stride * 2, mode_box(pl.mode, bn), 3);
   if (st != KF_OK) return st;
@@ -519,7 +523,7 @@ kf_status grouped_core(const GroupedArgs& g, const ChainPlan& pl, void* ws, uint
   CUtensorMap mc;  // grouped outputs are masked per group: plain stores, no TMA map
   std::memset(&mc, 0, sizeof(mc));
   // after the gather (when there is one) the GEMM follows a library kernel
-  return cuda_status(tc_grouped_launch(pl.mode, bn, ma, mb, mc, p, grid, s, pdl || g.a_row_index != nullptr));
+  return cuda_status(tc_grouped_launch(pl.mode, bn, ar, ma, mb, mc, p, grid, s, pdl || g.a_row_index != nullptr));
 }
 
 }  // namespace
@@ -980,6 +984,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
   else
     st = cuda_status(route_sort_launch(ids, w, static_cast<int32_t>(T), E, k, off, stok, sw, pos, s, true));
   if (st != KF_OK) return st;
+  // a token's k experts are distinct, so no expert holds more than T rows
   // gate/up: h = silu(Xg W_gate[e]^T) * (Xg W_up[e]^T), rows gathered by token
   {
     kf_epilogue_op op{};
@@ -990,6 +995,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     if (st != KF_OK) return st;
     GroupedArgs g{X, H, T, stok, W_gu, H, 2 * I * H, off, E, P, I, H, h, KF_BF16, I};
     GroupExtras ex;
+    ex.max_group_rows = T;
     if (!det) {
       ex.zero_ptr = yacc;
       ex.zero_bytes = T * H * 4;
@@ -1018,6 +1024,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     float* yp = reinterpret_cast<float*>(ws + L.yp);
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yp, KF_F32, H};
     GroupExtras ex;
+    ex.max_group_rows = T;
     if (act) {
       ex.gbias = act->b_down;
       ex.gbias_ld = H;
@@ -1044,6 +1051,7 @@ kf_status moe_ffn_impl(const void* X, const float* logits, const void* W_gu, con
     if (st != KF_OK) return st;
     GroupedArgs g{h, I, P, nullptr, W_down, I, H * I, off, E, P, H, I, yacc, KF_F32, H};
     GroupExtras ex;
+    ex.max_group_rows = T;
     if (act) {
       ex.gbias = act->b_down;
       ex.gbias_ld = H;

@@ -51,7 +51,8 @@ enum ChainSig : int {
 bool tc_dense_has(int mode, int bn, bool cta2);
 bool tc_dense2_has(int mode, int bn);
 bool tc_dense2_has_prog(int mode, int bn, int sig);  // a compiled chain program for (mode, bn, sig)
-bool tc_grouped_has(int mode, int bn);
+// ar: rows of an A ring slot (128, or 64 for groups known to hold at most 64 rows)
+bool tc_grouped_has(int mode, int bn, int ar = 128);
 // fp32 GEMM + element-wise chain as three tf32 tensor-core products (3xTF32)
 struct Tf32Params {
   int32_t M, N, K;
@@ -112,8 +113,8 @@ cudaError_t tc_dense_launch(int mode, int bn, bool cta2, int sig, const CUtensor
 cudaError_t tc_dense2_launch(int mode, int bn, int sig, const CUtensorMap& a, const CUtensorMap& b,
                              const CUtensorMap& c, const CUtensorMap& r, const TcParams& p, int sub_tiles, int grid,
                              cudaStream_t s);
-cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
-                              const TcParams& p, int grid, cudaStream_t s, bool pdl);
+cudaError_t tc_grouped_launch(int mode, int bn, int ar, const CUtensorMap& a, const CUtensorMap& b,
+                              const CUtensorMap& c, const TcParams& p, int grid, cudaStream_t s, bool pdl);
 // GroupNorm over 512-column groups on clusters of two CTA pairs (one 256-column
 // half of the group per pair); units = 256-row x 512-column blocks, the grid is
 // sized inside from the number of co-resident clusters.

@@ -73,7 +73,12 @@ constexpr bool kResTileFor = MODE == kModeStore && !GROUPED && CL == kClPair && 
 template <int MODE, bool GROUPED, int CL, class PRE>
 constexpr int kThreadsFor = 64 + 32 * (kResTileFor<MODE, GROUPED, CL, PRE> ? 12 : kEpiWarps);
 
-template <int BN, int STAGES, int MODE, bool GROUPED, int CL, bool RT = false>
+// AR: rows of an A ring slot.  128 (the MMA's M) except for grouped GEMMs whose
+// groups are known to hold at most AR rows (the MoE at decode): the TMA box
+// then brings AR rows, and the MMA's 128-row read of a slot runs on into the
+// next slot (or, from the last one, into the epilogue buffers that follow the
+// ring) -- those rows feed accumulator rows that are never stored.
+template <int BN, int STAGES, int MODE, bool GROUPED, int CL, bool RT = false, int AR = kBM>
 struct TcCfg {
   static constexpr bool CTA2 = CL != kClOne;  // tcgen05 CTA-pair MMAs
   static constexpr int kEpiW = RT ? 12 : kEpiWarps;  // epilogue warps
@@ -90,7 +95,9 @@ struct TcCfg {
   // With CTA pairs each CTA stages its own 128 rows of A and half of the BN rows of B.
   static constexpr int kBRows = CTA2 ? BN / 2 : BN;
   static constexpr int kBBytes = kBRows * kBK * 2;
-  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kASlot = AR * kBK * 2;
+  static_assert(AR == kBM || (GROUPED && !CTA2 && AR % 8 == 0 && AR < kBM), "short A slots: grouped, single CTA");
+  static constexpr int kStageBytes = kASlot + kBBytes;
   static constexpr uint32_t kTxBytes = (CTA2 ? 2 : 1) * kStageBytes;  // bytes landing per stage on the leader's barrier
   static constexpr int kRowsPerUnit = CTA2 ? 2 * kBM : kBM;
   // accumulator buffer b starts at TMEM column b * kAccStride
@@ -106,11 +113,12 @@ struct TcCfg {
   // residual tile: BN / 32 chunks x 4 row blocks of 32 x 32 bf16 (2 KB, 64-byte
   // swizzle), placed in the A then B regions of two ring slots
   static constexpr int kResTileBytes = 0;
-  static constexpr int kResBlocksA = kABytes / 2048;
-  static constexpr int kResBlocksPerSlot = kABytes / 2048 + kBBytes / 2048;
+  static constexpr int kResBlocksA = kASlot / 2048;
+  static constexpr int kResBlocksPerSlot = kASlot / 2048 + kBBytes / 2048;
   static_assert(!RT || 2 * kResBlocksPerSlot >= (BN / 32) * 4, "residual tile fits two ring slots");
   static_assert(!RT || STAGES >= 3, "residual tile needs two slots beside an operand slot");
   static constexpr int kStagingBytes = kEpiW * kWarpStaging;
+  static_assert(kStagingBytes >= kABytes - kASlot, "the MMA's read past the last short A slot stays in the CTA");
   // GroupNorm: per-warp cache of bias / gamma / beta for 4 chunks of 32 columns
   static constexpr int kGnCacheBytes = (MODE == kModeGroupNorm) ? kEpiW * 3 * 4 * 32 * 4 : 0;
   // flags + row-statistics exchange between the two warps of a quadrant (2 KB)
@@ -133,13 +141,13 @@ struct UnitInfo {
 
 // PRE / POST: compiled op programs (Prog<...>) for the chain before / after the
 // reduction, or Interp for arbitrary chains.
-template <int BN, int STAGES, int MODE, bool GROUPED, int CL, class PRE = Interp, class POST = Interp>
+template <int BN, int STAGES, int MODE, bool GROUPED, int CL, class PRE = Interp, class POST = Interp, int AR = kBM>
 __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     kf_tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmR,
                       const __grid_constant__ TcParams p, const int32_t sub_tiles) {
   constexpr bool RT = kResTileFor<MODE, GROUPED, CL, PRE>;
-  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CL, RT>;
+  using Cfg = TcCfg<BN, STAGES, MODE, GROUPED, CL, RT, AR>;
   constexpr bool CTA2 = Cfg::CTA2;
   constexpr bool QUAD = Cfg::kQuad;
   constexpr bool COUPLE = CL == kClCouple;
@@ -301,7 +309,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
     const int bi = c * 4 + qq;
     const int sl = bi < Cfg::kResBlocksPerSlot ? s0 : s1;
     const int j = bi % Cfg::kResBlocksPerSlot;
-    return j < Cfg::kResBlocksA ? smA + sl * kABytes + j * 2048 : smB + sl * Cfg::kBBytes + (j - Cfg::kResBlocksA) * 2048;
+    return j < Cfg::kResBlocksA ? smA + sl * Cfg::kASlot + j * 2048 : smB + sl * Cfg::kBBytes + (j - Cfg::kResBlocksA) * 2048;
   };
 
   auto decode = [&](int32_t u) -> UnitInfo {
@@ -358,7 +366,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
               ok = false;
               break;
             }
-            uint8_t* a = smA + st * kABytes;
+            uint8_t* a = smA + st * Cfg::kASlot;
             uint8_t* b = smB + st * Cfg::kBBytes;
             if constexpr (CTA2) {
               // both CTAs' copies complete on the leader's full barrier
@@ -452,7 +460,7 @@ __global__ void __launch_bounds__(kThreadsFor<MODE, GROUPED, CL, PRE>, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t a0 = smem_u32(smA + st * kABytes);
+            const uint32_t a0 = smem_u32(smA + st * Cfg::kASlot);
             const uint32_t b0 = smem_u32(smB + st * Cfg::kBBytes);
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {

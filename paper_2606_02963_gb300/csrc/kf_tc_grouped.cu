@@ -6,11 +6,11 @@
 namespace kf {
 namespace {
 
-template <int BN, int STAGES, int MODE>
+template <int BN, int STAGES, int MODE, int AR>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p, int grid, cudaStream_t s,
                        bool pdl) {
-  using Cfg = TcCfg<BN, STAGES, MODE, true, kClOne>;
-  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, kClOne>;
+  using Cfg = TcCfg<BN, STAGES, MODE, true, kClOne, false, AR>;
+  auto kern = kf_tc_gemm_kernel<BN, STAGES, MODE, true, kClOne, Interp, Interp, AR>;
   static std::atomic<bool> configured[64];  // the attribute is per device
   int dev = 0;
   cudaGetDevice(&dev);
@@ -26,29 +26,35 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
 
 }  // namespace
 
-#define KF_GROUPED_VARIANTS(X) \
-  X(kModeSwiglu, 128, 6)       \
-  X(kModeSwiglu, 192, 5)       \
-  X(kModeSwiglu, 256, 4)       \
-  X(kModeScatter, 128, 6)      \
-  X(kModeScatter, 192, 5)      \
-  X(kModeScatter, 256, 4)      \
-  X(kModeStore, 128, 6)        \
-  X(kModeStore, 192, 4)        \
-  X(kModeStore, 256, 4)
+// (mode, BN, stages, rows of an A slot).  The 64-row variants serve groups of
+// at most 64 rows (the MoE at decode): the shared memory an A slot no longer
+// needs holds more stages, i.e. more weight bytes in flight.
+#define KF_GROUPED_VARIANTS(X)  \
+  X(kModeSwiglu, 128, 6, 128)   \
+  X(kModeSwiglu, 192, 5, 128)   \
+  X(kModeSwiglu, 256, 4, 128)   \
+  X(kModeSwiglu, 256, 5, 64)    \
+  X(kModeScatter, 128, 6, 128)  \
+  X(kModeScatter, 192, 5, 128)  \
+  X(kModeScatter, 256, 4, 128)  \
+  X(kModeScatter, 128, 8, 64)   \
+  X(kModeStore, 128, 6, 128)    \
+  X(kModeStore, 192, 4, 128)    \
+  X(kModeStore, 256, 4, 128)    \
+  X(kModeStore, 128, 8, 64)
 
-bool tc_grouped_has(int mode, int bn) {
-#define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return true;
+bool tc_grouped_has(int mode, int bn, int ar) {
+#define X(M_, B_, S_, R_) \
+  if (mode == M_ && bn == B_ && ar == R_) return true;
   KF_GROUPED_VARIANTS(X)
 #undef X
   return false;
 }
 
-cudaError_t tc_grouped_launch(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const TcParams& p,
-                              int grid, cudaStream_t s, bool pdl) {
-#define X(M_, B_, S_) \
-  if (mode == M_ && bn == B_) return launch_one<B_, S_, M_>(a, b, c, p, grid, s, pdl);
+cudaError_t tc_grouped_launch(int mode, int bn, int ar, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                              const TcParams& p, int grid, cudaStream_t s, bool pdl) {
+#define X(M_, B_, S_, R_) \
+  if (mode == M_ && bn == B_ && ar == R_) return launch_one<B_, S_, M_, R_>(a, b, c, p, grid, s, pdl);
   KF_GROUPED_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;
